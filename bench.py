@@ -1,0 +1,380 @@
+"""Benchmark of the WaveFilter hot path on GB300.
+
+One step = one denoising-step layer of the method after the cache exists:
+wf_filter (skim + multi-scale scan, Eq. 7-11) then wf_sparse_attn (final
+step of Algorithm 1) over every (batch, head) of the workload, with the
+Haar pyramid of the prompt keys already built (the paper computes it at the
+initial step; the 32-layer workload "c5" instead refreshes it every 8 steps
+inside the timed loop).
+
+value = algorithmic HBM bytes of the step / device time (GB/s): the bytes
+that must move are the query block, the candidate coefficient rows of every
+scale, the level-0 trim rows, K[mu0] and V[mu0], the generation rows, the
+output block and the index list.  L2 is flushed (256 MiB write) before every
+timed step; each step is timed with CUDA events on the launching stream.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c3]
+                       [--impl reference]
+Under torchrun every rank runs its own replica of the workload (the path
+shards by (batch, head) with no exchange: weak scaling); rank 0 prints one
+JSON line with the max time over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2606_00724_gb300 import synth  # noqa: E402
+
+METRIC = "fused filter+sparse-attn step latency (us) & achieved HBM GB/s vs roofline, 1 GB300"
+DEFAULT_WORKLOAD = "c3"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic bytes (per (batch, head) unit).
+# ---------------------------------------------------------------------------
+def unit_bytes(w: synth.Workload) -> dict:
+    e = 4 if w.dtype == "f32" else 2
+    row = w.head_dim * e
+    L, keep = w.levels, [int(x) for x in w.keep]
+    cands = [w.n >> L] + [2 * keep[b + 1] for b in range(L - 1, 0, -1)]
+    trim = 2 * keep[1] if keep[0] < 2 * keep[1] else 0
+    k = keep[0]
+    q = w.q * row
+    coeff = sum(cands) * row
+    filt = q + coeff + trim * row + 4 * k
+    attn = q + 4 * k + 2 * k * row + 2 * w.ng * row + q
+    step = q + coeff + trim * row + 2 * k * row + 2 * w.ng * row + q + 4 * k
+    dwt = w.n * row + (w.n - (w.n >> L)) * row
+    return {"filter": filt, "attn": attn, "step": step, "dwt": dwt}
+
+
+def launches_per_step(w: synth.Workload, refresh: bool = False) -> int:
+    trim = int(w.keep[0]) < 2 * int(w.keep[1])
+    return 3 * w.levels + 3 * trim + 2 + (1 if refresh else 0)
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region.
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.lines = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.dev}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (baseline / reference arm).
+# ---------------------------------------------------------------------------
+def oracle_units_seconds(w: synth.Workload, cfg: str, budget_s: float, max_units: int | None = None,
+                         start_unit: int = 0):
+    """Time the oracle's filter + sparse attention on consecutive units until
+    the time budget is spent.  Returns (units, seconds)."""
+    import oracle
+    oracle.build()
+    done, spent, u = 0, 0.0, start_unit
+    while True:
+        b, h = divmod(u % w.units, w.heads)
+        unit = synth.make_unit(w, b, h, planted=False, device="cpu", cfg=cfg)
+        dt = synth.storage_dtype(w)
+        Q, K, V, Kg, Vg = (t.to(dt).double().numpy() for t in (unit.Q, unit.K, unit.V, unit.Kg, unit.Vg))
+        pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, w.dtype == "bf16").astype(np.float64)
+        t0 = time.perf_counter()
+        mu0 = oracle.filter(Q, pyr, K, w.n, w.levels, np.array(w.keep))
+        oracle.sparse_attn(Q, K, V, mu0, Kg, Vg)
+        spent += time.perf_counter() - t0
+        done += 1
+        u += 1
+        if spent >= budget_s or (max_units is not None and done >= max_units):
+            return done, spent
+
+
+# ---------------------------------------------------------------------------
+# GPU arm.
+# ---------------------------------------------------------------------------
+def make_inputs(w, cfg, device, rank):
+    if cfg == "c5":
+        return [synth.make_batch_fast(w, layer=l, device=device, seed_salt=rank) for l in range(w.layers)]
+    return [synth.make_batch(w, layer=rank, planted=False, device=device, cfg=cfg)]
+
+
+def run_gpu(args, cfg, rank, world, device):
+    from paper_2606_00724_gb300 import wf
+
+    w = synth.WORKLOADS[cfg]
+    keep = [int(x) for x in w.keep]
+    layers = make_inputs(w, cfg, device, rank)
+    bufs = []
+    for lay in layers:
+        coeffs = torch.empty(wf.wf_coeffs_bytes(lay.K, w.levels), dtype=torch.uint8, device=device)
+        wf.wf_dwt_build(lay.K, w.levels, coeffs)
+        ws = torch.empty(wf.wf_step_workspace_bytes(lay.Q, lay.K, w.levels, keep, w.ng), dtype=torch.uint8,
+                         device=device)
+        bufs.append(dict(coeffs=coeffs, ws=ws, idx=torch.empty(w.units, w.k, dtype=torch.int32, device=device),
+                         O=torch.empty_like(lay.Q)))
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    stream = torch.cuda.current_stream()
+    refresh_every = w.refresh_every
+
+    def step(i):
+        for lay, bf in zip(layers, bufs):
+            refresh = bool(refresh_every) and (i % refresh_every == 0)
+            wf.wf_step(lay.Q, lay.K, lay.V, lay.Kg, lay.Vg, bf["coeffs"], refresh, w.levels, keep, bf["idx"],
+                       bf["O"], bf["ws"], stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+
+    # Pre-roll of the same steps so that the clock samples see the GPU under load.
+    sampler = ClockSampler(device.index if device.index is not None else 0)
+    sampler.start()
+    t_end = time.time() + args.preroll
+    i = 0
+    while time.time() < t_end:
+        flush.zero_()
+        step(i)
+        i += 1
+        if i % 32 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        flush.zero_()
+        evs[i][0].record(stream)
+        step(i)
+        evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop()
+    step_ms = [a.elapsed_time(b) for a, b in evs]
+    total_ms = sum(step_ms)
+
+    # Per-call timing of the two library calls (same flush protocol), for the
+    # dominant-kernel roofline.
+    lay, bf = layers[0], bufs[0]
+    calls = {}
+    for name in ("filter", "attn"):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(max(args.steps, 20))]
+        for a, b in ev:
+            flush.zero_()
+            a.record(stream)
+            if name == "filter":
+                wf.wf_filter(lay.Q, bf["coeffs"], lay.K, w.levels, keep, bf["idx"], bf["ws"], None, stream)
+            else:
+                wf.wf_sparse_attn(lay.Q, lay.K, lay.V, bf["idx"], w.k, lay.Kg, lay.Vg, bf["O"], bf["ws"], 0.0,
+                                  stream)
+            b.record(stream)
+        torch.cuda.synchronize()
+        calls[name] = statistics.mean(a.elapsed_time(b) for a, b in ev)
+
+    # End to end through the public API with host buffers: copy the step's
+    # query block and generation rows in from pinned memory, run the step,
+    # copy O and the indices out.
+    hQ = lay.Q.cpu().pin_memory()
+    hKg = lay.Kg.cpu().pin_memory()
+    hVg = lay.Vg.cpu().pin_memory()
+    hO = torch.empty(lay.Q.shape, dtype=lay.Q.dtype, pin_memory=True)
+    hidx = torch.empty(w.units, w.k, dtype=torch.int32, pin_memory=True)
+    dQ, dKg, dVg = torch.empty_like(lay.Q), torch.empty_like(lay.Kg), torch.empty_like(lay.Vg)
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(max(args.steps, 20))]
+    for a, b in e2e_ev:
+        flush.zero_()
+        a.record(stream)
+        dQ.copy_(hQ, non_blocking=True)
+        dKg.copy_(hKg, non_blocking=True)
+        dVg.copy_(hVg, non_blocking=True)
+        wf.wf_step(dQ, lay.K, lay.V, dKg, dVg, bf["coeffs"], False, w.levels, keep, bf["idx"], bf["O"], bf["ws"],
+                   stream)
+        hO.copy_(bf["O"], non_blocking=True)
+        hidx.copy_(bf["idx"], non_blocking=True)
+        b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
+    h2d = sum(t.numel() * t.element_size() for t in (hQ, hKg, hVg))
+    d2h = hO.numel() * hO.element_size() + hidx.numel() * 4
+    return dict(w=w, total_ms=total_ms, step_ms=step_ms, calls=calls, clocks=clocks, e2e_ms=e2e_ms,
+                h2d=h2d, d2h=d2h, layers=len(layers))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=list(synth.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--preroll", type=float, default=1.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    cfg = args.workload
+    w = synth.WORKLOADS[cfg]
+    ub = unit_bytes(w)
+    hbm_peak, peak_kind = peaks()
+
+    config = {"workload": w.name, "batch": w.batch, "heads": w.heads, "head_dim": w.head_dim,
+              "context": w.n, "query_block": w.q, "generation_rows": w.ng, "levels": w.levels, "k": w.k,
+              "keep": list(w.keep), "layers": w.layers, "storage": w.dtype,
+              "step": "wf_filter + wf_sparse_attn per layer" + (
+                  f"; wf_dwt_build refresh every {w.refresh_every} steps" if w.refresh_every else
+                  "; pyramid built once before timing"),
+              "l2": "flushed before every timed step (256 MiB write)", "parallelism": f"replicas{args.gpus}"}
+    step_bytes = ub["step"] * w.units * w.layers
+    if w.refresh_every:
+        step_bytes += ub["dwt"] * w.units * w.layers / w.refresh_every
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        units, secs = oracle_units_seconds(w, cfg, budget_s=0.0, max_units=1)  # warm-up / build
+        tot_units, tot_s = 0, 0.0
+        for i in range(args.warmup):
+            oracle_units_seconds(w, cfg, budget_s=0.0, max_units=1, start_unit=i)
+        for i in range(args.steps):
+            u, s = oracle_units_seconds(w, cfg, budget_s=0.0, max_units=1, start_unit=args.warmup + i)
+            tot_units += u
+            tot_s += s
+        gbs = tot_units * ub["step"] / tot_s / 1e9
+        line = {"metric": METRIC, "value": gbs, "unit": "GB/s", "impl": "reference", "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot_s / args.steps * 1e3,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic", "config": config,
+                "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                 "sample": f"one (batch, head) unit per step ({tot_units} units), "
+                                           "filter + sparse attention, pyramid precomputed"},
+                "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py: no CUDA device (the GPU arm has no CPU fallback)")
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    from paper_2606_00724_gb300 import build as wf_build
+    wf_build.build()
+
+    r = run_gpu(args, cfg, rank, world, device)
+    total_ms = r["total_ms"]
+    e2e_ms = r["e2e_ms"]
+    if world > 1:
+        t = torch.tensor([total_ms, e2e_ms], device=device, dtype=torch.float64)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms, e2e_ms = float(t[0]), float(t[1])
+    ms_per_step = total_ms / args.steps
+    value = world * step_bytes / (ms_per_step * 1e-3) / 1e9
+
+    # Dominant call and its roofline.
+    calls = r["calls"]
+    dom = max(calls, key=calls.get)
+    dom_bytes = ub[dom] * w.units
+    achieved = dom_bytes / (calls[dom] * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                "traffic": None, "kernel": f"wf_{dom} ({'3 kernels per scale' if dom == 'filter' else '2 kernels'})",
+                "peak_kind": peak_kind, "step_frac": (step_bytes / (ms_per_step * 1e-3) / 1e9) / hbm_peak,
+                "call_ms": calls}
+    e2e_bytes_per_step = ub["step"] * w.units
+    line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "step_us": ms_per_step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": config, "roofline": roofline, "clocks": r["clocks"],
+            "e2e": {"value": world * e2e_bytes_per_step / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+                    "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"], "ms_per_step": e2e_ms,
+                    "layers": 1},
+            "gpu_launches": launches_per_step(w) * w.layers * args.steps + (
+                w.layers * math.ceil(args.steps / w.refresh_every) if w.refresh_every else 0)}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        units, secs = oracle_units_seconds(w, cfg, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": units * ub["step"] / secs / 1e9, "unit": "GB/s", "cores": 1,
+                                "kind": "oracle",
+                                "sample": f"{units} (batch, head) units of the same workload, filter + sparse "
+                                          f"attention ({secs:.1f} s single-threaded fp64, pyramid precomputed)"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

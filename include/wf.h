@@ -1,0 +1,176 @@
+/*
+ * libwf — WaveFilter hot path on GB300 (sm_103a), C ABI.
+ *
+ * WaveFilter (Sections 3.1-3.2, Algorithm 1) replaces the cached attention of
+ * Eq. 3 for one denoising block by four steps, all implemented here as CUDA
+ * kernels:
+ *   1. a multi-level Haar DWT of the cached prompt keys along the token axis
+ *      (Eq. 5, Eq. 6)                                       -> wf_dwt_build
+ *   2. a coarse "skim": perception weights of the query block against the
+ *      scale-B approximation coefficients and their column sums (Eq. 7, 8)
+ *   3. a multi-scale "scan": Top-K of the weights at each scale, mapped to the
+ *      next finer scale (Eq. 9, 10, 11), down to token positions mu^0
+ *                                                            -> wf_filter
+ *   4. attention of the query block over [K[mu^0]; K[I_g]], [V[mu^0]; V[I_g]]
+ *      (Algorithm 1, final step)                             -> wf_sparse_attn
+ * and wf_step runs 1 (optionally) + 2-3 + 4 as one stream-ordered call.
+ *
+ * Conventions shared by every entry point
+ * - A tensor is described by wf_tensor: [batch, heads, seq, head_dim] with
+ *   element strides for the first three axes; the head_dim axis is
+ *   contiguous.  BHSD and BSHD layouts are both expressible.
+ * - Pointers named Q, K, V, Kg, Vg, O, coeffs, idx, level_sets, ws are DEVICE
+ *   pointers owned by the caller; libwf allocates no device memory and keeps
+ *   no state between calls.  Arrays named keep and m are HOST arrays.
+ * - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *   stream).  Every call only enqueues work on that stream and returns; the
+ *   outputs are valid once the stream reaches that point.
+ * - Every argument is checked on the host before anything is launched; a
+ *   failed check returns a negative wf_status and enqueues nothing.  A failed
+ *   launch returns WF_ERR_CUDA.  The library has no device-side waits in the
+ *   kernels declared here, so no call can hang the device.
+ * - Supported: dtype WF_F32 or WF_BF16 (Q, K, V, Kg, Vg, coeffs and O all of
+ *   the same dtype); head_dim 64 or 128; 1 <= query rows <= 64; prompt length
+ *   n a multiple of 2^levels with 1 <= levels <= 10; base pointers and the
+ *   three strides (in bytes) 16-byte aligned.
+ */
+#ifndef WF_H
+#define WF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  WF_OK = 0,
+  WF_ERR_INVALID_ARG = -1, /* NULL pointer where one is required, bad count */
+  WF_ERR_SHAPE = -2,       /* shapes disagree, unsupported head_dim, n % 2^L != 0 */
+  WF_ERR_DTYPE = -3,       /* unknown dtype or mixed dtypes */
+  WF_ERR_ALIGN = -4,       /* pointer or stride not 16-byte aligned */
+  WF_ERR_WORKSPACE = -5,   /* workspace or coefficient buffer too small */
+  WF_ERR_CUDA = -6,        /* a CUDA runtime call or launch failed */
+  WF_ERR_TIMEOUT = -7,     /* a bounded device-side wait gave up */
+  WF_ERR_UNSUPPORTED = -8, /* valid request outside what this build implements */
+  WF_ERR_SCHEDULE = -9     /* kept counts infeasible for the shape */
+} wf_status;
+
+typedef enum { WF_F32 = 0, WF_BF16 = 1 } wf_dtype;
+
+typedef struct {
+  int32_t batch;    /* B */
+  int32_t heads;    /* H */
+  int32_t seq;      /* rows per (batch, head): n for K/V, q for Q/O, n_g for Kg/Vg */
+  int32_t head_dim; /* d */
+  int64_t stride_b; /* elements between consecutive batch entries */
+  int64_t stride_h; /* elements between consecutive heads */
+  int64_t stride_s; /* elements between consecutive rows */
+  int32_t dtype;    /* wf_dtype */
+} wf_tensor;
+
+/* Human-readable name of a status code (static string). */
+const char* wf_status_str(int status);
+
+/* ---------------------------------------------------------------------------
+ * 1. DWT pyramid (Eq. 5 recursion of Section 2.2; Eq. 6 keys only).
+ *
+ * For every (batch b, head h) the level cascade a_0 = K[b,h],
+ *   a_l[j] = (a_{l-1}[2j] + a_{l-1}[2j+1]) * (1/sqrt 2),   l = 1..levels,
+ * is evaluated in fp32 (one fp32 add, one fp32 multiply by fl32(1/sqrt 2),
+ * no fused multiply-add) and each a_l row is stored rounded to the key dtype
+ * (bf16: round to nearest even).  Coefficient j of level l pairs tokens
+ * [2^l j, 2^l (j+1)) (the blocks of Eq. 10); the taps are the orthonormal Haar
+ * pair of Table 3.  Detail coefficients are not stored: filtering only reads
+ * approximations.
+ *
+ * coeffs layout (contiguous, dtype of K): unit u = b*H + h owns
+ * R = n - n/2^levels rows of head_dim elements starting at row u*R; inside it
+ * level l starts at row n - n/2^(l-1) and has n/2^l rows.
+ *
+ * V must be NULL: Section 3.1 decomposes the cache keys only.
+ * Errors: WF_ERR_WORKSPACE if coeffs_bytes < wf_coeffs_bytes(kv, levels).
+ * ------------------------------------------------------------------------- */
+size_t wf_coeffs_bytes(const wf_tensor* kv, int levels); /* 0 if invalid */
+wf_status wf_dwt_build(const void* K, const void* V, const wf_tensor* kv, int levels, void* coeffs,
+                       size_t coeffs_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Kept counts (Eq. 9 "proportion m_B").  keep has levels+1 entries: keep[l]
+ * = number of level-l coefficients kept (l = 1..levels), keep[0] = final
+ * number of prompt tokens k.  Feasible iff 1 <= keep[L] <= n/2^L,
+ * 1 <= keep[l] <= 2 keep[l+1], 1 <= keep[0] <= 2 keep[1].
+ *
+ * wf_default_schedule: one proportion m = (k/n)^(1/L) for every scale:
+ *   keep[l] = min(|C_l|, max(1, ceil(m |C_l|))) for l = L..2 with
+ *   |C_L| = n/2^L, |C_{l-1}| = 2 keep[l]; keep[1] = ceil(k/2); keep[0] = k.
+ * wf_schedule_from_proportions: per-scale proportions m[l] in (0, 1]
+ *   (m[0] unused): keep[l] = min(|C_l|, max(1, ceil(m[l] |C_l|))),
+ *   keep[0] = 2 keep[1].
+ * "ceil" ignores a product that exceeds an integer by less than 1e-9.
+ * Host-only; return WF_ERR_SCHEDULE if no feasible schedule exists.
+ * ------------------------------------------------------------------------- */
+wf_status wf_default_schedule(int64_t n, int levels, int64_t k, int32_t* keep);
+wf_status wf_schedule_from_proportions(int64_t n, int levels, const double* m, int32_t* keep);
+
+/* ---------------------------------------------------------------------------
+ * 2-3. Skim and scan (Eq. 7-11, Algorithm 1 inner loop).
+ *
+ * For every unit, with C_L = {0..n/2^L - 1} and for l = L..1:
+ *   logits  s_ij = Q_i . A_l[j] / sqrt(d)           (j in C_l; fp32)
+ *   P       = softmax over j in C_l of each query row (Eq. 7)
+ *   W_j     = sum_i P_ij                            (Eq. 8)
+ *   J_l     = the keep[l] candidates of largest W (ties: lower index)  (Eq. 9)
+ *   C_{l-1} = {2j, 2j+1 : j in J_l}                 (Eq. 10-11)
+ * C_0 holds 2 keep[1] token positions; if keep[0] < 2 keep[1] the same
+ * scoring on the raw keys K[C_0] keeps the top keep[0] of them.
+ *
+ * Inputs: Q [B,H,q,d] (descriptor q), coeffs from wf_dwt_build on K with the
+ * same levels, K [B,H,n,d] (descriptor kv; read only by the level-0 trim).
+ * keep: host array of levels+1 counts (e.g. from wf_default_schedule).
+ * Outputs: idx int32 [B*H][keep[0]] token positions, ascending per unit.
+ * level_sets (optional, NULL to skip): int32
+ * [B*H][keep[L] + .. + keep[1] + keep[0]] = J_L, .., J_1, mu^0 per unit.
+ * ws: device scratch of at least wf_filter_workspace_bytes() bytes,
+ * 256-byte aligned; its contents on entry do not matter.
+ * ------------------------------------------------------------------------- */
+size_t wf_filter_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep);
+wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const void* K, const wf_tensor* kv,
+                    int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets, void* ws,
+                    size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * 4. Sparse attention (Algorithm 1, final step; Eq. 3 form).
+ *
+ * For every unit: K_s = [K[idx[0..k)]; Kg], V_s = [V[idx[0..k)]; Vg] and
+ *   O = softmax(Q K_s^T * scale) V_s      (fp32 logits, softmax, accumulation)
+ * with scale = 1/sqrt(d) when the argument is 0.  No mask (the DLMs attend
+ * bidirectionally).  idx: int32 [B*H][k], each entry in [0, n) (any order).
+ * Kg, Vg: [B,H,n_g,d] (descriptor g, may be NULL when n_g = 0).  O: [B,H,q,d]
+ * (descriptor o: same shape and dtype as Q), written rounded to that dtype.
+ * ws: device scratch of at least wf_attn_workspace_bytes() bytes.
+ * Out-of-range idx entries are clamped to [0, n) (never read out of bounds).
+ * ------------------------------------------------------------------------- */
+size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g);
+wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const void* V, const wf_tensor* kv,
+                         const int32_t* idx, int k, const void* Kg, const void* Vg, const wf_tensor* g, void* O,
+                         const wf_tensor* o, float scale, void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * One denoising-step layer (Algorithm 1 body): if refresh_coeffs != 0, first
+ * rebuild coeffs from K (wf_dwt_build); then wf_filter; then wf_sparse_attn
+ * with scale 1/sqrt(d), writing idx and O.  Same arguments and rules as the
+ * three calls; ws must hold wf_step_workspace_bytes().
+ * ------------------------------------------------------------------------- */
+size_t wf_step_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
+                               int n_g);
+wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const void* V, const wf_tensor* kv,
+                  const void* Kg, const void* Vg, const wf_tensor* g, void* coeffs, size_t coeffs_bytes,
+                  int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, void* O,
+                  const wf_tensor* o, void* ws, size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* WF_H */

@@ -1,0 +1,234 @@
+// libwf C ABI: argument checks, workspace planning and stream-ordered
+// launches.  Nothing here allocates device memory or synchronises the stream.
+#include <math.h>
+#include <string.h>
+
+#include "wf_internal.cuh"
+
+#define WF_API extern "C" __attribute__((visibility("default")))
+
+namespace {
+
+using wf::align_up;
+
+int elem_size(int dtype) { return dtype == WF_BF16 ? 2 : 4; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Shape, dtype and alignment of one descriptor (seq may be 0 when allow_empty).
+wf_status check_desc(const wf_tensor* t, bool allow_empty) {
+  if (!t) return WF_ERR_INVALID_ARG;
+  if (t->dtype != WF_F32 && t->dtype != WF_BF16) return WF_ERR_DTYPE;
+  if (t->batch < 1 || t->heads < 1 || t->seq < (allow_empty ? 0 : 1)) return WF_ERR_SHAPE;
+  if (t->head_dim != 64 && t->head_dim != 128) return WF_ERR_SHAPE;
+  if (t->stride_b < 0 || t->stride_h < 0 || t->stride_s < 0) return WF_ERR_SHAPE;
+  const int64_t es = elem_size(t->dtype);
+  if ((t->stride_b * es) % 16 || (t->stride_h * es) % 16 || (t->stride_s * es) % 16) return WF_ERR_ALIGN;
+  if (t->seq > 1 && t->stride_s < t->head_dim) return WF_ERR_SHAPE;
+  return WF_OK;
+}
+
+bool same_units(const wf_tensor* a, const wf_tensor* b) {
+  return a->batch == b->batch && a->heads == b->heads && a->head_dim == b->head_dim;
+}
+
+wf_status check_levels(const wf_tensor* kv, int levels) {
+  if (levels < 1 || levels > 10) return WF_ERR_UNSUPPORTED;
+  const int64_t n = kv->seq;
+  if ((n >> levels) < 1 || ((n >> levels) << levels) != n) return WF_ERR_SHAPE;
+  return WF_OK;
+}
+
+wf_status check_keep(int64_t n, int levels, const int32_t* keep) {
+  if (!keep) return WF_ERR_INVALID_ARG;
+  int64_t cnt = n >> levels;
+  for (int l = levels; l >= 1; --l) {
+    if (keep[l] < 1 || keep[l] > cnt) return WF_ERR_SCHEDULE;
+    cnt = 2 * (int64_t)keep[l];
+  }
+  if (keep[0] < 1 || keep[0] > cnt) return WF_ERR_SCHEDULE;
+  return WF_OK;
+}
+
+wf_status cuda_status(cudaError_t e) { return e == cudaSuccess ? WF_OK : WF_ERR_CUDA; }
+
+int64_t ceil_guarded(double v) { return (int64_t)ceil(v - 1e-9); }
+
+wf_status check_filter_args(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep) {
+  wf_status st;
+  if ((st = check_desc(q, false)) != WF_OK) return st;
+  if ((st = check_desc(kv, false)) != WF_OK) return st;
+  if (!same_units(q, kv)) return WF_ERR_SHAPE;
+  if (q->dtype != kv->dtype) return WF_ERR_DTYPE;
+  if (q->seq > wf::kMaxQ) return WF_ERR_UNSUPPORTED;
+  if ((st = check_levels(kv, levels)) != WF_OK) return st;
+  return check_keep(kv->seq, levels, keep);
+}
+
+wf_status check_attn_args(const wf_tensor* q, const wf_tensor* kv, int k, const wf_tensor* g, int n_g,
+                          const wf_tensor* o) {
+  wf_status st;
+  if ((st = check_desc(q, false)) != WF_OK) return st;
+  if ((st = check_desc(kv, false)) != WF_OK) return st;
+  if ((st = check_desc(o, false)) != WF_OK) return st;
+  if (!same_units(q, kv) || !same_units(q, o) || o->seq != q->seq) return WF_ERR_SHAPE;
+  if (q->dtype != kv->dtype || o->dtype != q->dtype) return WF_ERR_DTYPE;
+  if (q->seq > wf::kMaxQ) return WF_ERR_UNSUPPORTED;
+  if (k < 1 || k > kv->seq || n_g < 0) return WF_ERR_INVALID_ARG;
+  if (n_g > 0) {
+    if ((st = check_desc(g, true)) != WF_OK) return st;
+    if (!same_units(q, g) || g->seq != n_g) return WF_ERR_SHAPE;
+    if (g->dtype != q->dtype) return WF_ERR_DTYPE;
+  }
+  return WF_OK;
+}
+
+}  // namespace
+
+WF_API const char* wf_status_str(int status) {
+  switch (status) {
+    case WF_OK: return "WF_OK";
+    case WF_ERR_INVALID_ARG: return "WF_ERR_INVALID_ARG: missing pointer or bad count";
+    case WF_ERR_SHAPE: return "WF_ERR_SHAPE: shapes disagree or are unsupported";
+    case WF_ERR_DTYPE: return "WF_ERR_DTYPE: unknown or mixed dtypes";
+    case WF_ERR_ALIGN: return "WF_ERR_ALIGN: pointer or stride not 16-byte aligned";
+    case WF_ERR_WORKSPACE: return "WF_ERR_WORKSPACE: buffer too small";
+    case WF_ERR_CUDA: return "WF_ERR_CUDA: CUDA runtime or launch failure";
+    case WF_ERR_TIMEOUT: return "WF_ERR_TIMEOUT: a bounded device wait gave up";
+    case WF_ERR_UNSUPPORTED: return "WF_ERR_UNSUPPORTED: outside what this build implements";
+    case WF_ERR_SCHEDULE: return "WF_ERR_SCHEDULE: kept counts infeasible";
+    default: return "unknown wf_status";
+  }
+}
+
+WF_API size_t wf_coeffs_bytes(const wf_tensor* kv, int levels) {
+  if (check_desc(kv, false) != WF_OK || check_levels(kv, levels) != WF_OK) return 0;
+  const int64_t rows = (int64_t)kv->seq - ((int64_t)kv->seq >> levels);
+  return (size_t)kv->batch * kv->heads * rows * kv->head_dim * elem_size(kv->dtype);
+}
+
+WF_API wf_status wf_dwt_build(const void* K, const void* V, const wf_tensor* kv, int levels, void* coeffs,
+                              size_t coeffs_bytes, void* stream) {
+  wf_status st;
+  if ((st = check_desc(kv, false)) != WF_OK) return st;
+  if ((st = check_levels(kv, levels)) != WF_OK) return st;
+  if (!K || !coeffs || V) return WF_ERR_INVALID_ARG;
+  if (!aligned16(K) || !aligned16(coeffs)) return WF_ERR_ALIGN;
+  if (coeffs_bytes < wf_coeffs_bytes(kv, levels)) return WF_ERR_WORKSPACE;
+  return cuda_status(wf::launch_dwt(K, *kv, levels, coeffs, static_cast<cudaStream_t>(stream)));
+}
+
+WF_API wf_status wf_default_schedule(int64_t n, int levels, int64_t k, int32_t* keep) {
+  if (!keep || levels < 1 || levels > 30 || n < 1 || k < 1 || k > n) return WF_ERR_INVALID_ARG;
+  if ((n >> levels) < 1 || ((n >> levels) << levels) != n) return WF_ERR_SHAPE;
+  const double m = pow((double)k / (double)n, 1.0 / levels);
+  int64_t cnt = n >> levels;
+  for (int l = levels; l >= 2; --l) {
+    int64_t kb = ceil_guarded(m * (double)cnt);
+    kb = kb < 1 ? 1 : (kb > cnt ? cnt : kb);
+    keep[l] = (int32_t)kb;
+    cnt = 2 * kb;
+  }
+  const int64_t k1 = (k + 1) / 2;
+  if (k1 > cnt) return WF_ERR_SCHEDULE;
+  keep[1] = (int32_t)k1;
+  keep[0] = (int32_t)k;
+  return WF_OK;
+}
+
+WF_API wf_status wf_schedule_from_proportions(int64_t n, int levels, const double* m, int32_t* keep) {
+  if (!keep || !m || levels < 1 || levels > 30 || n < 1) return WF_ERR_INVALID_ARG;
+  if ((n >> levels) < 1 || ((n >> levels) << levels) != n) return WF_ERR_SHAPE;
+  int64_t cnt = n >> levels;
+  for (int l = levels; l >= 1; --l) {
+    if (!(m[l] > 0.0 && m[l] <= 1.0)) return WF_ERR_SCHEDULE;
+    int64_t kb = ceil_guarded(m[l] * (double)cnt);
+    kb = kb < 1 ? 1 : (kb > cnt ? cnt : kb);
+    keep[l] = (int32_t)kb;
+    cnt = 2 * kb;
+  }
+  keep[0] = 2 * keep[1];
+  return WF_OK;
+}
+
+WF_API size_t wf_filter_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep) {
+  if (check_filter_args(q, kv, levels, keep) != WF_OK) return 0;
+  return wf::plan_filter(*q, *kv, levels, keep).total;
+}
+
+WF_API wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const void* K,
+                           const wf_tensor* kv, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
+                           void* ws, size_t ws_bytes, void* stream) {
+  wf_status st = check_filter_args(q, kv, levels, keep);
+  if (st != WF_OK) return st;
+  if (!Q || !coeffs || !K || !idx || !ws) return WF_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(coeffs) || !aligned16(K)) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(idx) & 3u) != 0 || (reinterpret_cast<uintptr_t>(level_sets) & 3u) != 0)
+    return WF_ERR_ALIGN;
+  const wf::FilterPlan p = wf::plan_filter(*q, *kv, levels, keep);
+  if (ws_bytes < p.total) return WF_ERR_WORKSPACE;
+  return cuda_status(wf::launch_filter(p, Q, *q, coeffs, K, *kv, idx, level_sets, ws,
+                                       static_cast<cudaStream_t>(stream)));
+}
+
+WF_API size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g) {
+  if (check_desc(q, false) != WF_OK || k < 1 || n_g < 0 || q->seq > wf::kMaxQ) return 0;
+  return wf::plan_attn(*q, k, n_g).total;
+}
+
+WF_API wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const void* V,
+                                const wf_tensor* kv, const int32_t* idx, int k, const void* Kg, const void* Vg,
+                                const wf_tensor* g, void* O, const wf_tensor* o, float scale, void* ws,
+                                size_t ws_bytes, void* stream) {
+  const int n_g = g ? g->seq : 0;
+  wf_status st = check_attn_args(q, kv, k, g, n_g, o);
+  if (st != WF_OK) return st;
+  if (!Q || !K || !V || !idx || !O || !ws) return WF_ERR_INVALID_ARG;
+  if (n_g > 0 && (!Kg || !Vg)) return WF_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O)) return WF_ERR_ALIGN;
+  if (n_g > 0 && (!aligned16(Kg) || !aligned16(Vg))) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || (reinterpret_cast<uintptr_t>(idx) & 3u) != 0)
+    return WF_ERR_ALIGN;
+  if (!(scale >= 0.f) || isinf(scale)) return WF_ERR_INVALID_ARG;
+  const wf::AttnPlan p = wf::plan_attn(*q, k, n_g);
+  if (ws_bytes < p.total) return WF_ERR_WORKSPACE;
+  const float sc = scale == 0.f ? 1.0f / sqrtf((float)q->head_dim) : scale;
+  return cuda_status(wf::launch_attn(p, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, ws,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+WF_API size_t wf_step_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
+                                      int n_g) {
+  if (check_filter_args(q, kv, levels, keep) != WF_OK || n_g < 0) return 0;
+  const size_t f = wf::plan_filter(*q, *kv, levels, keep).total;
+  const size_t a = wf::plan_attn(*q, keep[0], n_g).total;
+  return f > a ? f : a;
+}
+
+WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const void* V, const wf_tensor* kv,
+                         const void* Kg, const void* Vg, const wf_tensor* g, void* coeffs, size_t coeffs_bytes,
+                         int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, void* O,
+                         const wf_tensor* o, void* ws, size_t ws_bytes, void* stream) {
+  wf_status st = check_filter_args(q, kv, levels, keep);
+  if (st != WF_OK) return st;
+  const int n_g = g ? g->seq : 0;
+  if ((st = check_attn_args(q, kv, keep[0], g, n_g, o)) != WF_OK) return st;
+  if (!Q || !K || !V || !coeffs || !idx || !O || !ws) return WF_ERR_INVALID_ARG;
+  if (n_g > 0 && (!Kg || !Vg)) return WF_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(coeffs)) return WF_ERR_ALIGN;
+  if (n_g > 0 && (!aligned16(Kg) || !aligned16(Vg))) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || (reinterpret_cast<uintptr_t>(idx) & 3u) != 0)
+    return WF_ERR_ALIGN;
+  if (coeffs_bytes < wf_coeffs_bytes(kv, levels)) return WF_ERR_WORKSPACE;
+  if (ws_bytes < wf_step_workspace_bytes(q, kv, levels, keep, n_g)) return WF_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (refresh_coeffs && (e = wf::launch_dwt(K, *kv, levels, coeffs, s)) != cudaSuccess) return WF_ERR_CUDA;
+  const wf::FilterPlan fp = wf::plan_filter(*q, *kv, levels, keep);
+  if ((e = wf::launch_filter(fp, Q, *q, coeffs, K, *kv, idx, nullptr, ws, s)) != cudaSuccess) return WF_ERR_CUDA;
+  const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g);
+  const float sc = 1.0f / sqrtf((float)q->head_dim);
+  e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, ws, s);
+  return cuda_status(e);
+}

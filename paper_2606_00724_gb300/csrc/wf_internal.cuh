@@ -1,0 +1,96 @@
+// Internal declarations shared by the libwf translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "wf.h"
+
+namespace wf {
+
+typedef __nv_bfloat16 bf16;
+
+// Elements per 16-byte vector.
+template <typename T> struct Vec;
+template <> struct Vec<float> { static constexpr int N = 4; };
+template <> struct Vec<bf16> { static constexpr int N = 8; };
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Load one 16-byte vector of T and widen it to fp32 (exact).
+__device__ __forceinline__ void ld_vec(const float* p, float* o) {
+  float4 v = __ldg(reinterpret_cast<const float4*>(p));
+  o[0] = v.x; o[1] = v.y; o[2] = v.z; o[3] = v.w;
+}
+__device__ __forceinline__ void ld_vec(const bf16* p, float* o) {
+  uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
+  o[0] = bf16_lo(v.x); o[1] = bf16_hi(v.x); o[2] = bf16_lo(v.y); o[3] = bf16_hi(v.y);
+  o[4] = bf16_lo(v.z); o[5] = bf16_hi(v.z); o[6] = bf16_lo(v.w); o[7] = bf16_hi(v.w);
+}
+
+// Round fp32 to the storage type (bf16: round to nearest even) and store 16 bytes.
+__device__ __forceinline__ void st_vec(float* p, const float* v) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);  // .x = a (low half), .y = b
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ void st_vec(bf16* p, const float* v) {
+  uint4 w;
+  w.x = pack_bf16(v[0], v[1]); w.y = pack_bf16(v[2], v[3]);
+  w.z = pack_bf16(v[4], v[5]); w.w = pack_bf16(v[6], v[7]);
+  *reinterpret_cast<uint4*>(p) = w;
+}
+
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(bf16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ void from_f32(float& d, float x) { d = x; }
+__device__ __forceinline__ void from_f32(bf16& d, float x) { d = __float2bfloat16_rn(x); }
+
+// A [B, H, rows, d] row source: element (b, h, r, c) at
+// base + b*sb + h*sh + off + r*ss + c.
+struct RowSrc {
+  const void* base;
+  int64_t sb, sh, ss, off;
+};
+
+// ---------------------------------------------------------------------------
+// Launchers (each returns cudaSuccess or the launch error).
+// ---------------------------------------------------------------------------
+
+// DWT pyramid of the keys: see wf_dwt_build.
+cudaError_t launch_dwt(const void* K, const wf_tensor& kv, int levels, void* coeffs, cudaStream_t s);
+
+// Filter workspace plan for one call.
+struct FilterPlan {
+  int U, H, q, d, n, L, dtype;
+  int32_t keep[16];
+  int cmax;        // largest candidate count over the scales (and the trim)
+  int tiles_max;   // ceil(cmax / kScoreTile)
+  bool trim;
+  size_t off_cand_a, off_cand_b, off_w, off_logits, off_part, total;
+};
+constexpr int kScoreTile = 32;
+constexpr int kMaxQ = 64;
+FilterPlan plan_filter(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep);
+cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* coeffs,
+                          const void* K, const wf_tensor& kv, int32_t* idx, int32_t* level_sets, void* ws,
+                          cudaStream_t s);
+
+// Sparse attention workspace plan.
+struct AttnPlan {
+  int U, H, q, d, k, ng, nsplit, dtype;
+  size_t off_o, off_ml, total;
+};
+constexpr int kAttnChunk = 64;
+AttnPlan plan_attn(const wf_tensor& q, int k, int ng);
+cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
+                        const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
+                        const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s);
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace wf
