@@ -4,10 +4,11 @@
 //             candidates (gathered by index), plus the tile's per-query
 //             softmax partials (max, sum of exp).
 //   weights : the global per-query max / normaliser from the tile partials,
-//             then W_j = sum_i exp(s_ij - M_i) / S_i for 256 candidates.
-//   select  : one CTA per unit; radix select of the keep[l]-th largest W
+//             then the ranking key log W_j, W_j = sum_i exp(s_ij - M_i) / S_i,
+//             for 256 candidates.
+//   select  : one CTA per unit; radix select of the keep[l]-th largest key
 //             (four 8-bit passes over the fp32 bit patterns), then an
-//             order-preserving compaction: every W above the threshold plus
+//             order-preserving compaction: every key above the threshold plus
 //             the lowest-index ties, emitted in candidate (= index) order and
 //             expanded to the children {2c, 2c+1} of Eq. 10.
 // fp32 arithmetic throughout, exact fp32 exp (expf).
@@ -105,7 +106,12 @@ __global__ void __launch_bounds__(256) weights_kernel(const float* __restrict__ 
                                                       int64_t lg_row, const float2* __restrict__ part,
                                                       int64_t part_unit, int ntiles, int q, int m,
                                                       float* __restrict__ W, int64_t w_unit) {
-  __shared__ float Ms[QMAX], Is[QMAX];
+  // Per query row i: M_i = max_j s_ij and log S_i = log sum_j exp(s_ij - M_i),
+  // combined from the tile partials.  Then the ranking key of candidate j is
+  // log W_j = log sum_i exp(s_ij - M_i - log S_i), evaluated as a
+  // log-sum-exp over the query rows: the same order as W_j, without the
+  // underflow that would turn very small weights into ties.
+  __shared__ float Ms[QMAX];
   const int u = blockIdx.y;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float2* pt = part + (int64_t)u * part_unit;
@@ -121,15 +127,26 @@ __global__ void __launch_bounds__(256) weights_kernel(const float* __restrict__ 
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
-    if (lane == 0) { Ms[i] = mx; Is[i] = 1.f / z; }
+    if (lane == 0) Ms[i] = mx + logf(z);
   }
   __syncthreads();
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= m) return;
-  const float* lg = logits + (int64_t)u * lg_unit;
-  float w = 0.f;
-  for (int i = 0; i < q; ++i) w += expf(lg[(int64_t)i * lg_row + j] - Ms[i]) * Is[i];
-  W[(int64_t)u * w_unit + j] = w;
+  const float* lg = logits + (int64_t)u * lg_unit + j;
+  float t[QMAX];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < QMAX; ++i) {
+    if (i < q) {
+      t[i] = lg[(int64_t)i * lg_row] - Ms[i];
+      mx = fmaxf(mx, t[i]);
+    }
+  }
+  float z = 0.f;
+#pragma unroll
+  for (int i = 0; i < QMAX; ++i)
+    if (i < q) z += expf(t[i] - mx);
+  W[(int64_t)u * w_unit + j] = mx + logf(z);
 }
 
 __device__ __forceinline__ uint32_t order_key(float f) {

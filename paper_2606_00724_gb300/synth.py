@@ -187,13 +187,19 @@ def _plant(w: Workload, g: torch.Generator, dev, Q, K, Kg, needles) -> dict:
     """Planted ladder: pick target sets top-down and lift them along u.
 
     Every query's component along a random unit direction u is set to
-    PLANT_C.  For each scale b = L..1, keep[b] blocks are chosen among the
-    children of the previous choice (blocks holding needles first, the rest
-    at random) and every token of a chosen scale-b block gets
-    beta_b = PLANT_GAP sqrt(d) / (PLANT_C 2^(b/2)) along u, which lifts the
-    block's scale-b logit by G_b = PLANT_GAP * gap_growth^b for every query.  An optional level-0
-    trim chooses keep[0] tokens the same way.  The generation rows get the
-    whole bonus so they stay competitive in the final attention.
+    PLANT_C.  Scale L: keep[L] blocks are chosen (blocks holding needles
+    first, the rest at random) and each token of a chosen block gets
+    +beta_L along u.  Finer scales b = L-1..1 and the optional level-0 trim:
+    the candidates are the two children of every block chosen one scale up;
+    keep[b] of them are chosen, needle blocks first, then at most one child
+    per parent while the count allows.  A chosen child gets +beta_b and, when
+    its sibling is not chosen, the sibling gets -beta_b, so the parent's
+    coefficient (the sum of its children) is unchanged and the bonuses of
+    finer scales do not leak into coarser ones.  beta_b = G_b sqrt(d) /
+    (PLANT_C 2^(b/2)) lifts a scale-b coefficient's logit by
+    G_b = PLANT_GAP * gap_growth^b for every query.  The generation rows get
+    the whole bonus of a chosen token so they stay competitive in the final
+    attention.
     """
     d, n, L = w.head_dim, w.n, w.levels
     keep = [int(x) for x in w.keep]
@@ -212,18 +218,38 @@ def _plant(w: Workload, g: torch.Generator, dev, Q, K, Kg, needles) -> dict:
             break
         kb = keep[b]
         forced = torch.unique(needles >> b) if needles.numel() else needles
-        if forced.numel() > kb:
-            raise ValueError(f"{w.name}: {forced.numel()} needle blocks exceed keep[{b}]={kb}")
         is_forced = torch.isin(cand, forced)
-        rest = cand[~is_forced]
-        pick = rest[torch.randperm(rest.numel(), generator=g, device=dev)[: kb - int(is_forced.sum())]]
-        chosen = torch.cat([cand[is_forced], pick]).sort().values
+        nf = int(is_forced.sum())
+        if nf > kb:
+            raise ValueError(f"{w.name}: {nf} needle blocks exceed keep[{b}]={kb}")
+        chosen_mask = is_forced.clone()
+        if b == L:
+            rest = torch.nonzero(~is_forced).reshape(-1)
+            chosen_mask[rest[torch.randperm(rest.numel(), generator=g, device=dev)[: kb - nf]]] = True
+        else:
+            cm = chosen_mask.view(-1, 2)
+            free = torch.nonzero(~cm.any(dim=1)).reshape(-1)
+            free = free[torch.randperm(free.numel(), generator=g, device=dev)]
+            first = free[: kb - nf]
+            side = torch.randint(0, 2, (first.numel(),), generator=g, device=dev)
+            cm[first, side] = True
+            extra = kb - nf - first.numel()
+            if extra > 0:
+                rest = torch.nonzero(~chosen_mask).reshape(-1)
+                chosen_mask[rest[torch.randperm(rest.numel(), generator=g, device=dev)[:extra]]] = True
+        chosen = cand[chosen_mask]
         targets[b] = chosen
         gap = PLANT_GAP * w.extra.get("gap_growth", 1.0) ** b
         beta = gap * math.sqrt(d) / (PLANT_C * 2.0 ** (b / 2.0))
         total += beta
-        tok = (chosen[:, None] << b) + torch.arange(1 << b, device=dev)[None, :]
-        bonus[tok.reshape(-1)] += beta
+        val = torch.zeros(cand.numel(), dtype=torch.float64, device=dev)
+        val[chosen_mask] = beta
+        if b < L:
+            cm = chosen_mask.view(-1, 2)
+            lone = (cm.sum(dim=1) == 1)[:, None] & ~cm
+            val.view(-1, 2)[lone] = -beta
+        tok = (cand[:, None] << b) + torch.arange(1 << b, device=dev)[None, :]
+        bonus[tok.reshape(-1)] += val[:, None].expand(-1, 1 << b).reshape(-1)
         cand = torch.stack([2 * chosen, 2 * chosen + 1], dim=1).reshape(-1)
     K += (bonus[:, None] * u[None, :]).to(torch.float32)
     Kg += (total * u)[None, :].to(torch.float32)
