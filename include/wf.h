@@ -158,6 +158,35 @@ wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const
                          const wf_tensor* o, float scale, void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * 4'. Sparse attention without a caller workspace.  The paper has no
+ * counterpart to this call: it exists for callers that cannot allocate device
+ * memory (for example a plugin inside a host engine that owns every device
+ * allocation and offers no scratch, or code on a path where allocating after
+ * start-up is not allowed) and therefore cannot pass the ws buffer that
+ * wf_sparse_attn needs.
+ *
+ * Same arguments, semantics and results as wf_sparse_attn, minus ws and
+ * ws_bytes.  The split-K scratch comes from one static device array of
+ * WF_NOALLOC_SCRATCH_BYTES inside libwf, reserved on every device that loads
+ * it until the process exits; the call allocates nothing.
+ * - Limit: returns WF_ERR_WORKSPACE, and launches nothing, when the call would
+ *   need more than WF_NOALLOC_SCRATCH_BYTES (the need is
+ *   wf_attn_workspace_bytes(q, k, n_g); e.g. 32 heads with k + n_g <= 960
+ *   rows with head_dim 128 fits).
+ * - The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture.  It returns WF_ERR_CUDA if the lookup fails.
+ * - All calls on a device share the one array and each call overwrites it:
+ *   calls whose kernels may overlap on the GPU (other streams, other host
+ *   threads) race and corrupt each other's results.  Serialise them, e.g.
+ *   on one stream.  No part of the array has to start at zero.
+ * ------------------------------------------------------------------------- */
+#define WF_NOALLOC_SCRATCH_BYTES (16u << 20)
+wf_status wf_sparse_attn_noalloc(const void* Q, const wf_tensor* q, const void* K, const void* V,
+                                 const wf_tensor* kv, const int32_t* idx, int k, const void* Kg, const void* Vg,
+                                 const wf_tensor* g, void* O, const wf_tensor* o, float scale, void* stream);
+
+/* ---------------------------------------------------------------------------
  * One denoising-step layer (Algorithm 1 body): if refresh_coeffs != 0, first
  * rebuild coeffs from K (wf_dwt_build); then wf_filter; then wf_sparse_attn
  * with scale 1/sqrt(d), writing idx and O.  Same arguments and rules as the
