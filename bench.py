@@ -1,11 +1,12 @@
 """Benchmark of the WaveFilter hot path on GB300.
 
 One step = one denoising-step layer of the method after the cache exists:
-wf_filter (skim + multi-scale scan, Eq. 7-11) then wf_sparse_attn (final
-step of Algorithm 1) over every (batch, head) of the workload, with the
-Haar pyramid of the prompt keys already built (the paper computes it at the
-initial step; the 32-layer workload "c5" instead refreshes it every 8 steps
-inside the timed loop).
+wf_step, i.e. the skim + multi-scale scan filter (Eq. 7-11) and the sparse
+attention (final step of Algorithm 1) over every (batch, head) of the
+workload, with the Haar pyramid of the prompt keys already built (the paper
+computes it at the initial step; the 32-layer workload "c5" instead
+refreshes it every 8 steps inside the timed loop).  For bf16 / head_dim 128
+that is one fused kernel launch per layer.
 
 value = algorithmic HBM bytes of the step / device time (GB/s): the bytes
 that must move are the query block, the candidate coefficient rows of every
@@ -70,9 +71,16 @@ def unit_bytes(w: synth.Workload) -> dict:
     return {"filter": filt, "attn": attn, "step": step, "dwt": dwt}
 
 
-def launches_per_step(w: synth.Workload, refresh: bool = False) -> int:
+def fused_eligible(w: synth.Workload) -> bool:
+    """wf_step runs its single fused kernel for bf16, head_dim 128, <= 32 query rows."""
+    return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32
+
+
+def launches_per_step(w: synth.Workload) -> int:
+    if fused_eligible(w):
+        return 1
     trim = int(w.keep[0]) < 2 * int(w.keep[1])
-    return 3 * w.levels + 3 * trim + 2 + (1 if refresh else 0)
+    return 3 * w.levels + 3 * trim + 2
 
 
 # ---------------------------------------------------------------------------
@@ -221,25 +229,7 @@ def run_gpu(args, cfg, rank, world, device):
     step_ms = [a.elapsed_time(b) for a, b in evs]
     total_ms = sum(step_ms)
 
-    # Per-call timing of the two library calls (same flush protocol), for the
-    # dominant-kernel roofline.
     lay, bf = layers[0], bufs[0]
-    calls = {}
-    for name in ("filter", "attn"):
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(max(args.steps, 20))]
-        for a, b in ev:
-            flush.zero_()
-            a.record(stream)
-            if name == "filter":
-                wf.wf_filter(lay.Q, bf["coeffs"], lay.K, w.levels, keep, bf["idx"], bf["ws"], None, stream)
-            else:
-                wf.wf_sparse_attn(lay.Q, lay.K, lay.V, bf["idx"], w.k, lay.Kg, lay.Vg, bf["O"], bf["ws"], 0.0,
-                                  stream)
-            b.record(stream)
-        torch.cuda.synchronize()
-        calls[name] = statistics.mean(a.elapsed_time(b) for a, b in ev)
-
     # End to end through the public API with host buffers: copy the step's
     # query block and generation rows in from pinned memory, run the step,
     # copy O and the indices out.
@@ -266,8 +256,8 @@ def run_gpu(args, cfg, rank, world, device):
     e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
     h2d = sum(t.numel() * t.element_size() for t in (hQ, hKg, hVg))
     d2h = hO.numel() * hO.element_size() + hidx.numel() * 4
-    return dict(w=w, total_ms=total_ms, step_ms=step_ms, calls=calls, clocks=clocks, e2e_ms=e2e_ms,
-                h2d=h2d, d2h=d2h, layers=len(layers))
+    return dict(w=w, total_ms=total_ms, step_ms=step_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
+                layers=len(layers))
 
 
 def main():
@@ -345,19 +335,23 @@ def main():
     ms_per_step = total_ms / args.steps
     value = world * step_bytes / (ms_per_step * 1e-3) / 1e9
 
-    # Dominant call and its roofline.
-    calls = r["calls"]
-    dom = max(calls, key=calls.get)
-    dom_bytes = ub[dom] * w.units
-    achieved = dom_bytes / (calls[dom] * 1e-3) / 1e9
+    # Roofline of the dominant kernel: the fused step kernel is the only kernel
+    # of a step (one launch per layer), so its algorithmic bytes per launch are
+    # the step's bytes of one layer and its launch time is the step time per
+    # layer (a 4-byte status reset rides along on the same stream).
+    per_layer_ms = ms_per_step / w.layers
+    achieved = ub["step"] * w.units / (per_layer_ms * 1e-3) / 1e9
+    if w.refresh_every:
+        achieved = step_bytes / w.layers / (per_layer_ms * 1e-3) / 1e9
+    kname = "wf_fused_kernel" if fused_eligible(w) else "per-stage kernels (score/weights/select/attn)"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
-                "traffic": None, "kernel": f"wf_{dom} ({'3 kernels per scale' if dom == 'filter' else '2 kernels'})",
-                "peak_kind": peak_kind, "step_frac": (step_bytes / (ms_per_step * 1e-3) / 1e9) / hbm_peak,
-                "call_ms": calls}
+                "traffic": None, "kernel": kname, "peak_kind": peak_kind,
+                "bytes_per_launch": ub["step"] * w.units, "launch_us": per_layer_ms * 1e3}
     e2e_bytes_per_step = ub["step"] * w.units
     line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "step_us": ms_per_step * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if fused_eligible(w) else "f32",
             "data": "synthetic", "config": config, "roofline": roofline, "clocks": r["clocks"],
             "e2e": {"value": world * e2e_bytes_per_step / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                     "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"], "ms_per_step": e2e_ms,

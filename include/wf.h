@@ -27,8 +27,8 @@
  *   outputs are valid once the stream reaches that point.
  * - Every argument is checked on the host before anything is launched; a
  *   failed check returns a negative wf_status and enqueues nothing.  A failed
- *   launch returns WF_ERR_CUDA.  The library has no device-side waits in the
- *   kernels declared here, so no call can hang the device.
+ *   launch returns WF_ERR_CUDA.  The only device-side waits (in wf_step's
+ *   fused kernel) are bounded, so no call can hang the device.
  * - Supported: dtype WF_F32 or WF_BF16 (Q, K, V, Kg, Vg, coeffs and O all of
  *   the same dtype); head_dim 64 or 128; 1 <= query rows <= 64; prompt length
  *   n a multiple of 2^levels with 1 <= levels <= 10; base pointers and the
@@ -188,16 +188,29 @@ wf_status wf_sparse_attn_noalloc(const void* Q, const wf_tensor* q, const void* 
 
 /* ---------------------------------------------------------------------------
  * One denoising-step layer (Algorithm 1 body): if refresh_coeffs != 0, first
- * rebuild coeffs from K (wf_dwt_build); then wf_filter; then wf_sparse_attn
- * with scale 1/sqrt(d), writing idx and O.  Same arguments and rules as the
- * three calls; ws must hold wf_step_workspace_bytes().
+ * rebuild coeffs from K (wf_dwt_build); then the skim/scan filter and the
+ * sparse attention with scale 1/sqrt(d), writing idx (and level_sets, if not
+ * NULL) and O exactly as wf_filter + wf_sparse_attn define them.  Same
+ * arguments and rules as those calls; ws must hold wf_step_workspace_bytes().
+ *
+ * For bf16 with head_dim 128 and at most 32 query rows the filter and the
+ * attention run as one fused kernel (one thread-block cluster per (batch,
+ * head)); other shapes run the per-stage kernels.  The fused kernel's waits
+ * on tensor-core completion are bounded: if one gives up (it never should),
+ * the kernel returns early, outputs are undefined, and a status word at the
+ * start of ws is set; wf_workspace_status() reports it.
  * ------------------------------------------------------------------------- */
 size_t wf_step_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
                                int n_g);
 wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const void* V, const wf_tensor* kv,
                   const void* Kg, const void* Vg, const wf_tensor* g, void* coeffs, size_t coeffs_bytes,
-                  int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, void* O,
-                  const wf_tensor* o, void* ws, size_t ws_bytes, void* stream);
+                  int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
+                  void* O, const wf_tensor* o, void* ws, size_t ws_bytes, void* stream);
+
+/* Device status of the last wf_step calls that used workspace ws: waits for
+ * `stream`, returns WF_ERR_TIMEOUT (and clears the word) if a bounded device
+ * wait gave up, else WF_OK.  Synchronising; not for the hot loop. */
+wf_status wf_workspace_status(void* ws, void* stream);
 
 #ifdef __cplusplus
 }

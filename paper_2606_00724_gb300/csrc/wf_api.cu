@@ -198,18 +198,23 @@ WF_API wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K
                                      static_cast<cudaStream_t>(stream)));
 }
 
+// wf_step keeps a 256-byte status block at the start of its workspace (the
+// fused kernel's bounded waits report there); the rest is the scratch of the
+// per-stage kernels when the fused kernel does not apply.
+constexpr size_t kStatusBytes = 256;
+
 WF_API size_t wf_step_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
                                       int n_g) {
   if (check_filter_args(q, kv, levels, keep) != WF_OK || n_g < 0) return 0;
   const size_t f = wf::plan_filter(*q, *kv, levels, keep).total;
   const size_t a = wf::plan_attn(*q, keep[0], n_g).total;
-  return f > a ? f : a;
+  return kStatusBytes + (f > a ? f : a);
 }
 
 WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const void* V, const wf_tensor* kv,
                          const void* Kg, const void* Vg, const wf_tensor* g, void* coeffs, size_t coeffs_bytes,
-                         int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, void* O,
-                         const wf_tensor* o, void* ws, size_t ws_bytes, void* stream) {
+                         int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
+                         void* O, const wf_tensor* o, void* ws, size_t ws_bytes, void* stream) {
   wf_status st = check_filter_args(q, kv, levels, keep);
   if (st != WF_OK) return st;
   const int n_g = g ? g->seq : 0;
@@ -218,17 +223,46 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   if (n_g > 0 && (!Kg || !Vg)) return WF_ERR_INVALID_ARG;
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(coeffs)) return WF_ERR_ALIGN;
   if (n_g > 0 && (!aligned16(Kg) || !aligned16(Vg))) return WF_ERR_ALIGN;
-  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || (reinterpret_cast<uintptr_t>(idx) & 3u) != 0)
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || (reinterpret_cast<uintptr_t>(idx) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(level_sets) & 3u) != 0)
     return WF_ERR_ALIGN;
   if (coeffs_bytes < wf_coeffs_bytes(kv, levels)) return WF_ERR_WORKSPACE;
   if (ws_bytes < wf_step_workspace_bytes(q, kv, levels, keep, n_g)) return WF_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return WF_ERR_CUDA;
+  int* status = static_cast<int*>(ws);
+  void* scratch = static_cast<char*>(ws) + kStatusBytes;
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), s);
+  if (e != cudaSuccess) return WF_ERR_CUDA;
   if (refresh_coeffs && (e = wf::launch_dwt(K, *kv, levels, coeffs, s)) != cudaSuccess) return WF_ERR_CUDA;
-  const wf::FilterPlan fp = wf::plan_filter(*q, *kv, levels, keep);
-  if ((e = wf::launch_filter(fp, Q, *q, coeffs, K, *kv, idx, nullptr, ws, s)) != cudaSuccess) return WF_ERR_CUDA;
+  const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, n_g, sms);
+  if (fp.ok) {
+    e = wf::launch_fused(fp, Q, *q, K, V, *kv, Kg, Vg, n_g > 0 ? g : nullptr, coeffs, levels, keep, idx,
+                         level_sets, O, *o, status, s);
+    return cuda_status(e);
+  }
+  const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
+  if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, s)) != cudaSuccess)
+    return WF_ERR_CUDA;
   const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g);
   const float sc = 1.0f / sqrtf((float)q->head_dim);
-  e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, ws, s);
+  e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, s);
   return cuda_status(e);
+}
+
+WF_API wf_status wf_workspace_status(void* ws, void* stream) {
+  if (!ws) return WF_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int h = 0;
+  if (cudaMemcpyAsync(&h, ws, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess) return WF_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return WF_ERR_CUDA;
+  if (h != 0) {
+    if (cudaMemsetAsync(ws, 0, sizeof(int), s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
+      return WF_ERR_CUDA;
+    return WF_ERR_TIMEOUT;
+  }
+  return WF_OK;
 }

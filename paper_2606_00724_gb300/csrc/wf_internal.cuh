@@ -91,6 +91,20 @@ cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, c
                         const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
                         const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s);
 
+// Fused step (bf16, head_dim 128, <= 32 query rows): one cluster per unit.
+struct FusedPlan {
+  bool ok;
+  int cs, stages, tmem_cols, cmax, kmax, U;
+  size_t smem;
+  bool trim;
+};
+FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int n_g,
+                     int num_sms);
+cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd, const void* K, const void* V,
+                         const wf_tensor& kv, const void* Kg, const void* Vg, const wf_tensor* g,
+                         const void* coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
+                         void* O, const wf_tensor& od, int* status, cudaStream_t s);
+
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 }  // namespace wf

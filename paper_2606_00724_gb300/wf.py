@@ -52,7 +52,8 @@ SIGNATURES = {
     "wf_sparse_attn": (_I, [_P, _T, _P, _P, _T, _P, _I, _P, _P, _T, _P, _T, ctypes.c_float, _P, _SZ, _P]),
     "wf_step_workspace_bytes": (_SZ, [_T, _T, _I, _P, _I]),
     "wf_sparse_attn_noalloc": (_I, [_P, _T, _P, _P, _T, _P, _I, _P, _P, _T, _P, _T, ctypes.c_float, _P]),
-    "wf_step": (_I, [_P, _T, _P, _P, _T, _P, _P, _T, _P, _SZ, _I, _I, _P, _P, _P, _T, _P, _SZ, _P]),
+    "wf_step": (_I, [_P, _T, _P, _P, _T, _P, _P, _T, _P, _SZ, _I, _I, _P, _P, _P, _P, _T, _P, _SZ, _P]),
+    "wf_workspace_status": (_I, [_P, _P]),
 }
 
 
@@ -183,7 +184,8 @@ def wf_step_workspace_bytes(Q: torch.Tensor, K: torch.Tensor, levels: int, keep,
     return int(lib().wf_step_workspace_bytes(ctypes.byref(dq), ctypes.byref(dk), levels, _keep_arr(keep), n_g))
 
 
-def wf_step(Q, K, V, Kg, Vg, coeffs, refresh: bool, levels: int, keep, idx, O, ws, stream=None):
+def wf_step(Q, K, V, Kg, Vg, coeffs, refresh: bool, levels: int, keep, idx, O, ws, stream=None,
+            level_sets=None):
     dq, dk, do = desc(Q), desc(K), desc(O)
     dg = desc(Kg) if Kg is not None else None
     if V.stride() != K.stride() or V.shape != K.shape:
@@ -191,5 +193,11 @@ def wf_step(Q, K, V, Kg, Vg, coeffs, refresh: bool, levels: int, keep, idx, O, w
     _check(lib().wf_step(_ptr(Q), ctypes.byref(dq), _ptr(K), _ptr(V), ctypes.byref(dk), _ptr(Kg), _ptr(Vg),
                          ctypes.byref(dg) if dg is not None else None, _ptr(coeffs),
                          coeffs.numel() * coeffs.element_size(), int(bool(refresh)), levels, _keep_arr(keep),
-                         _ptr(idx), _ptr(O), ctypes.byref(do), _ptr(ws), ws.numel() * ws.element_size(),
-                         _stream(stream)), "wf_step")
+                         _ptr(idx), _ptr(level_sets), _ptr(O), ctypes.byref(do), _ptr(ws),
+                         ws.numel() * ws.element_size(), _stream(stream)), "wf_step")
+
+
+def wf_workspace_status(ws: torch.Tensor, stream=None):
+    """Raise WfError(WF_ERR_TIMEOUT) if a bounded device wait of the fused
+    step kernel gave up since the last check (synchronising)."""
+    _check(lib().wf_workspace_status(_ptr(ws), _stream(stream)), "wf_workspace_status")

@@ -142,7 +142,9 @@ def test_step_matches_separate_calls():
     torch.cuda.synchronize()
     assert torch.equal(coeffs, a.coeffs)
     assert torch.equal(idx, a.idx)
-    assert torch.equal(O, a.O)
+    # wf_step runs the fused kernel (bf16 P on the tensor cores): same
+    # indices, outputs within the bf16 tolerance of the per-stage kernels.
+    assert_close_out(f64(O), f64(a.O), torch.bfloat16)
     # Second step re-using the cached pyramid (no refresh) gives the same answer.
     O2 = torch.empty_like(O)
     wf.wf_step(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, coeffs, False, w.levels, w.keep, idx, O2, ws)

@@ -1,0 +1,99 @@
+"""GPU parity of wf_step, which runs the fused filter + sparse-attention
+kernel (one thread-block cluster per (batch, head), tcgen05 tensor cores)
+for bf16 / head_dim 128 / <= 32 query rows, against the fp64 oracle.
+
+Same bars as the per-stage kernels: pyramid bit-exact, indices bit-exact on
+planted inputs (every scale), bf16 outputs within max-abs 2e-2 and rel-L2
+1e-2; unplanted inputs must give a valid Top-K at every scale."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import GpuRun, assert_close_out, eps_valid, f64, make_layer, oracle_unit
+from paper_2606_00724_gb300 import synth, wf
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a GPU", allow_module_level=True)
+
+
+def _check(w, batch, run, units):
+    for u in units:
+        b, h = divmod(u, w.heads)
+        Q, K, V, Kg, Vg = (f64(t[b, h]) for t in (batch.Q, batch.K, batch.V, batch.Kg, batch.Vg))
+        pyr, mu0, sets, O = oracle_unit(Q, K, V, Kg, Vg, w.levels, w.keep, True)
+        assert np.array_equal(run.pyramid(u), pyr.astype(np.float64)), f"pyramid unit {u}"
+        gsets = run.level_sets(u)
+        for lev in range(w.levels, -1, -1):
+            assert np.array_equal(gsets[lev], sets[lev]), f"unit {u} scale {lev}"
+        assert np.array_equal(run.idx[u].cpu().numpy(), mu0), f"unit {u} mu0"
+        assert_close_out(f64(run.O[b, h]), O, torch.bfloat16)
+
+
+@pytest.mark.parametrize("cfg", ["c2", "c3", "c4", "c5"])
+def test_step_full_size(cfg):
+    w, batch = make_layer(cfg)
+    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).step()
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    units = [0, 1, w.units // 2 + 3, w.units - 1]
+    _check(w, batch, run, units)
+    idx = run.idx.cpu().numpy()
+    for u in range(w.units):
+        assert np.array_equal(idx[u], batch.targets[u][0].cpu().numpy()), f"unit {u} planted"
+
+
+def test_step_matches_per_stage_kernels():
+    # Planted 8K layer: the fused kernel and the per-stage kernels select the
+    # same indices and agree on the output.
+    w, batch = make_layer("c2")
+    a = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    b = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
+    b.coeffs.copy_(a.coeffs)
+    b.step(refresh=False)
+    torch.cuda.synchronize()
+    assert torch.equal(a.idx, b.idx)
+    assert torch.equal(a.sets, b.sets)
+    assert_close_out(f64(b.O), f64(a.O), torch.bfloat16)
+
+
+def _rand(seed, B, H, n, q, ng, bshd=False):
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    d = 128
+
+    def r(rows):
+        x = torch.randn(B, rows, H, d, generator=g) if bshd else torch.randn(B, H, rows, d, generator=g)
+        x = x.to(torch.bfloat16).cuda()
+        return x.transpose(1, 2) if bshd else x
+    return r(q), r(n), r(n), (r(ng) if ng else None), (r(ng) if ng else None)
+
+
+@pytest.mark.parametrize("B,H,n,q,ng,L,keep,bshd", [
+    (1, 3, 4096, 32, 32, 3, [300, 150, 160, 170], False),          # cluster of 4, ragged tiles
+    (2, 2, 2048, 7, 3, 2, [201, 101, 130], True),                  # trim, odd q, BSHD
+    (1, 2, 1024, 1, 0, 1, [512, 256], False),                      # q = 1, no generation rows, L = 1
+    (1, 1, 256, 32, 5, 4, [256, 128, 64, 32, 16], False),          # keep everything
+    (1, 2, 512, 16, 1, 6, [1, 1, 1, 1, 1, 1, 1], False),           # k = 1, deep pyramid
+    (1, 4, 65536, 32, 32, 5, [3000, 1500, 1600, 1700, 1800, 1900], False),  # large ragged schedule
+])
+def test_step_random_shapes(B, H, n, q, ng, L, keep, bshd):
+    Q, K, V, Kg, Vg = _rand(n + q + L, B, H, n, q, ng, bshd)
+    run = GpuRun(Q, K, V, Kg, Vg, L, keep).step()
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    for u in range(B * H):
+        b, h = divmod(u, H)
+        Qn, Kn, Vn = f64(Q[b, h]), f64(K[b, h]), f64(V[b, h])
+        Kgn = f64(Kg[b, h]) if ng else None
+        Vgn = f64(Vg[b, h]) if ng else None
+        pyr = oracle.haar_pyramid_spec32(Kn.astype(np.float32), L, True).astype(np.float64)
+        assert np.array_equal(run.pyramid(u), pyr)
+        gsets = run.level_sets(u)
+        eps_valid(Qn, pyr, Kn, n, L, keep, gsets)
+        idx = run.idx[u].cpu().numpy()
+        assert np.array_equal(idx, gsets[0])
+        assert np.all(np.diff(idx) > 0) and idx.min() >= 0 and idx.max() < n
+        O = oracle.sparse_attn(Qn, Kn, Vn, idx, Kgn, Vgn)
+        assert_close_out(f64(run.O[b, h]), O, torch.bfloat16)
