@@ -238,7 +238,7 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), s);
   if (e != cudaSuccess) return WF_ERR_CUDA;
   if (refresh_coeffs && (e = wf::launch_dwt(K, *kv, levels, coeffs, s)) != cudaSuccess) return WF_ERR_CUDA;
-  const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, n_g, sms);
+  const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, n_g, n_g > 0 ? g : nullptr, sms);
   if (fp.ok) {
     e = wf::launch_fused(fp, Q, *q, K, V, *kv, Kg, Vg, n_g > 0 ? g : nullptr, coeffs, levels, keep, idx,
                          level_sets, O, *o, status, s);

@@ -99,7 +99,7 @@ struct FusedPlan {
   bool trim;
 };
 FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int n_g,
-                     int num_sms);
+                     const wf_tensor* g, int num_sms);
 cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                          const wf_tensor& kv, const void* Kg, const void* Vg, const wf_tensor* g,
                          const void* coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
