@@ -76,6 +76,25 @@ def fused_eligible(w: synth.Workload) -> bool:
     return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32
 
 
+def recorded_traffic(w: synth.Workload):
+    """DRAM bytes per launch of the fused kernel from the committed ncu record,
+    if it was taken on this workload with the current kernel source."""
+    import hashlib
+    rec = os.path.join(ROOT, "profiles", "wf_fused_kernel_traffic.md")
+    src = os.path.join(ROOT, "paper_2606_00724_gb300", "csrc", "wf_fused.cu")
+    if not (os.path.exists(rec) and os.path.exists(src)):
+        return None
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    for ln in open(rec):
+        cells = [c.strip() for c in ln.strip().strip("|").split("|")]
+        if len(cells) == 6 and cells[0] == w.name and cells[5] == h:
+            try:
+                return int(cells[3])
+            except ValueError:
+                return None
+    return None
+
+
 def launches_per_step(w: synth.Workload) -> int:
     if fused_eligible(w):
         return 1
@@ -270,6 +289,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--preroll", type=float, default=1.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=None, help="override the workload's batch (small profiling cases)")
+    ap.add_argument("--heads", type=int, default=None, help="override the workload's head count")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -279,6 +300,11 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     cfg = args.workload
     w = synth.WORKLOADS[cfg]
+    if args.batch or args.heads:
+        import dataclasses
+        w = dataclasses.replace(w, batch=args.batch or w.batch, heads=args.heads or w.heads,
+                                name=f"{w.name}_B{args.batch or w.batch}_H{args.heads or w.heads}")
+        synth.WORKLOADS[cfg] = w
     ub = unit_bytes(w)
     hbm_peak, peak_kind = peaks()
 
@@ -345,7 +371,8 @@ def main():
         achieved = step_bytes / w.layers / (per_layer_ms * 1e-3) / 1e9
     kname = "wf_fused_kernel" if fused_eligible(w) else "per-stage kernels (score/weights/select/attn)"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
-                "traffic": None, "kernel": kname, "peak_kind": peak_kind,
+                "traffic": recorded_traffic(w) if fused_eligible(w) else None, "kernel": kname,
+                "peak_kind": peak_kind,
                 "bytes_per_launch": ub["step"] * w.units, "launch_us": per_layer_ms * 1e3}
     e2e_bytes_per_step = ub["step"] * w.units
     line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
