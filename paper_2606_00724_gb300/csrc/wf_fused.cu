@@ -1,37 +1,40 @@
 // Fused WaveFilter step (Algorithm 1 body): multi-scale skim/scan filtering
 // (Eq. 7-11) and the final sparse attention, in one kernel.
 //
-// One thread-block cluster per (batch, head) unit; the cluster's CTAs split
-// every scale's candidate list (and finally the sparse key list) into
-// contiguous slices.  Per scale, each CTA:
-//   1. gathers its candidate rows (pyramid level b, or raw keys for the
-//      level-0 trim) with 16-byte cp.async copies straight into
-//      128-byte-swizzled tiles of 128 rows; every thread pipelines its own
-//      copies through a ring of stages and signals completion on the stage's
-//      mbarrier (cp.async.mbarrier.arrive), and one thread issues
-//      tcgen05.mma (bf16 in, fp32 out) for each tile that has landed,
-//      writing S^T = rows . Q^T into TMEM (32 columns per tile);
-//   2. reads the logits back from TMEM (tcgen05.ld) for the per-query max and
-//      sum of exp over its slice and exchanges them through distributed
-//      shared memory, giving every CTA the softmax normaliser of Eq. 7;
-//   3. computes the ranking key log2 W_j (Eq. 8, as a log-sum-exp over the
-//      query rows) of its candidates and writes them into every CTA's key
-//      array (DSMEM all-gather);
-//   4. runs the same deterministic Top-K (radix select on the key bits,
-//      lowest index first on ties, Eq. 9) in every CTA, so each knows J_b and
-//      hence the next scale's candidates {2j, 2j+1} (Eq. 10) without a
-//      broadcast.
-// The attention stage gathers the K rows of mu^0 and the generation rows the
-// same way, forms S^T = K_s Q^T in TMEM, and then streams the V rows while
-// four warps turn S into P = exp(S - m) (bf16) and the MMA thread
-// accumulates O^T = V_s^T P^T (both operands MN-major); the cluster's partial
-// (m, l, O) are combined in CTA 0.
+// A thread-block cluster of CS CTAs serves P (1 or 2) (batch, head) units;
+// every CTA holds one contiguous slice of each unit's candidate list at every
+// scale (and finally of its sparse key list).  The warps of a CTA specialise:
+//   * producer warps gather candidate rows (pyramid level b, raw keys for the
+//     level-0 trim, or K/V rows of mu^0 and the generation rows) with 16-byte
+//     cp.async copies into 128-byte-swizzled tiles of 128 rows, through a ring
+//     of stages; each copy's completion arrives on the stage's mbarrier;
+//   * one MMA thread issues tcgen05.mma (bf16 in, fp32 out) per landed tile,
+//     writing S^T = rows . Q^T into the unit's TMEM region (32 columns per
+//     tile), and in the attention O^T += V_s^T P^T;
+//   * four compute warps (one per TMEM lane quarter, one candidate row per
+//     thread) read the logits back (tcgen05.ld), form the per-query max and
+//     sum of exp of the slice, exchange them with the cluster (st.async into
+//     every CTA, completion counted on its mbarrier), compute the ranking key
+//     log2 W_j (Eq. 8) of each candidate, all-gather the keys the same way,
+//     and run the same deterministic Top-K (Eq. 9, lowest position first on
+//     ties) in every CTA, giving J_b and hence the next scale's candidates
+//     {2j, 2j+1} (Eq. 10).
+// The units of a cluster alternate: while the compute warps score, exchange
+// and select one unit, the producers already stream the other unit's rows, so
+// copies overlap the latency-bound phases.  In the attention the compute warps
+// turn S into P = 2^(s - m) (bf16) for the MMA thread, and each CTA's partial
+// (m, l, O^T) is reduce-scattered over head-dimension slices: CTA r combines
+// rows d of O for its slice and writes them.
 //
-// Every wait on asynchronous work (copies, MMA completion) is bounded
-// (~1 s): on timeout the CTA records a status word, stops issuing MMAs, keeps
-// joining every barrier and returns.
+// Every wait is bounded (~1 s): on timeout the CTA records a status word,
+// stops issuing MMAs and skips the remaining waits, so every thread reaches
+// the final cluster barrier.
 #include <math.h>
 #include <string.h>
+
+#include <map>
+#include <mutex>
+#include <tuple>
 
 #include "wf_internal.cuh"
 #include "wf_sm100.cuh"
@@ -41,43 +44,66 @@ namespace {
 
 using namespace sm100;
 
-constexpr int NT = 256;                  // threads per CTA (8 warps)
-constexpr int D = 128;                   // head_dim
-constexpr int TM = 128;                  // rows per MMA tile (M)
-constexpr int NQ = 32;                   // query rows per MMA (N), zero padded
-constexpr int HALF_BYTES = TM * 128;     // one 64-column half of a tile, 128-byte rows
+constexpr int D = 128;                     // head_dim
+constexpr int TM = 128;                    // rows per MMA tile (M)
+constexpr int NQ = 32;                     // query rows per MMA (N), zero padded
+constexpr int MAXP = 2;                    // units per cluster
+constexpr int NCW = 4;                     // compute warps of a unit (one per TMEM lane quarter)
+constexpr int NCT = 32 * NCW;              // compute threads of a unit
+constexpr int MMA_WARP = MAXP * NCW;       // TMEM allocation and MMA issue (lane 0)
+constexpr int NPW = 3;                     // producer warps
+constexpr int NPT = 32 * NPW;              // producer threads
+constexpr int P0 = 32 * (MMA_WARP + 1);    // first producer thread
+constexpr int NT = 32 * (MMA_WARP + 1 + NPW);  // threads per CTA
+constexpr int MAXCS = 8;                   // CTAs per cluster
+constexpr int HALF_BYTES = TM * 128;       // one 64-column half of a tile, 128-byte rows
 constexpr int TILE_BYTES = 2 * HALF_BYTES;
-constexpr int QGRP = (D / 8) * 128;      // bytes per 8-row group of the query tile (core matrices)
+constexpr int QGRP = (D / 8) * 128;        // bytes per 8-row group of a query tile (core matrices)
 constexpr int Q_BYTES = NQ * D * 2;
 constexpr int P_BYTES = NQ * TM * 2;
+constexpr int COMB_BYTES = NQ * D * 4;     // received partial O rows of this CTA's head-dim slice
+constexpr int UNIT_P_BYTES = 2 * P_BYTES;  // a unit's P double buffer (also its Top-K scratch and combine buffer)
+constexpr int kMaxCand = 32 * NCT;         // largest candidate list the Top-K holds in registers
 constexpr long long kWaitLimit = 1ll << 31;
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr uint32_t kCsyncId = 1;           // named barriers 1, 2: the compute warps of unit 0, 1
 
 constexpr uint32_t kIdescScore = idesc_bf16(TM, NQ, 0, 0);  // A = rows (K-major), B = Q (K-major)
 constexpr uint32_t kIdescPV = idesc_bf16(D, NQ, 1, 1);      // A = V^T (MN-major), B = P^T (MN-major)
 
+struct UnitState {
+  float2 xstat[MAXCS][NQ];  // (max, sum of exp) of every cluster CTA's slice
+  float2 cstat[MAXCS][NQ];  // attention (max, row sum) of every CTA (d-slice owner side)
+  float mloc[NQ], cvec[NQ], lacc[NQ];
+  float red[NCW][32];
+};
+
 struct Misc {
-  unsigned long long full[8], empty[8], done, pfull[2], pempty[2];
-  float2 xstat[8][32];
-  float red[8][32];
-  float cvec[32];
-  float mloc[32];
-  float lacc[32];
-  int wsum[8];
-  uint32_t sel_bin, sel_need, sel_cnt;
+  unsigned long long full[4], empty[4];
+  unsigned long long mdone[MAXP], jready[MAXP], xbar[MAXP], kbar[MAXP];
+  unsigned long long pfull[MAXP][2], pempty[MAXP][2], cbar[MAXP], cready[MAXP];
+  UnitState us[MAXP];
   int abort;
   uint32_t tmem_base;
 };
 
-template <int STAGES>
-struct Layout {
-  static constexpr uint32_t off_stage = 0;
-  static constexpr uint32_t off_q = STAGES * TILE_BYTES;
-  static constexpr uint32_t off_p = off_q + Q_BYTES;
-  static constexpr uint32_t off_hist = off_p + 2 * P_BYTES;
-  static constexpr uint32_t off_misc = off_hist + 8 * 256 * 4;
-  static constexpr uint32_t off_keys = (off_misc + sizeof(Misc) + 127) / 128 * 128;
+// Shared-memory layout (byte offsets; the stage ring starts at 0, 1024-byte
+// aligned for the 128-byte swizzle).
+struct SmemLayout {
+  uint32_t q, p, misc, buf, bufw, total;
 };
+__host__ __device__ inline SmemLayout smem_layout(int stages, int P, int cmax, int kmax) {
+  SmemLayout l;
+  l.q = (uint32_t)stages * TILE_BYTES;
+  l.p = l.q + (uint32_t)P * Q_BYTES;
+  l.misc = l.p + (uint32_t)P * UNIT_P_BYTES;
+  // Two buffers per unit alternate by scale: one receives the scale's keys and
+  // then its selection J_b, the other still holds J_{b+1}.
+  l.buf = (l.misc + (uint32_t)sizeof(Misc) + 127u) / 128u * 128u;
+  l.bufw = (uint32_t)((max(cmax, kmax) + 3) / 4 * 4);
+  l.total = l.buf + (uint32_t)P * 2u * 4u * l.bufw;
+  return l;
+}
 
 struct FusedParams {
   const bf16* Q;
@@ -96,16 +122,305 @@ struct FusedParams {
   int32_t* level_sets;
   int64_t sets_stride;
   int* status;
-  int q, n, ng, H, L, trim, cmax, kmax;
-  uint32_t tmem_cols;
+  int q, n, ng, U, H, L, trim, P, cmax, kmax;
+  uint32_t tmem_cols, ucols;  // TMEM allocation; columns per unit region
   int32_t keep[12];
-  float scale_log2;  // log2(e) / sqrt(d)
+  float scale_log2;           // log2(e) / sqrt(d)
 };
 
-__device__ __forceinline__ uint32_t okey(float f) {
-  const uint32_t b = __float_as_uint(f);
-  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+// Per-CTA constants and shared-memory addresses.
+struct Ctx {
+  uint8_t* smem;
+  Misc* ms;
+  SmemLayout ly;
+  uint32_t rank, cs, tmem;
+  int np, u0, lev_end, stages;
+};
+
+// Thread index within its unit's compute warps, and their barrier.
+__device__ __forceinline__ int ctid() { return threadIdx.x & (NCT - 1); }
+__device__ __forceinline__ void csync() { named_sync(kCsyncId + (threadIdx.x >> 7), NCT); }
+
+__device__ __forceinline__ bool aborted(const Misc& ms) { return abort_set(smem_u32(&ms.abort)); }
+
+__device__ __forceinline__ void set_abort(Misc& ms, int* status) {
+  ms.abort = 1;
+  atomicExch(status, 1);
 }
+
+__device__ __noinline__ void wait_or_abort(uint32_t bar, uint32_t parity, Misc& ms, int* status) {
+  if (!aborted(ms) && !mbar_wait_bounded(bar, parity, kWaitLimit, smem_u32(&ms.abort))) set_abort(ms, status);
+}
+
+// Wait for a phase completed by other CTAs of the cluster (acquire, cluster scope).
+__device__ __noinline__ void wait_cluster_or_abort(uint32_t bar, uint32_t parity, Misc& ms, int* status) {
+  if (!aborted(ms) && !mbar_wait_cluster_bounded(bar, parity, kWaitLimit, smem_u32(&ms.abort))) set_abort(ms, status);
+}
+
+__device__ __forceinline__ uint32_t bar_addr(const unsigned long long& b) { return smem_u32(&b); }
+
+// Candidate count of scale `lev`: the top coefficients, or the children of
+// the coefficients kept one scale up (Eq. 10).
+__device__ __forceinline__ int m_total(const FusedParams& p, int lev) {
+  return lev == p.L ? (p.n >> p.L) : 2 * p.keep[lev + 1];
+}
+
+// This CTA's slice [g0, g0 + mc) of a candidate list of m (sibling pairs kept
+// together).
+__device__ __forceinline__ void scale_slice(int m, uint32_t rank, uint32_t cs, int& g0, int& mc) {
+  const int pairs = (m + 1) >> 1;
+  g0 = min(m, 2 * (int)((int64_t)rank * pairs / cs));
+  const int g1 = min(m, 2 * (int)((int64_t)(rank + 1) * pairs / cs));
+  mc = g1 - g0;
+}
+
+// This CTA's slice of the sparse key list of `total` rows.
+__device__ __forceinline__ void attn_slice(int total, uint32_t rank, uint32_t cs, int& a0, int& mc) {
+  a0 = (int)((int64_t)rank * total / cs);
+  mc = (int)((int64_t)(rank + 1) * total / cs) - a0;
+}
+
+__device__ __forceinline__ int tiles_of(int mc) { return (mc + TM - 1) / TM; }
+
+// Where the rows of a candidate or key list come from.
+//  kind 0: position j -> row j (top scale);
+//  kind 1: position j -> row 2 J[j/2] + j%2 (children of the kept coefficients);
+//  kind 2: sparse key list, positions < kk -> token 2 J[j/2] + j%2, then
+//          generation rows;
+//  kind 3: the same with a trimmed level 0, positions < kk -> token J[j].
+struct RowSrc {
+  const bf16* base;
+  int64_t stride;
+  const bf16* gbase;
+  int64_t gstride;
+  uint32_t J;  // shared address of the selection the rows derive from
+  int kind, g0, mc, kk;
+};
+
+// Branch-free, so a batch of row addresses is formed without divergence.
+template <int KIND>
+__device__ __forceinline__ const bf16* row_ptr(const RowSrc& s, int r) {
+  const int pos = s.g0 + (r < s.mc ? r : 0);  // rows past the slice repeat its first row
+  if (KIND == 0) return s.base + (int64_t)pos * s.stride;
+  if (KIND == 1) return s.base + (int64_t)(2 * (int)lds_u32(s.J + 4u * (uint32_t)(pos >> 1)) + (pos & 1)) * s.stride;
+  const int pk = min(pos, s.kk - 1);
+  const int tok = KIND == 3 ? (int)lds_u32(s.J + 4u * (uint32_t)pk)
+                            : 2 * (int)lds_u32(s.J + 4u * (uint32_t)(pk >> 1)) + (pk & 1);
+  const bf16* key = s.base + (int64_t)tok * s.stride;
+  const bf16* gen = s.gbase + (int64_t)(pos - s.kk) * s.gstride;
+  return pos < s.kk ? key : gen;
+}
+
+// Buffer k (0, 1) of unit pp; scale lev's keys and selection use buffer
+// (L - lev) % 2.
+__device__ __forceinline__ int32_t* unit_buf(const Ctx& c, int pp, int k) {
+  return reinterpret_cast<int32_t*>(c.smem + c.ly.buf) + (pp * 2 + k) * (int)c.ly.bufw;
+}
+// Buffer holding the selection J made at scale lev.
+__device__ __forceinline__ int32_t* unit_J(const Ctx& c, const FusedParams& p, int pp, int lev) {
+  return unit_buf(c, pp, (p.L - lev) & 1);
+}
+
+// Rows of unit u at scale lev (pyramid level lev, or the raw keys at level 0).
+__device__ __forceinline__ RowSrc scale_src(const Ctx& c, const FusedParams& p, int pp, int lev, int g0, int mc) {
+  const int u = c.u0 + pp;
+  RowSrc s;
+  if (lev >= 1) {
+    s.base = p.coeffs + ((int64_t)u * p.rows_total + ((int64_t)p.n - ((int64_t)p.n >> (lev - 1)))) * D;
+    s.stride = D;
+  } else {
+    s.base = p.K + (int64_t)(u / p.H) * p.ksb + (int64_t)(u % p.H) * p.ksh;
+    s.stride = p.kss;
+  }
+  s.gbase = nullptr;
+  s.gstride = 0;
+  s.J = smem_u32(unit_J(c, p, pp, lev + 1));  // the children of the selection one scale up (unused at the top)
+  s.kind = lev == p.L ? 0 : 1;
+  s.g0 = g0;
+  s.mc = mc;
+  s.kk = 0;
+  return s;
+}
+
+// Sparse key list [K[mu^0]; Kg] (or the V rows) of unit pp.
+__device__ __forceinline__ RowSrc attn_src(const Ctx& c, const FusedParams& p, int pp, bool values, int a0,
+                                           int mc) {
+  const int u = c.u0 + pp;
+  const int64_t b = u / p.H, h = u % p.H;
+  RowSrc s;
+  s.base = (values ? p.V : p.K) + b * p.ksb + h * p.ksh;
+  s.stride = p.kss;
+  s.gbase = (values ? p.Vg : p.Kg) + b * p.gsb + h * p.gsh;
+  s.gstride = p.gss;
+  s.J = smem_u32(unit_J(c, p, pp, p.trim ? 0 : 1));  // mu^0 from the last selection
+  s.kind = p.trim ? 3 : 2;
+  s.g0 = a0;
+  s.mc = mc;
+  s.kk = p.keep[0];
+  return s;
+}
+
+// ---------------------------------------------------------------------------
+// Producer warps.
+// ---------------------------------------------------------------------------
+
+// This producer thread's share of one 128-row tile: 16-byte chunk c = pt % 16
+// of rows pt/16 + RSTEP i, written in the 128-byte-swizzled K-major layout
+// (row r, chunk c at half c/8, byte r*128 + ((c%8) ^ (r%8))*16).  The source
+// addresses of a batch of rows are formed before its copies are issued, so
+// the index loads overlap.
+constexpr int RSTEP = NPT / 16;
+constexpr int RROWS = (TM + RSTEP - 1) / RSTEP;  // most rows of one thread
+template <int KIND>
+__device__ __forceinline__ void load_share(uint32_t st, int t, const RowSrc& src, int pt) {
+  const int c = pt & 15, r0 = pt >> 4;
+  const uint32_t cbase = st + ((c >> 3) << 14);
+#pragma unroll 1
+  for (int b = 0; b < RROWS; b += 8) {
+    const bf16* g[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) g[k] = row_ptr<KIND>(src, t * TM + min(r0 + RSTEP * (b + k), TM - 1)) + c * 8;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int r = r0 + RSTEP * (b + k);
+      if (b + k < RROWS && r < TM) cp_async16(cbase + r * 128 + (((c & 7) ^ (r & 7)) << 4), g[k]);
+    }
+  }
+}
+
+template <int S>
+__device__ __noinline__ void produce(Misc& ms, int* status, uint32_t ring, int it0, int ntl, const RowSrc src, int pt) {
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
+    const int it = it0 + t, s = it % S, n = it / S;
+    if (n > 0) wait_or_abort(bar_addr(ms.empty[s]), (uint32_t)(n - 1) & 1u, ms, status);
+    if (!aborted(ms)) {
+      const uint32_t st = ring + s * TILE_BYTES;
+      switch (src.kind) {
+        case 0: load_share<0>(st, t, src, pt); break;
+        case 1: load_share<1>(st, t, src, pt); break;
+        case 2: load_share<2>(st, t, src, pt); break;
+        default: load_share<3>(st, t, src, pt); break;
+      }
+    }
+    cp_async_arrive_noinc(bar_addr(ms.full[s]));
+  }
+}
+
+template <int S>
+__device__ void producer_role(const Ctx& c, const FusedParams& p) {
+  Misc& ms = *c.ms;
+  const int pt = threadIdx.x - P0;
+  int it = 0;
+  for (int lev = p.L; lev >= c.lev_end; --lev) {
+    for (int pp = 0; pp < c.np; ++pp) {
+      // The rows of a lower scale are the children of the unit's last selection.
+      if (lev != p.L) wait_or_abort(bar_addr(ms.jready[pp]), (uint32_t)(p.L - lev - 1) & 1u, ms, p.status);
+      int g0, mc;
+      scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
+      const int ntl = tiles_of(mc);
+      produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, scale_src(c, p, pp, lev, g0, mc), pt);
+      it += ntl;
+    }
+  }
+  const int nsel = p.L - c.lev_end + 1;
+  for (int pp = 0; pp < c.np; ++pp) {
+    wait_or_abort(bar_addr(ms.jready[pp]), (uint32_t)(nsel - 1) & 1u, ms, p.status);
+    int a0, mc;
+    attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
+    const int ntl = tiles_of(mc);
+    produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, attn_src(c, p, pp, false, a0, mc), pt);
+    it += ntl;
+    produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, attn_src(c, p, pp, true, a0, mc), pt);
+    it += ntl;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// MMA thread.
+// ---------------------------------------------------------------------------
+
+// S^T tile t = rows . Q^T into TMEM columns tb + 32 t, for ntl landed tiles.
+template <int S>
+__device__ __forceinline__ void mma_scores(const Ctx& c, const FusedParams& p, int it0, int ntl, uint32_t tb,
+                                           uint32_t sq) {
+  Misc& ms = *c.ms;
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
+    const int it = it0 + t, s = it % S, n = it / S;
+    wait_or_abort(bar_addr(ms.full[s]), (uint32_t)n & 1u, ms, p.status);
+    fence_proxy_async();
+    if (!aborted(ms)) {
+      tc_fence_after();
+      const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_bf16(tb + 32 * t, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
+                   smem_desc(sq + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
+    }
+    mma_commit(bar_addr(ms.empty[s]));
+  }
+}
+
+// O^T += V_s^T P^T over ntl landed V tiles, P tile t from unit pp's compute warps.
+template <int S>
+__device__ __forceinline__ void mma_pv(const Ctx& c, const FusedParams& p, int pp, int it0, int ntl, uint32_t ocol) {
+  Misc& ms = *c.ms;
+  const uint32_t pa = smem_u32(c.smem + c.ly.p + pp * UNIT_P_BYTES);
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
+    const int it = it0 + t, s = it % S, n = it / S;
+    const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
+    wait_or_abort(bar_addr(ms.full[s]), (uint32_t)n & 1u, ms, p.status);
+    wait_or_abort(bar_addr(ms.pfull[pp][pb]), pn & 1u, ms, p.status);
+    fence_proxy_async();
+    if (!aborted(ms)) {
+      tc_fence_after();
+      const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
+#pragma unroll
+      for (int kq = 0; kq < TM / 16; ++kq)
+        mma_bf16(ocol, smem_desc_sw128(st + kq * 2048, HALF_BYTES, 1024),
+                 smem_desc(pa + pb * P_BYTES + kq * 1024, 512, 128), kIdescPV, (t > 0 || kq > 0) ? 1u : 0u);
+    }
+    mma_commit(bar_addr(ms.empty[s]));
+    mma_commit(bar_addr(ms.pempty[pp][pb]));
+  }
+}
+
+template <int S>
+__device__ void mma_role(const Ctx& c, const FusedParams& p) {
+  Misc& ms = *c.ms;
+  int it = 0;
+  for (int lev = p.L; lev >= c.lev_end; --lev) {
+    for (int pp = 0; pp < c.np; ++pp) {
+      int g0, mc;
+      scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
+      const int ntl = tiles_of(mc);
+      mma_scores<S>(c, p, it, ntl, c.tmem + pp * p.ucols, smem_u32(c.smem + c.ly.q + pp * Q_BYTES));
+      it += ntl;
+      if (ntl > 0) mma_commit(bar_addr(ms.mdone[pp]));  // an empty slice has no phase
+    }
+  }
+  for (int pp = 0; pp < c.np; ++pp) {
+    int a0, mc;
+    attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
+    const int ntl = tiles_of(mc);
+    const uint32_t tb = c.tmem + pp * p.ucols;
+    if (ntl == 0) continue;
+    mma_scores<S>(c, p, it, ntl, tb, smem_u32(c.smem + c.ly.q + pp * Q_BYTES));
+    it += ntl;
+    mma_commit(bar_addr(ms.mdone[pp]));
+    mma_pv<S>(c, p, pp, it, ntl, tb + p.ucols - 32);
+    it += ntl;
+    mma_commit(bar_addr(ms.mdone[pp]));
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Compute warps.
+// ---------------------------------------------------------------------------
 
 // Reduce 32 values per lane across the warp's 32 lanes; afterwards lane i
 // holds the reduction of column i (31 shuffles).
@@ -125,84 +440,84 @@ __device__ __forceinline__ float transpose_reduce32(float (&v)[32], int lane) {
   return v[0];
 }
 
-// Reduce 8 values per lane across the warp's 32 lanes; afterwards every lane
-// L holds the reduction of column (L / 4) % 8 (9 shuffles).
-template <bool MAX>
-__device__ __forceinline__ float transpose_reduce8(float (&v)[8], int lane) {
-#pragma unroll
-  for (int off = 16, n = 4; off >= 4; off >>= 1, n >>= 1) {
-    const bool up = (lane & off) != 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (j < n) {
-        const float keep = up ? v[j + n] : v[j];
-        const float send = up ? v[j] : v[j + n];
-        const float recv = __shfl_xor_sync(0xffffffffu, send, off);
-        v[j] = MAX ? fmaxf(keep, recv) : keep + recv;
-      }
-    }
-  }
-  float r = v[0];
-#pragma unroll
-  for (int off = 2; off >= 1; off >>= 1) {
-    const float o = __shfl_xor_sync(0xffffffffu, r, off);
-    r = MAX ? fmaxf(r, o) : r + o;
-  }
-  return r;
-}
+// Top-K scratch.  It lives in the P buffers, which nothing uses before the
+// attention.
+constexpr int NB = 2048;  // histogram buckets
+constexpr int BPT = NB / NCT;
+struct SelScratch {
+  uint32_t hist[NB];
+  float2 blist[NCT];             // boundary-bucket keys (key, position)
+  uint32_t bmap[kMaxCand / 32];  // chosen boundary positions
+  float2 sred[2][NCW];           // (min, max) per warp, alternating rounds
+  uint32_t ssel[2][4];           // boundary bucket, missing count, bucket count
+  int wsum[NCW];
+  uint32_t bcnt;
+};
+static_assert(sizeof(SelScratch) <= 2 * P_BYTES, "Top-K scratch must fit the P buffers");
+static_assert(kMaxCand / 32 == NCT, "one bitmap word per compute thread");
+static_assert(BPT % 4 == 0, "buckets are read four at a time");
 
-// Exclusive prefix sum over the CTA's 256 threads (thread order).
-__device__ __forceinline__ int block_excl_scan(int v, Misc& ms) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#define SC_ADDR(sc_a, field) ((sc_a) + (uint32_t)offsetof(SelScratch, field))
+
+// Exclusive prefix sum over the compute threads (thread order).
+__device__ __forceinline__ int cta_excl_scan(int v, uint32_t wsum_a) {
+  const int lane = threadIdx.x & 31, warp = ctid() >> 5;
   int incl = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const int t = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += t;
   }
-  if (lane == 31) ms.wsum[warp] = incl;
-  __syncthreads();
-  int before = 0;
-#pragma unroll
-  for (int w = 0; w < 8; ++w) before += w < warp ? ms.wsum[w] : 0;
-  __syncthreads();
+  if (lane == 31) sts_u32(wsum_a + 4u * warp, (uint32_t)incl);
+  csync();
+  const uint4 w = lds_v4(wsum_a);
+  csync();
+  const int before = (warp > 0 ? (int)w.x : 0) + (warp > 1 ? (int)w.y : 0) + (warp > 2 ? (int)w.z : 0);
   return before + incl - v;
 }
 
-// Candidate (or token) index of position j of the current candidate list.
-__device__ __forceinline__ int cand_of(int j, bool top, const int32_t* Jprev) {
-  return top ? j : 2 * Jprev[j >> 1] + (j & 1);
+// Bucket of key v in NB buckets linear over [lo, hi): the same fp32
+// operations in every pass and every CTA give the same bucket.
+__device__ __forceinline__ int bucket_of(float v, float lo, float scale) {
+  // floor(x) for 0 <= x < 2^23: adding 2^23 rounded toward -inf leaves
+  // floor(x) in the low mantissa bits.
+  const float x = fmaxf((v - lo) * scale, 0.f);
+  return min(NB - 1, __float_as_int(__fadd_rd(x, 8388608.f)) - 0x4B000000);
 }
 
-// Top-K of keys[0..m) (largest first, lower position wins ties); writes the
-// kk chosen candidate indices in ascending position order to Jout.
-// Each thread holds a run of R <= 32 keys in registers (slot x holds position
-// j0 + (x + rot) % R; the rotation spreads a warp's reads over the banks).
-// The boundary is found by range bucketing: the still-undecided keys are
-// spread over 256 buckets linear in [min, max] of those keys (fp32
-// arithmetic is monotone, so a key in a higher bucket is strictly larger),
-// the bucket holding the boundary is located from the bucket counts, keys
-// above it are taken and keys below it dropped, and the boundary bucket is
-// bucketed again over its own range until it holds exactly the missing count
-// or only equal keys, which are then taken lowest position first.  Buckets
-// stay evenly filled, so the shared-memory histogram atomics rarely collide.
+// Top-K of the m keys at keys_a (largest first, lower position wins ties):
+// the kk chosen candidate indices, in ascending position order, overwrite the
+// key array.  A candidate's index is its position at the top scale, else
+// 2 J[j/2] + j%2 with J the previous selection at jprev_a (Eq. 10).
+// Each thread holds a run of R keys in registers (slot x holds position
+// j0 + (x + rot) % R; the rotation spreads a warp's reads over the banks) and
+// one bit per slot for "undecided" and "taken".  The undecided keys are
+// spread over NB buckets linear in [min, max] of those keys (fp32 arithmetic
+// is monotone, so a key in a higher bucket is strictly larger) and the bucket
+// holding the boundary is located from the bucket counts: keys above it are
+// taken, keys below it dropped.  A boundary bucket of at most NCT keys is
+// resolved exactly by ranking its keys on (key, -position); a larger one is
+// bucketed again over its own range.  If only equal keys remain, the lowest
+// positions are taken.
 template <int R>
-__device__ __forceinline__ void select_impl(const float* keys, int m, int kk, int32_t* Jout, bool top,
-                                            const int32_t* Jprev, Misc& ms, uint32_t* hist) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+__device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const int j0 = tid * R;
-  const int rot = ((tid & 31) * R) >> 5;
+  const int rot = (lane * R) >> 5;
   float kv[R];
   uint32_t act = 0, took = 0;  // bit x = slot x
 #pragma unroll
   for (int x = 0; x < R; ++x) {
     const int j = j0 + ((x + rot) & (R - 1));
-    kv[x] = j < m ? keys[j] : 0.f;
+    kv[x] = lds_f32(keys_a + 4u * (uint32_t)min(j, m - 1));
     act |= (uint32_t)(j < m) << x;
   }
   uint32_t need = (uint32_t)kk;
-  uint32_t* wh = hist + warp * 256;
-  for (int iter = 0; iter < 8; ++iter) {
+  bool resolved = false;
+  const uint32_t hist_a = SC_ADDR(sc_a, hist);
+#pragma unroll 1
+  for (int iter = 0; iter < 6; ++iter) {
+    const int par = iter & 1;  // reduction slots alternate, so no barrier is needed between rounds
     float lo = INFINITY, hi = -INFINITY;
 #pragma unroll
     for (int x = 0; x < R; ++x) {
@@ -215,275 +530,262 @@ __device__ __forceinline__ void select_impl(const float* keys, int m, int kk, in
       lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
       hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
     }
-    if (lane == 0) {
-      ms.red[warp][0] = lo;
-      ms.red[warp][1] = hi;
-    }
+    if (lane == 0)
+      sts_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + warp), __float_as_uint(lo), __float_as_uint(hi));
 #pragma unroll
-    for (int i = 0; i < 8; ++i) wh[lane + 32 * i] = 0u;
-    __syncthreads();
+    for (int i = 0; i < BPT / 4; ++i) sts_v4(hist_a + 16u * (tid * (BPT / 4) + i), make_uint4(0, 0, 0, 0));
+    sts_u32(SC_ADDR(sc_a, bmap) + 4u * tid, 0u);
+    csync();
 #pragma unroll
-    for (int w = 0; w < 8; ++w) {
-      lo = fminf(lo, ms.red[w][0]);
-      hi = fmaxf(hi, ms.red[w][1]);
+    for (int w = 0; w < NCW; ++w) {
+      const uint2 r = lds_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + w));
+      lo = fminf(lo, __uint_as_float(r.x));
+      hi = fmaxf(hi, __uint_as_float(r.y));
     }
     if (!(hi > lo)) break;  // every undecided key is equal (or none is left)
-    const float scale = 256.f / (hi - lo);
-    int bk[R];
+    const float scale = (float)NB / (hi - lo);
 #pragma unroll
-    for (int x = 0; x < R; ++x) {
-      bk[x] = min(255, (int)((kv[x] - lo) * scale));
-      if ((act >> x) & 1u) atomicAdd(&wh[bk[x]], 1u);
+    for (int x = 0; x < R; ++x)
+      if ((act >> x) & 1u) reds_add(hist_a + 4u * bucket_of(kv[x], lo, scale), 1u);
+    csync();
+    // Thread tid owns buckets bhi, bhi - 1, ..., bhi - BPT + 1 (high to low).
+    const int bhi = NB - 1 - BPT * tid;
+    const uint32_t own_a = hist_a + 4u * (uint32_t)(bhi - BPT + 1);
+    uint32_t cw[BPT];
+#pragma unroll
+    for (int i = 0; i < BPT / 4; ++i) {
+      const uint4 v = lds_v4(own_a + 16u * i);
+      cw[4 * i] = v.x;
+      cw[4 * i + 1] = v.y;
+      cw[4 * i + 2] = v.z;
+      cw[4 * i + 3] = v.w;
     }
-    __syncthreads();
-    const int bin = 255 - tid;  // thread order = buckets from high to low
     uint32_t tot = 0;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) tot += hist[w * 256 + bin];
-    const uint32_t above = (uint32_t)block_excl_scan((int)tot, ms);
+    for (int i = 0; i < BPT; ++i) tot += cw[i];
+    const uint32_t above = (uint32_t)cta_excl_scan((int)tot, SC_ADDR(sc_a, wsum));
     if (above < need && above + tot >= need) {
-      ms.sel_bin = (uint32_t)bin;
-      ms.sel_need = need - above;
-      ms.sel_cnt = tot;
+      // This thread's buckets hold the boundary: walk them from high to low.
+      uint32_t acc = above, sb = 0, sneed = 0, scnt = 0;
+      bool found = false;
+#pragma unroll
+      for (int k = BPT - 1; k >= 0; --k) {  // cw[k] is bucket bhi - (BPT - 1 - k)
+        if (!found && acc + cw[k] >= need) {
+          sb = (uint32_t)(bhi - (BPT - 1 - k));
+          sneed = need - acc;
+          scnt = cw[k];
+          found = true;
+        }
+        acc += cw[k];
+      }
+      sts_v4(SC_ADDR(sc_a, ssel) + 16u * par, make_uint4(sb, sneed, scnt, 0));
+      sts_u32(SC_ADDR(sc_a, bcnt), 0u);
     }
-    __syncthreads();
-    const int sb = (int)ms.sel_bin;
-    const uint32_t cnt = ms.sel_cnt;
-    need = ms.sel_need;
+    csync();
+    const uint4 sel = lds_v4(SC_ADDR(sc_a, ssel) + 16u * par);
+    const int sb = (int)sel.x;
+    need = sel.y;
+    const uint32_t cnt = sel.z;
 #pragma unroll
     for (int x = 0; x < R; ++x) {
       if ((act >> x) & 1u) {
-        if (bk[x] > sb) took |= 1u << x;
-        if (bk[x] != sb) act &= ~(1u << x);
+        const int bk = bucket_of(kv[x], lo, scale);
+        if (bk > sb) took |= 1u << x;
+        if (bk != sb) act &= ~(1u << x);
       }
     }
-    __syncthreads();  // ms.red / ms.sel are reused by the next round
     if (cnt == need) {
       took |= act;
       act = 0;
+      resolved = true;
+      break;
+    }
+    if (cnt <= (uint32_t)NCT) {
+      // Exact rank of each boundary key among the cnt of them.  The keys are
+      // appended with one atomic per warp.
+      const int nb = __popc(act);
+      int incl = nb;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      uint32_t wbase = 0;
+      if (lane == 31 && incl > 0) wbase = atoms_add(SC_ADDR(sc_a, bcnt), (uint32_t)incl);
+      wbase = __shfl_sync(0xffffffffu, wbase, 31);
+      uint32_t slot = wbase + (uint32_t)(incl - nb);
+#pragma unroll
+      for (int x = 0; x < R; ++x) {
+        if ((act >> x) & 1u) {
+          sts_v2(SC_ADDR(sc_a, blist) + 8u * slot, __float_as_uint(kv[x]), (uint32_t)(j0 + ((x + rot) & (R - 1))));
+          ++slot;
+        }
+      }
+      csync();
+      if (tid < (int)cnt) {
+        const uint2 me = lds_v2(SC_ADDR(sc_a, blist) + 8u * tid);
+        const float km = __uint_as_float(me.x);
+        const int jm = (int)me.y;
+        uint32_t rank = 0;
+#pragma unroll 1
+        for (uint32_t v0 = 0; v0 < cnt; v0 += 4) {
+          uint2 o[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) o[k] = lds_v2(SC_ADDR(sc_a, blist) + 8u * min(v0 + k, cnt - 1));
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float ko = __uint_as_float(o[k].x);
+            rank += (v0 + k < cnt) && ((ko > km) || (ko == km && (int)o[k].y < jm));
+          }
+        }
+        if (rank < need) reds_or(SC_ADDR(sc_a, bmap) + 4u * (uint32_t)(jm >> 5), 1u << (jm & 31));
+      }
+      csync();
+#pragma unroll
+      for (int x = 0; x < R; ++x) {
+        if ((act >> x) & 1u) {
+          const int j = j0 + ((x + rot) & (R - 1));
+          if ((lds_u32(SC_ADDR(sc_a, bmap) + 4u * (uint32_t)(j >> 5)) >> (j & 31)) & 1u) took |= 1u << x;
+        }
+      }
+      act = 0;
+      resolved = true;
       break;
     }
   }
   // Position-order masks (bit i = position j0 + i).
-  uint32_t gt = 0, eq = 0;
+  uint32_t take = 0, eq = 0;
 #pragma unroll
   for (int x = 0; x < R; ++x) {
     const int i = (x + rot) & (R - 1);
-    gt |= ((took >> x) & 1u) << i;
+    take |= ((took >> x) & 1u) << i;
     eq |= ((act >> x) & 1u) << i;
   }
-  // The still-undecided (equal) keys: the first `need` by position are taken.
-  const int eq_base = block_excl_scan(__popc(eq), ms);
-  uint32_t take = gt;
-  int remaining = (int)need - eq_base;
-  for (uint32_t e = eq; e && remaining > 0; --remaining) {
-    const uint32_t low = e & (~e + 1u);
-    take |= low;
-    e ^= low;
-  }
-  int pos = block_excl_scan(__popc(take), ms);
-  while (take) {
-    const int i = __ffs(take) - 1;
-    take &= take - 1u;
-    Jout[pos++] = cand_of(j0 + i, top, Jprev);
-  }
-  __syncthreads();
-}
-
-__device__ __forceinline__ void select_topk(const float* keys, int m, int kk, int32_t* Jout, bool top,
-                                            const int32_t* Jprev, Misc& ms, uint32_t* hist) {
-  if (m <= NT) select_impl<1>(keys, m, kk, Jout, top, Jprev, ms, hist);
-  else if (m <= 2 * NT) select_impl<2>(keys, m, kk, Jout, top, Jprev, ms, hist);
-  else if (m <= 4 * NT) select_impl<4>(keys, m, kk, Jout, top, Jprev, ms, hist);
-  else if (m <= 8 * NT) select_impl<8>(keys, m, kk, Jout, top, Jprev, ms, hist);
-  else if (m <= 16 * NT) select_impl<16>(keys, m, kk, Jout, top, Jprev, ms, hist);
-  else select_impl<32>(keys, m, kk, Jout, top, Jprev, ms, hist);
-}
-
-// Per-CTA shared-memory addresses and constants.
-struct Ctx {
-  uint32_t tmem, sq_a, p_a, keys_a, done_a, stage_a, full_a, empty_a, pfull_a, pempty_a;
-  uint32_t rank, cs;
-  int stages, q;
-  float sl2;
-};
-
-// Where the rows of a candidate or key list come from.
-//  kind 0: position j -> row j (top scale);
-//  kind 1: position j -> row 2 J[j/2] + j%2 (children of the kept coefficients);
-//  kind 2: sparse key list, positions < kk -> token 2 J[j/2] + j%2 (or J[j]
-//          when trimmed), then generation rows.
-struct RowSrc {
-  const bf16* base;
-  int64_t stride;
-  const bf16* gbase;
-  int64_t gstride;
-  const int32_t* J;
-  int kind, trim, g0, mc, kk;
-};
-
-__device__ __forceinline__ const bf16* row_ptr(const RowSrc& s, int r) {
-  const int valid = r < s.mc;
-  const int pos = s.g0 + (valid ? r : 0);
-  int row;
-  if (s.kind == 0) {
-    row = pos;
-  } else if (s.kind == 1) {
-    row = 2 * s.J[pos >> 1] + (pos & 1);
-  } else {
-    if (pos >= s.kk) return s.gbase + (int64_t)(pos - s.kk) * s.gstride;
-    row = s.trim ? s.J[pos] : 2 * s.J[pos >> 1] + (pos & 1);
-  }
-  return s.base + (int64_t)row * s.stride;
-}
-
-__device__ __forceinline__ uint32_t stage_addr(const Ctx& c, int s) { return c.stage_a + s * TILE_BYTES; }
-
-__device__ __forceinline__ bool aborted(const Misc& ms) { return *reinterpret_cast<const volatile int*>(&ms.abort); }
-
-__device__ __forceinline__ void set_abort(Misc& ms, int* status) {
-  ms.abort = 1;
-  atomicExch(status, 1);
-}
-
-__device__ __forceinline__ void wait_or_abort(uint32_t bar, uint32_t parity, Misc& ms, int* status) {
-  if (!aborted(ms) && !mbar_wait_bounded(bar, parity, kWaitLimit, &ms.abort)) set_abort(ms, status);
-}
-
-// This thread's share of one 128-row tile: chunk c = tid % 16 of rows
-// tid/16 + 16 i, written in the 128-byte-swizzled K-major layout (row r,
-// 16-byte chunk c at half c/8, byte r*128 + ((c%8) ^ (r%8))*16).
-__device__ __forceinline__ void load_tile(uint32_t st, int t, const RowSrc& src) {
-  const int tid = threadIdx.x;
-  const int c = tid & 15, r0 = tid >> 4;
-  const uint32_t cbase = st + ((c >> 3) << 14);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int r = r0 + 16 * i;
-    cp_async16(cbase + r * 128 + (((c & 7) ^ (r & 7)) << 4), row_ptr(src, t * TM + r) + c * 8);
-  }
-}
-
-// Stream ntl tiles of src through the stage ring (pipeline iterations
-// it0..): all threads copy, thread 0 also issues the score MMAs
-// S^T tile = rows . Q^T into TMEM columns 32 t, then commits `done`.
-__device__ __forceinline__ void stream_scores(const Ctx& c, Misc& ms, int* status, int it0, int ntl, RowSrc src) {
-  const int tid = threadIdx.x;
-  const int S = c.stages;
-  for (int t = 0; t < ntl + S - 1; ++t) {
-    if (t < ntl) {
-      const int it = it0 + t, s = it % S, n = it / S;
-      if (n > 0) wait_or_abort(c.empty_a + 8 * s, (uint32_t)(n - 1) & 1u, ms, status);
-      load_tile(stage_addr(c, s), t, src);
-      cp_async_arrive_noinc(c.full_a + 8 * s);
-    }
-    const int tp = t - (S - 1);
-    if (tid == 0 && tp >= 0) {
-      const int it = it0 + tp, s = it % S, n = it / S;
-      wait_or_abort(c.full_a + 8 * s, (uint32_t)n & 1u, ms, status);
-      fence_proxy_async();
-      if (!aborted(ms)) {
-        tc_fence_after();
-        const uint32_t st = stage_addr(c, s);
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma_bf16(c.tmem + 32 * tp, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
-                     smem_desc(c.sq_a + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
-      }
-      mma_commit(c.empty_a + 8 * s);
+  if (!resolved) {
+    // Only equal keys are undecided: the first `need` by position are taken.
+    const int eq_base = cta_excl_scan(__popc(eq), SC_ADDR(sc_a, wsum));
+    int remaining = (int)need - eq_base;
+    for (uint32_t e = eq; e && remaining > 0; --remaining) {
+      const uint32_t low = e & (~e + 1u);
+      take |= low;
+      e ^= low;
     }
   }
-  if (tid == 0) mma_commit(c.done_a);
+  // Candidate indices of the winners (read before anything is written), then
+  // each at its output rank.  The scan's barriers order every thread's key
+  // reads before the key array is overwritten.
+  int cid[R];
+#pragma unroll
+  for (int x = 0; x < R; ++x) {
+    const int j = j0 + ((x + rot) & (R - 1));
+    cid[x] = (top || j >= m) ? j : (int)lds_u32(jprev_a + 4u * (uint32_t)(j >> 1));
+  }
+  const int base = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum));
+#pragma unroll
+  for (int x = 0; x < R; ++x) {
+    const int i = (x + rot) & (R - 1);
+    if ((take >> i) & 1u) {
+      const int j = j0 + i;
+      const int c = top ? j : 2 * cid[x] + (j & 1);
+      sts_u32(keys_a + 4u * (uint32_t)(base + __popc(take & ((1u << i) - 1u))), (uint32_t)c);
+    }
+  }
+  csync();
 }
 
-// Thread 0 waits (bounded) for phase `parity` of mbarrier `bar`; uniform.
-__device__ __forceinline__ void wait_all(uint32_t bar, uint32_t parity, Misc& ms, int* status) {
-  if (threadIdx.x == 0) wait_or_abort(bar, parity, ms, status);
-  __syncthreads();
-  tc_fence_after();
+// Top-K dispatch: 16 keys per compute thread up to 2048 candidates, else 32.
+__device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a) {
+  if (m <= 16 * NCT) select_reg<16>(keys_a, m, kk, jprev_a, top, sc_a);
+  else select_reg<32>(keys_a, m, kk, jprev_a, top, sc_a);
 }
 
 // Per-query max (x sl2, log2 units) of the valid rows of TMEM tiles
-// 0..ntl-1 -> ms.mloc.
-__device__ __forceinline__ void pass_max(const Ctx& c, Misc& ms, int ntl, int mc) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, qd = warp & 3, half = warp >> 2;
-  const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+// 0..ntl-1 of region tb -> us.mloc.
+__device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int ntl, int mc, float sl2) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   float mx[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) mx[i] = -INFINITY;
-  for (int t = half; t < ntl; t += 2) {
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
     uint32_t ra[32];
-    tmem_ld32_issue(c.tmem + lane_base + 32 * t, ra);
+    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    if (t * TM + qd * 32 + lane < mc) {
+    if (t * TM + tid < mc) {
 #pragma unroll
       for (int i = 0; i < 32; ++i) mx[i] = fmaxf(mx[i], __uint_as_float(ra[i]));
     }
   }
-  ms.red[warp][lane] = transpose_reduce32<true>(mx, lane);
-  __syncthreads();
+  us.red[warp][lane] = transpose_reduce32<true>(mx, lane);
+  csync();
   if (tid < 32) {
     float m = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) m = fmaxf(m, ms.red[w][tid]);
-    ms.mloc[tid] = m * c.sl2;
+    for (int w = 0; w < NCW; ++w) m = fmaxf(m, us.red[w][tid]);
+    us.mloc[tid] = m * sl2;
   }
-  __syncthreads();
+  csync();
 }
 
-// Per-query sum of 2^(l - mloc) over the valid rows; (mloc, sum) of this CTA
-// are written into slot `rank` of every cluster CTA's xstat.
-__device__ __forceinline__ void pass_sum(const Ctx& c, Misc& ms, int ntl, int mc) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, qd = warp & 3, half = warp >> 2;
-  const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+// Per-query sum of 2^(l - mloc) over the valid rows -> (mloc, sum) into slot
+// `rank` of every cluster CTA's xstat.
+__device__ __noinline__ void pass_sum(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
+                                      int ntl, int mc, float sl2) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   float ml[32], acc[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
-    ml[i] = ms.mloc[i];
+    ml[i] = us.mloc[i];
     acc[i] = 0.f;
   }
-  for (int t = half; t < ntl; t += 2) {
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
     uint32_t ra[32];
-    tmem_ld32_issue(c.tmem + lane_base + 32 * t, ra);
+    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    if (t * TM + qd * 32 + lane < mc) {
+    if (t * TM + tid < mc) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i) acc[i] += ex2(fmaf(__uint_as_float(ra[i]), c.sl2, -ml[i]));
+      for (int i = 0; i < 32; ++i) acc[i] += ex2(fmaf(__uint_as_float(ra[i]), sl2, -ml[i]));
     }
   }
-  ms.red[warp][lane] = transpose_reduce32<false>(acc, lane);
-  __syncthreads();
+  us.red[warp][lane] = transpose_reduce32<false>(acc, lane);
+  csync();
   if (tid < 32) {
     float sum = 0.f;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) sum += ms.red[w][tid];
-    const uint32_t local = smem_u32(&ms.xstat[c.rank][tid]);
-    for (uint32_t r = 0; r < c.cs; ++r) st_cluster_v2f32(map_rank(local, r), ms.mloc[tid], sum);
+    for (int w = 0; w < NCW; ++w) sum += us.red[w][tid];
+    const uint32_t dst = smem_u32(&us.xstat[rank][tid]);
+    const uint32_t bar = bar_addr(ms.xbar[pp]);
+#pragma unroll 1
+    for (uint32_t r = 0; r < cs; ++r)
+      st_async_v2(map_rank(dst, r), __float_as_uint(us.mloc[tid]), __float_as_uint(sum), map_rank(bar, r));
   }
 }
 
 // Ranking key log2 W_j of each valid row (Eq. 8 as a log-sum-exp over the
-// query rows, against the normaliser c_i in ms.cvec), written to position
-// g0 + j of every cluster CTA's key array.
-__device__ __forceinline__ void pass_keys(const Ctx& c, Misc& ms, int ntl, int mc, int g0) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, qd = warp & 3, half = warp >> 2;
-  const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+// query rows, against the normaliser c_i in us.cvec), stored at position
+// g0 + j of every cluster CTA's key array of the unit.
+__device__ __noinline__ void pass_keys(uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb, int ntl, int mc,
+                                       int g0, int q, float sl2, uint32_t keys_a) {
+  const int tid = ctid(), warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  const uint32_t bar = bar_addr(ms.kbar[pp]);
   float cv[32];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) cv[i] = ms.cvec[i];
-  const int q = c.q;
-  for (int t = half; t < ntl; t += 2) {
+  for (int i = 0; i < 32; ++i) cv[i] = us.cvec[i];
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
     uint32_t ra[32];
-    tmem_ld32_issue(c.tmem + lane_base + 32 * t, ra);
+    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    const int j = t * TM + qd * 32 + lane;
+    const int j = t * TM + tid;
     float v[32];
     float mx = -INFINITY;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
-      v[i] = fmaf(__uint_as_float(ra[i]), c.sl2, -cv[i]);
+      v[i] = fmaf(__uint_as_float(ra[i]), sl2, -cv[i]);
       if (i < q) mx = fmaxf(mx, v[i]);
     }
     float z = 0.f;
@@ -492,193 +794,299 @@ __device__ __forceinline__ void pass_keys(const Ctx& c, Misc& ms, int ntl, int m
       if (i < q) z += ex2(v[i] - mx);
     const float key = mx + lg2(z);
     if (j < mc) {
-      const uint32_t local = c.keys_a + 4u * (uint32_t)(g0 + j);
-      for (uint32_t r = 0; r < c.cs; ++r) st_cluster_f32(map_rank(local, r), key);
+      const uint32_t dst = keys_a + 4u * (uint32_t)(g0 + j);
+#pragma unroll 1
+      for (uint32_t r = 0; r < cs; ++r) st_async_b32(map_rank(dst, r), __float_as_uint(key), map_rank(bar, r));
     }
   }
 }
 
-// Attention phase 2: every thread streams the V rows; warps 4-7 write
-// P = 2^(s - m) (bf16, P^T MN-major) and accumulate its row sums into
-// ms.lacc; thread 0 accumulates O^T += V_s^T P^T in TMEM column ocol.
-__device__ __forceinline__ void attn_pv(const Ctx& c, Misc& ms, int* status, int it_v, int ntl, RowSrc src,
-                                     uint32_t ocol, uint8_t* pbase) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, qd = warp & 3;
-  const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
-  const int S = c.stages;
+// Attention: P = 2^(s - m) (bf16, P^T MN-major core matrices) of every S tile
+// into the unit's P double buffer for the MMA thread, and the row sums of P
+// -> us.lacc.
+__device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* pbase, UnitState& us, int pp,
+                                    uint32_t tb, int ntl, int mc) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   float ml[32], lsum[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
-    ml[i] = ms.mloc[i];
+    ml[i] = us.mloc[i];
     lsum[i] = 0.f;
   }
-  for (int t = 0; t < ntl + S - 1; ++t) {
-    if (t < ntl) {
-      const int itv = it_v + t, s = itv % S, n = itv / S;
-      if (n > 0) wait_or_abort(c.empty_a + 8 * s, (uint32_t)(n - 1) & 1u, ms, status);
-      load_tile(stage_addr(c, s), t, src);
-      cp_async_arrive_noinc(c.full_a + 8 * s);
-    }
-    const int tp = t - (S - 1);
-    if (tp < 0) continue;
-    const int pb = tp & 1, pn = tp >> 1;
-    if (warp >= 4) {
-      if (tp >= 2) {
-        if (lane == 0) wait_or_abort(c.pempty_a + 8 * pb, (uint32_t)(pn - 1) & 1u, ms, status);
-        __syncwarp();
-      }
-      uint32_t ra[32];
-      tmem_ld32_issue(c.tmem + lane_base + 32 * tp, ra);
-      tmem_wait_ld();
-      const int r = qd * 32 + lane;
-      const bool ok = tp * TM + r < src.mc;
-      uint32_t w[16];
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        const float p0 = ok ? ex2(fmaf(__uint_as_float(ra[i]), c.sl2, -ml[i])) : 0.f;
-        const float p1 = ok ? ex2(fmaf(__uint_as_float(ra[i + 1]), c.sl2, -ml[i + 1])) : 0.f;
-        const __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
-        lsum[i] += __low2float(h2);
-        lsum[i + 1] += __high2float(h2);
-        w[i / 2] = *reinterpret_cast<const uint32_t*>(&h2);
-      }
-      // P^T, MN-major core matrices: key group r / 8, query chunk c.
-      uint8_t* dst = pbase + pb * P_BYTES + (r >> 3) * 512 + (r & 7) * 16;
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch)
-        *reinterpret_cast<uint4*>(dst + ch * 128) =
-            make_uint4(w[4 * ch], w[4 * ch + 1], w[4 * ch + 2], w[4 * ch + 3]);
-      fence_proxy_async();
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
+    const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
+    if (t >= 2) {
+      if (lane == 0) wait_or_abort(bar_addr(ms.pempty[pp][pb]), (pn - 1) & 1u, ms, status);
       __syncwarp();
-      if (lane == 0) mbar_arrive(c.pfull_a + 8 * pb);
     }
-    if (tid == 0) {
-      const int itv = it_v + tp, s = itv % S, n = itv / S;
-      wait_or_abort(c.full_a + 8 * s, (uint32_t)n & 1u, ms, status);
-      wait_or_abort(c.pfull_a + 8 * pb, (uint32_t)pn & 1u, ms, status);
-      fence_proxy_async();
-      if (!aborted(ms)) {
-        tc_fence_after();
-        const uint32_t st = stage_addr(c, s);
+    uint32_t ra[32];
+    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
+    tmem_wait_ld();
+    const bool ok = t * TM + tid < mc;
+    uint32_t w[16];
 #pragma unroll
-        for (int kq = 0; kq < TM / 16; ++kq)
-          mma_bf16(c.tmem + ocol, smem_desc_sw128(st + kq * 2048, HALF_BYTES, 1024),
-                   smem_desc(c.p_a + pb * P_BYTES + kq * 1024, 512, 128), kIdescPV, (tp > 0 || kq > 0) ? 1u : 0u);
-      }
-      mma_commit(c.empty_a + 8 * s);
-      mma_commit(c.pempty_a + 8 * pb);
+    for (int i = 0; i < 32; i += 2) {
+      const float p0 = ok ? ex2(fmaf(__uint_as_float(ra[i]), sl2, -ml[i])) : 0.f;
+      const float p1 = ok ? ex2(fmaf(__uint_as_float(ra[i + 1]), sl2, -ml[i + 1])) : 0.f;
+      const __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+      lsum[i] += __low2float(h2);
+      lsum[i + 1] += __high2float(h2);
+      w[i / 2] = *reinterpret_cast<const uint32_t*>(&h2);
     }
+    // P^T, MN-major core matrices: key group r / 8, query chunk ch.
+    const int r = tid;
+    uint8_t* dst = pbase + pb * P_BYTES + (r >> 3) * 512 + (r & 7) * 16;
+#pragma unroll
+    for (int ch = 0; ch < 4; ++ch)
+      *reinterpret_cast<uint4*>(dst + ch * 128) = make_uint4(w[4 * ch], w[4 * ch + 1], w[4 * ch + 2], w[4 * ch + 3]);
+    fence_proxy_async();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_addr(ms.pfull[pp][pb]));
   }
-  if (tid == 0) mma_commit(c.done_a);
-  if (warp >= 4) ms.red[warp][lane] = transpose_reduce32<false>(lsum, lane);
-  __syncthreads();
+  us.red[warp][lane] = transpose_reduce32<false>(lsum, lane);
+  csync();
   if (tid < 32) {
     float sum = 0.f;
 #pragma unroll
-    for (int w = 4; w < 8; ++w) sum += ms.red[w][tid];
-    ms.lacc[tid] = sum;
+    for (int w = 0; w < NCW; ++w) sum += us.red[w][tid];
+    us.lacc[tid] = sum;
   }
+  csync();
 }
 
-// Partial O^T of this CTA -> CTA 0, which combines the cluster's partials and
-// writes O (bf16).
-__device__ __forceinline__ void attn_combine(const Ctx& c, Misc& ms, const FusedParams& p, int64_t bb, int64_t hh,
-                                          uint32_t ocol, const float* part_base) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, qd = warp & 3;
-  const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+// Attention combine of unit pp: this CTA's partial O^T rows go to the CTA
+// owning their head-dim slice (with the CTA's (m, l) per query), and this
+// CTA combines the cluster's partials of its own slice and writes those
+// columns of O (bf16).  The partials land in each owner's P buffers of the
+// unit, which are free once the owner's own PV products are done; owners
+// announce that before any partial is sent.
+__device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32_t rank, uint32_t cs, int u,
+                                          uint8_t* comb, UnitState& us, int pp, uint32_t ocol) {
+  const int tid = ctid(), warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   uint32_t orow[32];
-  if (warp >= 4) {
-    tmem_ld32_issue(c.tmem + lane_base + ocol, orow);
-    tmem_wait_ld();
+  tmem_ld32_issue(ocol + lane_base, orow);
+  tmem_wait_ld();
+  const uint32_t ready = bar_addr(ms.cready[pp]);
+  if (tid == 0) {
+#pragma unroll 1
+    for (uint32_t r = 0; r < cs; ++r) mbar_arrive_cluster(map_rank(ready, r));
   }
-  tc_fence_before();
-  cluster_sync();
-  const uint32_t recv = c.stage_a;
-  if (warp >= 4) {
-    const int d = qd * 32 + lane;
-    const uint32_t dst = map_rank(recv + 4u * (uint32_t)((c.rank * D + d) * NQ), 0);
+  wait_cluster_or_abort(ready, 0u, ms, p.status);
+  const int rows = D / (int)cs;
+  const uint32_t comb_a = smem_u32(comb);
+  const uint32_t cbar = bar_addr(ms.cbar[pp]);
+  {
+    const uint32_t owner = (uint32_t)(tid / rows);
+    const int dl = tid % rows;
+    const uint32_t dst = map_rank(comb_a + 4u * (uint32_t)((rank * rows + dl) * NQ), owner);
+    const uint32_t rb = map_rank(cbar, owner);
 #pragma unroll
-    for (int i = 0; i < 32; i += 4)
-      st_cluster_v4f32(dst + 4u * i, __uint_as_float(orow[i]), __uint_as_float(orow[i + 1]),
-                       __uint_as_float(orow[i + 2]), __uint_as_float(orow[i + 3]));
+    for (int i = 0; i < 32; i += 4) st_async_v4(dst + 4u * i, orow[i], orow[i + 1], orow[i + 2], orow[i + 3], rb);
   }
   if (tid < 32) {
-    const uint32_t ml_a = recv + 4u * (uint32_t)(c.cs * NQ * D) + 8u * (c.rank * NQ + tid);
-    st_cluster_v2f32(map_rank(ml_a, 0), ms.mloc[tid], ms.lacc[tid]);
+    const uint32_t dst = smem_u32(&us.cstat[rank][tid]);
+#pragma unroll 1
+    for (uint32_t r = 0; r < cs; ++r)
+      st_async_v2(map_rank(dst, r), __float_as_uint(us.mloc[tid]), __float_as_uint(us.lacc[tid]),
+                  map_rank(cbar, r));
   }
-  cluster_sync();
-  if (c.rank == 0) {
-    const float2* mlp = reinterpret_cast<const float2*>(part_base + c.cs * NQ * D);
-    bf16* ob = p.O + bb * p.osb + hh * p.osh;
-    for (int e = tid; e < NQ * D; e += NT) {
-      const int qi = e % NQ, d = e / NQ;
-      if (qi >= c.q) continue;
-      float M = -INFINITY;
-      for (uint32_t r = 0; r < c.cs; ++r)
-        if (mlp[r * NQ + qi].y > 0.f) M = fmaxf(M, mlp[r * NQ + qi].x);
-      float num = 0.f, den = 0.f;
-      for (uint32_t r = 0; r < c.cs; ++r) {
-        const float2 x = mlp[r * NQ + qi];
-        if (!(x.y > 0.f)) continue;  // a CTA with no keys sent no partial output
-        const float f = ex2(x.x - M);
-        num = fmaf(part_base[(r * D + d) * NQ + qi], f, num);
-        den = fmaf(x.y, f, den);
+  wait_cluster_or_abort(cbar, 0u, ms, p.status);
+  // A thread always serves query qi = tid % 32: the weight 2^(m_r - M) of
+  // every source CTA and the denominator are formed once.
+  const int qi = tid & (NQ - 1);
+  const uint32_t cst_a = smem_u32(&us.cstat[0][qi]);
+  float2 st[MAXCS];
+#pragma unroll
+  for (int r = 0; r < MAXCS; ++r) {
+    const uint2 v = lds_v2(cst_a + (uint32_t)(min(r, (int)cs - 1) * NQ * 8));
+    st[r] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+  }
+  float M = -INFINITY;
+#pragma unroll
+  for (int r = 0; r < MAXCS; ++r)
+    if (r < (int)cs && st[r].y > 0.f) M = fmaxf(M, st[r].x);
+  float f[MAXCS], den = 0.f;
+#pragma unroll
+  for (int r = 0; r < MAXCS; ++r) {
+    f[r] = (r < (int)cs && st[r].y > 0.f) ? ex2(st[r].x - M) : 0.f;  // a CTA with no keys contributes nothing
+    den = fmaf(st[r].y, f[r], den);
+  }
+  const float inv = 1.f / den;
+  bf16* ob = p.O + (int64_t)(u / p.H) * p.osb + (int64_t)(u % p.H) * p.osh;
+  if (qi < p.q) {
+#pragma unroll 1
+    for (int dp = tid >> 5; dp < rows / 2; dp += NCT / NQ) {
+      float n0 = 0.f, n1 = 0.f;
+#pragma unroll
+      for (int r = 0; r < MAXCS; ++r) {
+        if (r < (int)cs) {
+          const uint32_t a = comb_a + 4u * (uint32_t)((r * rows + 2 * dp) * NQ + qi);
+          n0 = fmaf(lds_f32(a), f[r], n0);
+          n1 = fmaf(lds_f32(a + 4u * NQ), f[r], n1);
+        }
       }
-      ob[(int64_t)qi * p.oss + d] = __float2bfloat16_rn(num / den);
+      const int d = (int)rank * rows + 2 * dp;
+      *reinterpret_cast<__nv_bfloat162*>(ob + (int64_t)qi * p.oss + d) = __floats2bfloat162_rn(n0 * inv, n1 * inv);
     }
   }
 }
 
-template <int STAGES>
-__global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__ FusedParams p) {
-  using LY = Layout<STAGES>;
-  extern __shared__ __align__(1024) uint8_t smem[];
-  Misc& ms = *reinterpret_cast<Misc*>(smem + LY::off_misc);
-  uint32_t* hist = reinterpret_cast<uint32_t*>(smem + LY::off_hist);
-  float* keys = reinterpret_cast<float*>(smem + LY::off_keys);
-  int32_t* const J0 = reinterpret_cast<int32_t*>(smem + LY::off_keys + 4 * p.cmax);
-  int32_t* const J1 = J0 + p.kmax;
+// The compute warps of unit pp = threadIdx.x / NCT of the cluster's units.
+__device__ void compute_role(const Ctx& c, const FusedParams& p) {
+  Misc& ms = *c.ms;
+  const int tid = ctid();
+  const int pp = threadIdx.x / NCT;
+  if (pp >= c.np) return;
+  UnitState& us = ms.us[pp];
+  uint8_t* ubuf = c.smem + c.ly.p + pp * UNIT_P_BYTES;  // P buffers, Top-K scratch, combine buffer
+  const uint32_t sc_a = smem_u32(ubuf);
+  const uint32_t tb = c.tmem + pp * p.ucols;
+  const int u = c.u0 + pp;
+  const float sl2 = p.scale_log2;
+  int64_t sets_off = 0;
+  // Parity of the unit's next mdone phase.  The MMA thread commits a phase
+  // only for a non-empty stream, and every such stream waits on these warps'
+  // progress (through the producers' copies or the P tiles), so it is never
+  // two phases ahead.
+  uint32_t mdp = 0;
+  auto wait_mdone = [&]() {
+    wait_or_abort(bar_addr(ms.mdone[pp]), mdp, ms, p.status);
+    mdp ^= 1u;
+    tc_fence_after();
+  };
+#pragma unroll 1
+  for (int lev = p.L; lev >= c.lev_end; --lev) {
+    const uint32_t ph = (uint32_t)(p.L - lev) & 1u;  // phase of the per-scale barriers
+    const int m = m_total(p, lev);
+    int g0, mc;
+    scale_slice(m, c.rank, c.cs, g0, mc);
+    const int ntl = tiles_of(mc);
+    const int kb = p.keep[lev];
+    int32_t* J = unit_J(c, p, pp, lev);  // receives this scale's keys, then its selection
+    const uint32_t keys_a = smem_u32(J);
+    if (ntl > 0) wait_mdone();
+    pass_max(ms, us, tb, ntl, mc, sl2);
+    pass_sum(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2);
+    wait_cluster_or_abort(bar_addr(ms.xbar[pp]), ph, ms, p.status);
+    // Softmax normaliser per query: c = M + log2 S over the whole candidate set.
+    if (tid < 32) {
+      const uint32_t xs_a = smem_u32(&us.xstat[0][tid]);
+      float2 st[MAXCS];
+#pragma unroll
+      for (int r = 0; r < MAXCS; ++r) {
+        const uint2 v = lds_v2(xs_a + (uint32_t)(min(r, (int)c.cs - 1) * NQ * 8));
+        st[r] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+      }
+      float M = -INFINITY;
+#pragma unroll
+      for (int r = 0; r < MAXCS; ++r)
+        if (r < (int)c.cs && st[r].y > 0.f) M = fmaxf(M, st[r].x);
+      float S = 0.f;
+#pragma unroll
+      for (int r = 0; r < MAXCS; ++r)
+        if (r < (int)c.cs && st[r].y > 0.f) S += st[r].y * ex2(st[r].x - M);
+      us.cvec[tid] = M + lg2(S);
+    }
+    csync();
+    if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
+    pass_keys(c.cs, ms, us, pp, tb, ntl, mc, g0, p.q, sl2, keys_a);
+    wait_cluster_or_abort(bar_addr(ms.kbar[pp]), ph, ms, p.status);
+    // Eq. 9: Top-K (the same result in every CTA of the cluster).
+    select_topk(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a);
+    if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, lev - 1));
+    if (c.rank == 0) {
+      int32_t* ls = p.level_sets ? p.level_sets + (int64_t)u * p.sets_stride + sets_off : nullptr;
+      if (lev >= 1 && ls) {
+#pragma unroll 1
+        for (int i = tid; i < kb; i += NCT) ls[i] = J[i];
+      }
+      if (lev == c.lev_end) {
+        // mu^0: the children of J^1, or the trimmed level-0 selection.
+        const int kk = p.keep[0];
+        int32_t* out = p.idx + (int64_t)u * kk;
+        int32_t* ls0 = ls ? ls + (lev >= 1 ? kb : 0) : nullptr;
+#pragma unroll 1
+        for (int t = tid; t < kk; t += NCT) {
+          const int tok = p.trim ? J[t] : 2 * J[t >> 1] + (t & 1);
+          out[t] = tok;
+          if (ls0) ls0[t] = tok;
+        }
+      }
+    }
+    tc_fence_before();
+    csync();
+    if (tid == 0) mbar_arrive(bar_addr(ms.jready[pp]));
+    if (lev >= 1) sets_off += kb;
+  }
 
+  // Attention: S of the key slice, P for the MMA thread, then the combine.
+  int a0, mc;
+  attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
+  const int ntl = tiles_of(mc);
+  if (ntl > 0) wait_mdone();
+  pass_max(ms, us, tb, ntl, mc, sl2);
+  attn_p(ms, p.status, sl2, ubuf, us, pp, tb, ntl, mc);
+  if (ntl > 0) wait_mdone();
+  attn_combine(ms, p, c.rank, c.cs, u, ubuf, us, pp, tb + p.ucols - 32);
+}
+
+template <int S>
+__global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__ FusedParams p) {
+  extern __shared__ __align__(1024) uint8_t smem[];
   Ctx c;
-  c.sq_a = smem_u32(smem + LY::off_q);
-  c.p_a = smem_u32(smem + LY::off_p);
-  c.keys_a = smem_u32(keys);
-  c.done_a = smem_u32(&ms.done);
-  c.stage_a = smem_u32(smem + LY::off_stage);
-  c.full_a = smem_u32(&ms.full[0]);
-  c.empty_a = smem_u32(&ms.empty[0]);
-  c.pfull_a = smem_u32(&ms.pfull[0]);
-  c.pempty_a = smem_u32(&ms.pempty[0]);
+  c.smem = smem;
+  c.ly = smem_layout(S, p.P, p.cmax, p.kmax);
+  c.ms = reinterpret_cast<Misc*>(smem + c.ly.misc);
+  Misc& ms = *c.ms;
   c.rank = cluster_rank();
   c.cs = cluster_size();
-  c.stages = STAGES;
-  c.q = p.q;
-  c.sl2 = p.scale_log2;
-  const int u = (int)cluster_id_x();
-  const int64_t bb = u / p.H, hh = u % p.H;
+  c.u0 = (int)cluster_id_x() * p.P;
+  c.np = min(p.P, p.U - c.u0);
+  c.lev_end = p.trim ? 0 : 1;
+  c.stages = S;
   const int tid = threadIdx.x, warp = tid >> 5;
 
   if (tid == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(c.full_a + 8 * s, NT);
-      mbar_init(c.empty_a + 8 * s, 1);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(bar_addr(ms.full[s]), NPT);
+      mbar_init(bar_addr(ms.empty[s]), 1);
     }
-    mbar_init(c.done_a, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(c.pfull_a + 8 * i, 4);
-      mbar_init(c.pempty_a + 8 * i, 1);
+    for (int pp = 0; pp < MAXP; ++pp) {
+      mbar_init(bar_addr(ms.mdone[pp]), 1);
+      mbar_init(bar_addr(ms.jready[pp]), 1);
+      mbar_init(bar_addr(ms.xbar[pp]), 1);
+      mbar_init(bar_addr(ms.kbar[pp]), 1);
+    }
+    for (int pp = 0; pp < MAXP; ++pp) {
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(bar_addr(ms.pfull[pp][i]), NCW);
+        mbar_init(bar_addr(ms.pempty[pp][i]), 1);
+      }
+      mbar_init(bar_addr(ms.cbar[pp]), 1);
+      mbar_init(bar_addr(ms.cready[pp]), c.cs);
     }
     ms.abort = 0;
     fence_mbar_init();
+    // Arm the first phase of every receive barrier (bytes this CTA expects).
+    for (int pp = 0; pp < c.np; ++pp) {
+      mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
+      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)(p.n >> p.L));
+      mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), COMB_BYTES + c.cs * NQ * 8u);
+    }
   }
-  if (warp == 0) {
+  if (warp == MMA_WARP) {
     tmem_alloc(smem_u32(&ms.tmem_base), p.tmem_cols);
     tmem_relinquish();
   }
-  // Query block -> shared memory, K-major core matrices, rows >= q zero.
-  {
-    const bf16* qb = p.Q + bb * p.qsb + hh * p.qsh;
-    uint8_t* sq = smem + LY::off_q;
+  // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
+  for (int pp = 0; pp < c.np; ++pp) {
+    const int u = c.u0 + pp;
+    const bf16* qb = p.Q + (int64_t)(u / p.H) * p.qsb + (int64_t)(u % p.H) * p.qsh;
+    uint8_t* sq = smem + c.ly.q + pp * Q_BYTES;
     for (int e = tid; e < NQ * (D / 8); e += NT) {
       const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
       const int i = g * 8 + rr;
@@ -692,128 +1100,26 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   __syncthreads();
   tc_fence_after();
   c.tmem = ms.tmem_base;
-  cluster_sync();
+  cluster_sync();  // every CTA's barriers exist before any remote arrival
 
-  const int L = p.L;
-  int m_total = p.n >> L;
-  bool top = true;
-  bool jsel = false;  // false: the current level writes J0
-  const int32_t* Jprev = J1;
-  int64_t sets_off = 0;
-  int it = 0;             // pipeline iteration counter (uniform)
-  uint32_t done_cnt = 0;  // completions of `done` so far (uniform)
-  const int lev_end = p.trim ? 0 : 1;
-  const int64_t krow_off = bb * p.ksb + hh * p.ksh;
-
-  for (int lev = L; lev >= lev_end; --lev) {
-    // This CTA's slice of the candidate positions (pairs kept together).
-    const int pairs = (m_total + 1) >> 1;
-    const int g0 = min(m_total, 2 * (int)((int64_t)c.rank * pairs / c.cs));
-    const int g1 = min(m_total, 2 * (int)((int64_t)(c.rank + 1) * pairs / c.cs));
-    const int mc = g1 - g0;
-    const int ntl = (mc + TM - 1) / TM;
-    RowSrc src;
-    src.base = lev >= 1 ? p.coeffs + ((int64_t)u * p.rows_total + ((int64_t)p.n - ((int64_t)p.n >> (lev - 1)))) * D
-                        : p.K + krow_off;
-    src.stride = lev >= 1 ? D : p.kss;
-    src.gbase = nullptr;
-    src.gstride = 0;
-    src.J = Jprev;
-    src.kind = top ? 0 : 1;
-    src.trim = 0;
-    src.g0 = g0;
-    src.mc = mc;
-    src.kk = 0;
-    stream_scores(c, ms, p.status, it, ntl, src);
-    wait_all(c.done_a, done_cnt & 1u, ms, p.status);
-    ++done_cnt;
-    it += ntl;
-
-    pass_max(c, ms, ntl, mc);
-    pass_sum(c, ms, ntl, mc);
-    cluster_sync();
-    // Softmax normaliser per query: c = M + log2 S over the whole candidate set.
-    if (tid < 32) {
-      float M = -INFINITY;
-      for (uint32_t r = 0; r < c.cs; ++r)
-        if (ms.xstat[r][tid].y > 0.f) M = fmaxf(M, ms.xstat[r][tid].x);
-      float S = 0.f;
-      for (uint32_t r = 0; r < c.cs; ++r) {
-        const float2 x = ms.xstat[r][tid];
-        if (x.y > 0.f) S += x.y * ex2(x.x - M);
-      }
-      ms.cvec[tid] = M + lg2(S);
-    }
-    __syncthreads();
-    pass_keys(c, ms, ntl, mc, g0);
-    tc_fence_before();
-    cluster_sync();
-    tc_fence_after();
-
-    // Eq. 9: Top-K (same result in every CTA of the cluster).
-    const int kb = p.keep[lev];
-    int32_t* Jcur = jsel ? J1 : J0;
-    select_topk(keys, m_total, kb, Jcur, top, Jprev, ms, hist);
-    if (lev >= 1) {
-      if (c.rank == 0 && p.level_sets) {
-        int32_t* out = p.level_sets + (int64_t)u * p.sets_stride + sets_off;
-        for (int i = tid; i < kb; i += NT) out[i] = Jcur[i];
-      }
-      sets_off += kb;
-    }
-    Jprev = Jcur;
-    jsel = !jsel;
-    m_total = 2 * kb;  // Eq. 10: children of the kept coefficients
-    top = false;
+  if (warp < MMA_WARP) {
+    compute_role(c, p);
+  } else if (warp == MMA_WARP) {
+    if ((tid & 31) == 0) mma_role<S>(c, p);
+    __syncwarp();
+  } else {
+    producer_role<S>(c, p);
   }
 
-  // mu^0 and the sparse key list [K[mu^0]; Kg].
-  const int kk = p.keep[0];
-  const int32_t* Jfin = Jprev;
-  const bool trim = p.trim != 0;
-  if (c.rank == 0) {
-    int32_t* out = p.idx + (int64_t)u * kk;
-    int32_t* ls = p.level_sets ? p.level_sets + (int64_t)u * p.sets_stride + sets_off : nullptr;
-    for (int t = tid; t < kk; t += NT) {
-      const int tok = trim ? Jfin[t] : 2 * Jfin[t >> 1] + (t & 1);
-      out[t] = tok;
-      if (ls) ls[t] = tok;
-    }
-  }
-  const int total = kk + p.ng;
-  const int a0 = (int)((int64_t)c.rank * total / c.cs);
-  const int a1 = (int)((int64_t)(c.rank + 1) * total / c.cs);
-  const int mc = a1 - a0;
-  const int ntl = (mc + TM - 1) / TM;
-  const uint32_t ocol = p.tmem_cols - 32;
-  RowSrc src;
-  src.base = p.K + krow_off;
-  src.stride = p.kss;
-  src.gbase = p.Kg + (bb * p.gsb + hh * p.gsh);
-  src.gstride = p.gss;
-  src.J = Jfin;
-  src.kind = 2;
-  src.trim = trim ? 1 : 0;
-  src.g0 = a0;
-  src.mc = mc;
-  src.kk = kk;
-
-  // Attention phase 1: S^T = K_s Q^T and the per-query max (log2 units).
-  stream_scores(c, ms, p.status, it, ntl, src);
-  wait_all(c.done_a, done_cnt & 1u, ms, p.status);
-  ++done_cnt;
-  pass_max(c, ms, ntl, mc);
-
-  // Attention phase 2: O^T = V_s^T P^T.
-  src.base = p.V + krow_off;
-  src.gbase = p.Vg + (bb * p.gsb + hh * p.gsh);
-  attn_pv(c, ms, p.status, it + ntl, ntl, src, ocol, smem + LY::off_p);
-  wait_all(c.done_a, done_cnt & 1u, ms, p.status);
-  ++done_cnt;
-  attn_combine(c, ms, p, bb, hh, ocol, reinterpret_cast<const float*>(smem + LY::off_stage));
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(c.tmem, p.tmem_cols);
+  // No CTA leaves while another may still address its shared memory.
+  cluster_arrive();
+  cluster_wait();
+  if (warp == MMA_WARP) {
+    tc_fence_after();
+    tmem_dealloc(c.tmem, p.tmem_cols);
+  }
 }
 
 }  // namespace
@@ -821,6 +1127,49 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
 // ---------------------------------------------------------------------------
 // Host side.
 // ---------------------------------------------------------------------------
+namespace {
+
+// How many clusters of cs CTAs (with `smem` bytes each) can be resident at
+// once on the current device; cached per configuration.
+int max_active_clusters(int stages, int cs, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, int, int, size_t>, int> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  const auto key = std::make_tuple(dev, stages, cs, smem);
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)cs, 1, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  cudaError_t e;
+  if (stages == 4) {
+    e = cudaFuncSetAttribute(wf_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<4>, &cfg);
+  } else {
+    e = cudaFuncSetAttribute(wf_fused_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<3>, &cfg);
+  }
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    n = 0;
+  }
+  cache.emplace(key, n);
+  return n;
+}
+
+}  // namespace
+
 FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int n_g,
                      const wf_tensor* g, int num_sms) {
   (void)g;
@@ -833,9 +1182,11 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
   int cmax = n >> levels, kmax = 0;
   for (int l = 0; l <= levels; ++l) kmax = kmax > keep[l] ? kmax : keep[l];
   for (int l = 1; l <= levels; ++l) cmax = cmax > 2 * keep[l] ? cmax : 2 * keep[l];
-  if (cmax > 8192 || kmax > 8192) return fp;
+  if (cmax > kMaxCand || kmax > kMaxCand) return fp;
   const int total = keep[0] + n_g;
-  auto tiles_ok = [&](int cs, int* cols) {
+  // TMEM columns of one unit's region at cluster size cs: the widest scale
+  // slice, or the attention slice plus the O^T accumulator.
+  auto unit_cols = [&](int cs) {
     auto slice_tiles = [&](int m) { return (2 * (((m + 1) / 2 + cs - 1) / cs) + TM - 1) / TM; };
     int tmax = slice_tiles(n >> levels);
     for (int l = levels; l >= 1; --l) {
@@ -844,31 +1195,40 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
     }
     const int ta = ((total + cs - 1) / cs + TM - 1) / TM + 1;
     tmax = tmax > ta ? tmax : ta;
-    int c = 32;
-    while (c < 32 * tmax) c *= 2;
-    *cols = c;
-    return 32 * tmax <= 512;
+    return 32 * tmax;
   };
-  int cs = 1, cols = 0;
-  while (cs < 4 && (!tiles_ok(cs, &cols) || U * cs * 2 <= num_sms)) cs *= 2;
-  if (!tiles_ok(cs, &cols)) return fp;
+  // Two units per cluster (copies of one overlap the other's exchanges and
+  // Top-K) unless that leaves most SMs idle; the largest cluster that still
+  // fits the grid in one wave.
+  const int P = (U >= 2 && U * MAXCS > num_sms) ? 2 : 1;
+  const int clusters = (U + P - 1) / P;
   const size_t kMaxSmem = 227 * 1024;
-  const size_t tail = 4 * (size_t)cmax + 8 * (size_t)kmax;
   int stages = 4;
-  if (Layout<4>::off_keys + tail > kMaxSmem) stages = 3;
-  const size_t smem = (stages == 4 ? Layout<4>::off_keys : Layout<3>::off_keys) + tail;
+  if (smem_layout(4, P, cmax, kmax).total > kMaxSmem) stages = 3;
+  const size_t smem = smem_layout(stages, P, cmax, kmax).total;
   if (smem > kMaxSmem) return fp;
-  // CTA 0 receives every partial output in its stage area.
-  if ((size_t)cs * (NQ * D * 4 + NQ * 8) > (size_t)stages * TILE_BYTES) return fp;
+  int cs = 1;
+  while (cs < MAXCS && clusters * cs * 2 <= num_sms) cs *= 2;
+  while (cs < MAXCS && P * unit_cols(cs) > 512) cs *= 2;
+  if (P * unit_cols(cs) > 512) return fp;
+  // Prefer a smaller cluster over a second wave when the chosen one does not
+  // fit the SMs of its GPCs all at once.
+  while (cs > 1 && P * unit_cols(cs / 2) <= 512 && clusters > max_active_clusters(stages, cs, smem)) cs /= 2;
+  const int ucols = unit_cols(cs);
+  int cols = 32;
+  while (cols < P * ucols) cols *= 2;
   fp.ok = true;
   fp.cs = cs;
+  fp.P = P;
   fp.stages = stages;
   fp.smem = smem;
   fp.tmem_cols = cols;
+  fp.ucols = ucols;
   fp.cmax = cmax;
   fp.kmax = kmax;
   fp.trim = trim;
   fp.U = U;
+  fp.clusters = clusters;
   return fp;
 }
 
@@ -896,14 +1256,17 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   for (int l = 0; l <= levels; ++l) stride += keep[l];
   p.sets_stride = stride;
   p.status = status;
-  p.q = qd.seq; p.n = kv.seq; p.ng = g ? g->seq : 0; p.H = kv.heads; p.L = levels; p.trim = fp.trim ? 1 : 0;
+  p.q = qd.seq; p.n = kv.seq; p.ng = g ? g->seq : 0; p.U = fp.U; p.H = kv.heads; p.L = levels;
+  p.trim = fp.trim ? 1 : 0;
+  p.P = fp.P;
   p.cmax = fp.cmax; p.kmax = fp.kmax;
   p.tmem_cols = (uint32_t)fp.tmem_cols;
+  p.ucols = (uint32_t)fp.ucols;
   for (int l = 0; l <= levels; ++l) p.keep[l] = keep[l];
   p.scale_log2 = kLog2e / sqrtf((float)D);
 
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((unsigned)(fp.U * fp.cs), 1, 1);
+  cfg.gridDim = dim3((unsigned)(fp.clusters * fp.cs), 1, 1);
   cfg.blockDim = dim3(NT, 1, 1);
   cfg.dynamicSmemBytes = fp.smem;
   cfg.stream = s;

@@ -91,10 +91,11 @@ cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, c
                         const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
                         const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s);
 
-// Fused step (bf16, head_dim 128, <= 32 query rows): one cluster per unit.
+// Fused step (bf16, head_dim 128, <= 32 query rows): one cluster of cs CTAs
+// per P units.
 struct FusedPlan {
   bool ok;
-  int cs, stages, tmem_cols, cmax, kmax, U;
+  int cs, P, clusters, stages, tmem_cols, ucols, cmax, kmax, U;
   size_t smem;
   bool trim;
 };

@@ -51,6 +51,88 @@ __device__ __forceinline__ void st_cluster_v4f32(uint32_t addr, float a, float b
                : "memory");
 }
 
+// Split cluster barrier (every thread of every CTA of the cluster; not
+// warp-aligned, so it may follow divergent code).
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
+
+// Asynchronous stores into the shared memory of a CTA of this cluster (which
+// may be this CTA): the bytes are counted as completed transactions on that
+// CTA's mbarrier `mbar` (a shared::cluster address), which the receiver arms
+// with the total it expects.
+__device__ __forceinline__ void st_async_b32(uint32_t addr, uint32_t v, uint32_t mbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(addr), "r"(v),
+               "r"(mbar)
+               : "memory");
+}
+__device__ __forceinline__ void st_async_v2(uint32_t addr, uint32_t a, uint32_t b, uint32_t mbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.b32 [%0], {%1, %2}, [%3];" ::"r"(addr),
+               "r"(a), "r"(b), "r"(mbar)
+               : "memory");
+}
+__device__ __forceinline__ void st_async_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d,
+                                            uint32_t mbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   addr),
+               "r"(a), "r"(b), "r"(c), "r"(d), "r"(mbar)
+               : "memory");
+}
+// Arrive (release at cluster scope) on an mbarrier of a CTA of this cluster.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Barrier over a subset of the CTA's warps (`nthreads` a multiple of 32).
+__device__ __forceinline__ void named_sync(uint32_t id, uint32_t nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Explicit shared-space accesses (32-bit shared addresses).  Volatile, so
+// they stay ordered with the barriers around them; loads still overlap until
+// their results are used.
+__device__ __forceinline__ float lds_f32(uint32_t a) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t lds_u32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint2 lds_v2(uint32_t a) {
+  uint2 v;
+  asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint4 lds_v4(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void sts_u32(uint32_t a, uint32_t v) {
+  asm volatile("st.shared.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ void sts_v2(uint32_t a, uint32_t x, uint32_t y) {
+  asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(a), "r"(x), "r"(y) : "memory");
+}
+__device__ __forceinline__ void sts_v4(uint32_t a, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ uint32_t atoms_add(uint32_t a, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.shared.add.u32 %0, [%1], %2;" : "=r"(old) : "r"(a), "r"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ void reds_add(uint32_t a, uint32_t v) {
+  asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ void reds_or(uint32_t a, uint32_t v) {
+  asm volatile("red.shared.or.b32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // cp.async (16-byte global -> shared copies).
 // ---------------------------------------------------------------------------
@@ -86,26 +168,58 @@ __device__ __forceinline__ void mbar_init(uint32_t addr, uint32_t count) {
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
-__device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity) {
+// One test of the phase with the given parity; a thread whose phase is not
+// complete is suspended in hardware until it completes or about `hint_ns`
+// nanoseconds pass, so waiting threads do not compete for issue slots.
+__device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity, uint32_t hint_ns = 20000u) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(addr), "r"(parity)
+      : "r"(addr), "r"(parity), "r"(hint_ns)
       : "memory");
   return ok != 0;
 }
+// Acquire at cluster scope: for phases completed by other CTAs' arrivals or
+// asynchronous stores.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t addr, uint32_t parity, uint32_t hint_ns = 20000u) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+// Non-zero abort word at shared address `abort_a` (0: no abort word).
+__device__ __forceinline__ bool abort_set(uint32_t abort_a) {
+  if (!abort_a) return false;
+  uint32_t v;
+  asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(abort_a) : "memory");
+  return v != 0;
+}
 // Bounded wait for the phase with the given parity: gives up after about
-// `limit` clock cycles, or as soon as *abort becomes non-zero, and returns
-// false.
+// `limit` clock cycles, or as soon as the abort word becomes non-zero, and
+// returns false.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t addr, uint32_t parity, long long limit,
-                                                  const volatile int* abort = nullptr) {
+                                                  uint32_t abort_a = 0) {
+  if (mbar_try_wait(addr, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(addr, parity)) {
-    if (clock64() - t0 > limit) return false;
-    if (abort && *abort) return false;
+    if (clock64() - t0 > limit || abort_set(abort_a)) return false;
+  }
+  return true;
+}
+__device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t addr, uint32_t parity, long long limit,
+                                                          uint32_t abort_a = 0) {
+  if (mbar_try_wait_cluster(addr, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait_cluster(addr, parity)) {
+    if (clock64() - t0 > limit || abort_set(abort_a)) return false;
   }
   return true;
 }
