@@ -440,26 +440,26 @@ __device__ __forceinline__ float transpose_reduce32(float (&v)[32], int lane) {
   return v[0];
 }
 
-// Top-K scratch.  It lives in the P buffers, which nothing uses before the
-// attention.
+// Top-K scratch.  It lives in the unit's P buffers, which nothing uses before
+// the attention.
 constexpr int NB = 2048;  // histogram buckets
 constexpr int BPT = NB / NCT;
 struct SelScratch {
   uint32_t hist[NB];
-  float2 blist[NCT];             // boundary-bucket keys (key, position)
-  uint32_t bmap[kMaxCand / 32];  // chosen boundary positions
-  float2 sred[2][NCW];           // (min, max) per warp, alternating rounds
-  uint32_t ssel[2][4];           // boundary bucket, missing count, bucket count
-  int wsum[NCW];
+  float2 blist[NCT];    // boundary-bucket keys (key, position)
+  float2 sred[2][NCW];  // (min, max) per warp, alternating rounds
+  uint32_t ssel[2][4];  // boundary bucket, missing count, bucket count (alternating rounds)
+  int wsum[4][NCW];     // per-warp sums of the scans (slot per scan)
   uint32_t bcnt;
 };
-static_assert(sizeof(SelScratch) <= 2 * P_BYTES, "Top-K scratch must fit the P buffers");
-static_assert(kMaxCand / 32 == NCT, "one bitmap word per compute thread");
+static_assert(sizeof(SelScratch) <= UNIT_P_BYTES, "Top-K scratch must fit the P buffers");
 static_assert(BPT % 4 == 0, "buckets are read four at a time");
 
 #define SC_ADDR(sc_a, field) ((sc_a) + (uint32_t)offsetof(SelScratch, field))
 
-// Exclusive prefix sum over the compute threads (thread order).
+// Exclusive prefix sum over the compute threads (thread order), with its
+// per-warp sums in the NCW words at wsum_a.  One barrier: the caller does not
+// reuse those words before another barrier has passed.
 __device__ __forceinline__ int cta_excl_scan(int v, uint32_t wsum_a) {
   const int lane = threadIdx.x & 31, warp = ctid() >> 5;
   int incl = v;
@@ -471,7 +471,6 @@ __device__ __forceinline__ int cta_excl_scan(int v, uint32_t wsum_a) {
   if (lane == 31) sts_u32(wsum_a + 4u * warp, (uint32_t)incl);
   csync();
   const uint4 w = lds_v4(wsum_a);
-  csync();
   const int before = (warp > 0 ? (int)w.x : 0) + (warp > 1 ? (int)w.y : 0) + (warp > 2 ? (int)w.z : 0);
   return before + incl - v;
 }
@@ -485,23 +484,50 @@ __device__ __forceinline__ int bucket_of(float v, float lo, float scale) {
   return min(NB - 1, __float_as_int(__fadd_rd(x, 8388608.f)) - 0x4B000000);
 }
 
+// (min, max) of the undecided keys over the compute threads, via slot `par`.
+template <int R>
+__device__ __forceinline__ float2 cta_minmax(const float (&kv)[R], uint32_t act, uint32_t sc_a, int par) {
+  const int lane = threadIdx.x & 31, warp = ctid() >> 5;
+  float lo = INFINITY, hi = -INFINITY;
+#pragma unroll
+  for (int x = 0; x < R; ++x) {
+    const bool a = (act >> x) & 1u;
+    lo = fminf(lo, a ? kv[x] : INFINITY);
+    hi = fmaxf(hi, a ? kv[x] : -INFINITY);
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  if (lane == 0) sts_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + warp), __float_as_uint(lo), __float_as_uint(hi));
+  csync();
+#pragma unroll
+  for (int w = 0; w < NCW; ++w) {
+    const uint2 r = lds_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + w));
+    lo = fminf(lo, __uint_as_float(r.x));
+    hi = fmaxf(hi, __uint_as_float(r.y));
+  }
+  return make_float2(lo, hi);
+}
+
 // Top-K of the m keys at keys_a (largest first, lower position wins ties):
 // the kk chosen candidate indices, in ascending position order, overwrite the
 // key array.  A candidate's index is its position at the top scale, else
 // 2 J[j/2] + j%2 with J the previous selection at jprev_a (Eq. 10).
 // Each thread holds a run of R keys in registers (slot x holds position
 // j0 + (x + rot) % R; the rotation spreads a warp's reads over the banks) and
-// one bit per slot for "undecided" and "taken".  The undecided keys are
-// spread over NB buckets linear in [min, max] of those keys (fp32 arithmetic
-// is monotone, so a key in a higher bucket is strictly larger) and the bucket
-// holding the boundary is located from the bucket counts: keys above it are
-// taken, keys below it dropped.  A boundary bucket of at most NCT keys is
-// resolved exactly by ranking its keys on (key, -position); a larger one is
-// bucketed again over its own range.  If only equal keys remain, the lowest
-// positions are taken.
+// one bit per slot for "undecided" and "taken".  Each round spreads the
+// undecided keys over NB buckets linear in [min, max] of those keys (fp32
+// arithmetic is monotone, so a key in a higher bucket is strictly larger) and
+// locates the bucket holding the boundary from the bucket counts: keys above
+// it are taken, keys below it dropped.  A boundary bucket of at most NCT keys
+// is resolved exactly, each owner ranking its keys on (key, -position)
+// against the bucket's list; a larger one is bucketed again over its own
+// range.  If only equal keys remain, the lowest positions are taken.
 template <int R>
 __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
+  const int tid = ctid(), lane = tid & 31;
   const int j0 = tid * R;
   const int rot = (lane * R) >> 5;
   float kv[R];
@@ -512,45 +538,23 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
     kv[x] = lds_f32(keys_a + 4u * (uint32_t)min(j, m - 1));
     act |= (uint32_t)(j < m) << x;
   }
+  const uint32_t hist_a = SC_ADDR(sc_a, hist);
+  const uint32_t own_a = hist_a + 4u * (uint32_t)(NB - BPT * (tid + 1));  // buckets bhi - BPT + 1 .. bhi
+  const int bhi = NB - 1 - BPT * tid;  // thread order = buckets from high to low
+#pragma unroll
+  for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
+  float2 lh = cta_minmax<R>(kv, act, sc_a, 0);  // its barrier also publishes the cleared buckets
   uint32_t need = (uint32_t)kk;
   bool resolved = false;
-  const uint32_t hist_a = SC_ADDR(sc_a, hist);
 #pragma unroll 1
   for (int iter = 0; iter < 6; ++iter) {
-    const int par = iter & 1;  // reduction slots alternate, so no barrier is needed between rounds
-    float lo = INFINITY, hi = -INFINITY;
-#pragma unroll
-    for (int x = 0; x < R; ++x) {
-      const bool a = (act >> x) & 1u;
-      lo = fminf(lo, a ? kv[x] : INFINITY);
-      hi = fmaxf(hi, a ? kv[x] : -INFINITY);
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-    }
-    if (lane == 0)
-      sts_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + warp), __float_as_uint(lo), __float_as_uint(hi));
-#pragma unroll
-    for (int i = 0; i < BPT / 4; ++i) sts_v4(hist_a + 16u * (tid * (BPT / 4) + i), make_uint4(0, 0, 0, 0));
-    sts_u32(SC_ADDR(sc_a, bmap) + 4u * tid, 0u);
-    csync();
-#pragma unroll
-    for (int w = 0; w < NCW; ++w) {
-      const uint2 r = lds_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + w));
-      lo = fminf(lo, __uint_as_float(r.x));
-      hi = fmaxf(hi, __uint_as_float(r.y));
-    }
+    const int par = iter & 1;
+    const float lo = lh.x, hi = lh.y;
     if (!(hi > lo)) break;  // every undecided key is equal (or none is left)
     const float scale = (float)NB / (hi - lo);
 #pragma unroll
-    for (int x = 0; x < R; ++x)
-      if ((act >> x) & 1u) reds_add(hist_a + 4u * bucket_of(kv[x], lo, scale), 1u);
+    for (int x = 0; x < R; ++x) reds_add_if((act >> x) & 1u, hist_a + 4u * bucket_of(kv[x], lo, scale), 1u);
     csync();
-    // Thread tid owns buckets bhi, bhi - 1, ..., bhi - BPT + 1 (high to low).
-    const int bhi = NB - 1 - BPT * tid;
-    const uint32_t own_a = hist_a + 4u * (uint32_t)(bhi - BPT + 1);
     uint32_t cw[BPT];
 #pragma unroll
     for (int i = 0; i < BPT / 4; ++i) {
@@ -563,19 +567,22 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
     uint32_t tot = 0;
 #pragma unroll
     for (int i = 0; i < BPT; ++i) tot += cw[i];
-    const uint32_t above = (uint32_t)cta_excl_scan((int)tot, SC_ADDR(sc_a, wsum));
+    const uint32_t above = (uint32_t)cta_excl_scan((int)tot, SC_ADDR(sc_a, wsum) + 16u * par);
+    // Every thread has read its buckets: clear them for the next round.
+#pragma unroll
+    for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
     if (above < need && above + tot >= need) {
-      // This thread's buckets hold the boundary: walk them from high to low.
+      // This thread's buckets hold the boundary: walk them from high to low
+      // (branch-free; the first bucket that reaches `need` wins).
       uint32_t acc = above, sb = 0, sneed = 0, scnt = 0;
       bool found = false;
 #pragma unroll
       for (int k = BPT - 1; k >= 0; --k) {  // cw[k] is bucket bhi - (BPT - 1 - k)
-        if (!found && acc + cw[k] >= need) {
-          sb = (uint32_t)(bhi - (BPT - 1 - k));
-          sneed = need - acc;
-          scnt = cw[k];
-          found = true;
-        }
+        const bool hit = !found && acc + cw[k] >= need;
+        sb = hit ? (uint32_t)(bhi - (BPT - 1 - k)) : sb;
+        sneed = hit ? need - acc : sneed;
+        scnt = hit ? cw[k] : scnt;
+        found = found || hit;
         acc += cw[k];
       }
       sts_v4(SC_ADDR(sc_a, ssel) + 16u * par, make_uint4(sb, sneed, scnt, 0));
@@ -588,11 +595,10 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
     const uint32_t cnt = sel.z;
 #pragma unroll
     for (int x = 0; x < R; ++x) {
-      if ((act >> x) & 1u) {
-        const int bk = bucket_of(kv[x], lo, scale);
-        if (bk > sb) took |= 1u << x;
-        if (bk != sb) act &= ~(1u << x);
-      }
+      const uint32_t bit = ((act >> x) & 1u) << x;  // 0 for a decided slot
+      const int bk = bucket_of(kv[x], lo, scale);
+      took |= bk > sb ? bit : 0u;
+      act &= bk != sb ? ~bit : ~0u;
     }
     if (cnt == need) {
       took |= act;
@@ -601,8 +607,8 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
       break;
     }
     if (cnt <= (uint32_t)NCT) {
-      // Exact rank of each boundary key among the cnt of them.  The keys are
-      // appended with one atomic per warp.
+      // Append the boundary keys (one atomic per warp), then every owner
+      // ranks its own keys against the list.
       const int nb = __popc(act);
       int incl = nb;
 #pragma unroll
@@ -616,16 +622,19 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
       uint32_t slot = wbase + (uint32_t)(incl - nb);
 #pragma unroll
       for (int x = 0; x < R; ++x) {
-        if ((act >> x) & 1u) {
-          sts_v2(SC_ADDR(sc_a, blist) + 8u * slot, __float_as_uint(kv[x]), (uint32_t)(j0 + ((x + rot) & (R - 1))));
-          ++slot;
-        }
+        const bool a = (act >> x) & 1u;
+        sts_v2_if(a, SC_ADDR(sc_a, blist) + 8u * slot, __float_as_uint(kv[x]), (uint32_t)(j0 + ((x + rot) & (R - 1))));
+        slot += a ? 1u : 0u;
       }
       csync();
-      if (tid < (int)cnt) {
-        const uint2 me = lds_v2(SC_ADDR(sc_a, blist) + 8u * tid);
-        const float km = __uint_as_float(me.x);
-        const int jm = (int)me.y;
+#pragma unroll 1
+      for (uint32_t a = act; a; a &= a - 1) {
+        const int x = __ffs(a) - 1;
+        float kx = 0.f;
+#pragma unroll
+        for (int y = 0; y < R; ++y)
+          if (y == x) kx = kv[y];
+        const int jx = j0 + ((x + rot) & (R - 1));
         uint32_t rank = 0;
 #pragma unroll 1
         for (uint32_t v0 = 0; v0 < cnt; v0 += 4) {
@@ -635,23 +644,16 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const float ko = __uint_as_float(o[k].x);
-            rank += (v0 + k < cnt) && ((ko > km) || (ko == km && (int)o[k].y < jm));
+            rank += (v0 + k < cnt) && ((ko > kx) || (ko == kx && (int)o[k].y < jx));
           }
         }
-        if (rank < need) reds_or(SC_ADDR(sc_a, bmap) + 4u * (uint32_t)(jm >> 5), 1u << (jm & 31));
-      }
-      csync();
-#pragma unroll
-      for (int x = 0; x < R; ++x) {
-        if ((act >> x) & 1u) {
-          const int j = j0 + ((x + rot) & (R - 1));
-          if ((lds_u32(SC_ADDR(sc_a, bmap) + 4u * (uint32_t)(j >> 5)) >> (j & 31)) & 1u) took |= 1u << x;
-        }
+        if (rank < need) took |= 1u << x;
       }
       act = 0;
       resolved = true;
       break;
     }
+    lh = cta_minmax<R>(kv, act, sc_a, par ^ 1);  // the boundary bucket's range for the next round
   }
   // Position-order masks (bit i = position j0 + i).
   uint32_t take = 0, eq = 0;
@@ -663,7 +665,7 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
   }
   if (!resolved) {
     // Only equal keys are undecided: the first `need` by position are taken.
-    const int eq_base = cta_excl_scan(__popc(eq), SC_ADDR(sc_a, wsum));
+    const int eq_base = cta_excl_scan(__popc(eq), SC_ADDR(sc_a, wsum) + 48u);
     int remaining = (int)need - eq_base;
     for (uint32_t e = eq; e && remaining > 0; --remaining) {
       const uint32_t low = e & (~e + 1u);
@@ -671,24 +673,22 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
       e ^= low;
     }
   }
-  // Candidate indices of the winners (read before anything is written), then
-  // each at its output rank.  The scan's barriers order every thread's key
-  // reads before the key array is overwritten.
+  // Candidate indices of the slots (read before anything is written), then
+  // each winner at its output rank.  The scan's barrier orders every key read
+  // before the key array is overwritten.
   int cid[R];
 #pragma unroll
   for (int x = 0; x < R; ++x) {
     const int j = j0 + ((x + rot) & (R - 1));
     cid[x] = (top || j >= m) ? j : (int)lds_u32(jprev_a + 4u * (uint32_t)(j >> 1));
   }
-  const int base = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum));
+  const int base = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum) + 32u);
 #pragma unroll
   for (int x = 0; x < R; ++x) {
     const int i = (x + rot) & (R - 1);
-    if ((take >> i) & 1u) {
-      const int j = j0 + i;
-      const int c = top ? j : 2 * cid[x] + (j & 1);
-      sts_u32(keys_a + 4u * (uint32_t)(base + __popc(take & ((1u << i) - 1u))), (uint32_t)c);
-    }
+    const int j = j0 + i;
+    const int cv = top ? j : 2 * cid[x] + (j & 1);
+    sts_u32_if((take >> i) & 1u, keys_a + 4u * (uint32_t)(base + __popc(take & ((1u << i) - 1u))), (uint32_t)cv);
   }
   csync();
 }

@@ -129,6 +129,31 @@ __device__ __forceinline__ uint32_t atoms_add(uint32_t a, uint32_t v) {
 __device__ __forceinline__ void reds_add(uint32_t a, uint32_t v) {
   asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
+// Predicated forms: nothing happens where `pred` is false (no branch).
+__device__ __forceinline__ void reds_add_if(bool pred, uint32_t a, uint32_t v) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %0, 0;\n\t"
+      "@p red.shared.add.u32 [%1], %2;\n\t}" ::"r"((uint32_t)pred),
+      "r"(a), "r"(v)
+      : "memory");
+}
+__device__ __forceinline__ void sts_u32_if(bool pred, uint32_t a, uint32_t v) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %0, 0;\n\t"
+      "@p st.shared.u32 [%1], %2;\n\t}" ::"r"((uint32_t)pred),
+      "r"(a), "r"(v)
+      : "memory");
+}
+__device__ __forceinline__ void sts_v2_if(bool pred, uint32_t a, uint32_t x, uint32_t y) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %0, 0;\n\t"
+      "@p st.shared.v2.u32 [%1], {%2, %3};\n\t}" ::"r"((uint32_t)pred),
+      "r"(a), "r"(x), "r"(y)
+      : "memory");
+}
 __device__ __forceinline__ void reds_or(uint32_t a, uint32_t v) {
   asm volatile("red.shared.or.b32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
