@@ -61,8 +61,11 @@ constexpr int TILE_BYTES = 2 * HALF_BYTES;
 constexpr int QGRP = (D / 8) * 128;        // bytes per 8-row group of a query tile (core matrices)
 constexpr int Q_BYTES = NQ * D * 2;
 constexpr int P_BYTES = NQ * TM * 2;
-constexpr int COMB_BYTES = NQ * D * 4;     // received partial O rows of this CTA's head-dim slice
-constexpr int UNIT_P_BYTES = 2 * P_BYTES;  // a unit's P double buffer (also its Top-K scratch and combine buffer)
+constexpr int MAXCS_PAD_BYTES = 8 * NQ * 4;  // the ragged head-dim slices of a cluster of up to 8 CTAs
+// A unit's P double buffer; also its Top-K scratch and its combine buffer
+// (the partial O rows of this CTA's head-dim slice from every cluster CTA:
+// at most (D + cs) rows of 32 fp32 when cs does not divide D).
+constexpr int UNIT_P_BYTES = 2 * P_BYTES + MAXCS_PAD_BYTES;
 constexpr int kMaxCand = 32 * NCT;         // largest candidate list the Top-K holds in registers
 constexpr long long kWaitLimit = 1ll << 31;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -181,6 +184,9 @@ __device__ __forceinline__ void attn_slice(int total, uint32_t rank, uint32_t cs
 }
 
 __device__ __forceinline__ int tiles_of(int mc) { return (mc + TM - 1) / TM; }
+
+// Head-dim slice [dlo(r), dlo(r + 1)) whose output rows CTA r combines.
+__device__ __forceinline__ int dlo(int r, int cs) { return r * D / cs; }
 
 // Where the rows of a candidate or key list come from.
 //  kind 0: position j -> row j (top scale);
@@ -876,14 +882,16 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
     for (uint32_t r = 0; r < cs; ++r) mbar_arrive_cluster(map_rank(ready, r));
   }
   wait_cluster_or_abort(ready, 0u, ms, p.status);
-  const int rows = D / (int)cs;
   const uint32_t comb_a = smem_u32(comb);
   const uint32_t cbar = bar_addr(ms.cbar[pp]);
   {
-    const uint32_t owner = (uint32_t)(tid / rows);
-    const int dl = tid % rows;
-    const uint32_t dst = map_rank(comb_a + 4u * (uint32_t)((rank * rows + dl) * NQ), owner);
-    const uint32_t rb = map_rank(cbar, owner);
+    // Owner of head-dim row d = tid, and the row's place in its buffer.
+    int owner = tid * (int)cs / D;
+    while (owner + 1 < (int)cs && dlo(owner + 1, cs) <= tid) ++owner;
+    const int orows = dlo(owner + 1, cs) - dlo(owner, cs);
+    const int dl = tid - dlo(owner, cs);
+    const uint32_t dst = map_rank(comb_a + 4u * (uint32_t)(((int)rank * orows + dl) * NQ), (uint32_t)owner);
+    const uint32_t rb = map_rank(cbar, (uint32_t)owner);
 #pragma unroll
     for (int i = 0; i < 32; i += 4) st_async_v4(dst + 4u * i, orow[i], orow[i + 1], orow[i + 2], orow[i + 3], rb);
   }
@@ -917,20 +925,15 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
   }
   const float inv = 1.f / den;
   bf16* ob = p.O + (int64_t)(u / p.H) * p.osb + (int64_t)(u % p.H) * p.osh;
+  const int d0 = dlo((int)rank, cs), rows = dlo((int)rank + 1, cs) - d0;
   if (qi < p.q) {
 #pragma unroll 1
-    for (int dp = tid >> 5; dp < rows / 2; dp += NCT / NQ) {
-      float n0 = 0.f, n1 = 0.f;
+    for (int dl = tid >> 5; dl < rows; dl += NCT / NQ) {
+      float n = 0.f;
 #pragma unroll
-      for (int r = 0; r < MAXCS; ++r) {
-        if (r < (int)cs) {
-          const uint32_t a = comb_a + 4u * (uint32_t)((r * rows + 2 * dp) * NQ + qi);
-          n0 = fmaf(lds_f32(a), f[r], n0);
-          n1 = fmaf(lds_f32(a + 4u * NQ), f[r], n1);
-        }
-      }
-      const int d = (int)rank * rows + 2 * dp;
-      *reinterpret_cast<__nv_bfloat162*>(ob + (int64_t)qi * p.oss + d) = __floats2bfloat162_rn(n0 * inv, n1 * inv);
+      for (int r = 0; r < MAXCS; ++r)
+        if (r < (int)cs) n = fmaf(lds_f32(comb_a + 4u * (uint32_t)((r * rows + dl) * NQ + qi)), f[r], n);
+      ob[(int64_t)qi * p.oss + d0 + dl] = __float2bfloat16_rn(n * inv);
     }
   }
 }
@@ -1075,7 +1078,8 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     for (int pp = 0; pp < c.np; ++pp) {
       mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
       mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)(p.n >> p.L));
-      mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), COMB_BYTES + c.cs * NQ * 8u);
+      const uint32_t rows = (uint32_t)(dlo((int)c.rank + 1, c.cs) - dlo((int)c.rank, c.cs));
+      mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), c.cs * rows * NQ * 4u + c.cs * NQ * 8u);
     }
   }
   if (warp == MMA_WARP) {
@@ -1207,13 +1211,15 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
   if (smem_layout(4, P, cmax, kmax).total > kMaxSmem) stages = 3;
   const size_t smem = smem_layout(stages, P, cmax, kmax).total;
   if (smem > kMaxSmem) return fp;
-  int cs = 1;
-  while (cs < MAXCS && clusters * cs * 2 <= num_sms) cs *= 2;
-  while (cs < MAXCS && P * unit_cols(cs) > 512) cs *= 2;
-  if (P * unit_cols(cs) > 512) return fp;
-  // Prefer a smaller cluster over a second wave when the chosen one does not
-  // fit the SMs of its GPCs all at once.
-  while (cs > 1 && P * unit_cols(cs / 2) <= 512 && clusters > max_active_clusters(stages, cs, smem)) cs /= 2;
+  // The largest cluster (any size up to 8) whose grid fits the SMs in one
+  // wave, all clusters resident at once, and whose slices fit TMEM; else the
+  // smallest one that fits TMEM.
+  int cs = 0;
+  for (int c = MAXCS; c >= 1 && cs == 0; --c)
+    if (clusters * c <= num_sms && P * unit_cols(c) <= 512 && clusters <= max_active_clusters(stages, c, smem)) cs = c;
+  for (int c = 1; c <= MAXCS && cs == 0; ++c)
+    if (P * unit_cols(c) <= 512) cs = c;
+  if (cs == 0) return fp;
   const int ucols = unit_cols(cs);
   int cols = 32;
   while (cols < P * ucols) cols *= 2;
