@@ -201,7 +201,7 @@ def run_gpu(args, cfg, rank, world, device):
     for lay in layers:
         coeffs = torch.empty(wf.wf_coeffs_bytes(lay.K, w.levels), dtype=torch.uint8, device=device)
         wf.wf_dwt_build(lay.K, w.levels, coeffs)
-        ws = torch.empty(wf.wf_step_workspace_bytes(lay.Q, lay.K, w.levels, keep, w.ng), dtype=torch.uint8,
+        ws = torch.zeros(wf.wf_step_workspace_bytes(lay.Q, lay.K, w.levels, keep, w.ng), dtype=torch.uint8,
                          device=device)
         bufs.append(dict(coeffs=coeffs, ws=ws, idx=torch.empty(w.units, w.k, dtype=torch.int32, device=device),
                          O=torch.empty_like(lay.Q)))

@@ -196,9 +196,12 @@ wf_status wf_sparse_attn_noalloc(const void* Q, const wf_tensor* q, const void* 
  * For bf16 with head_dim 128 and at most 32 query rows the filter and the
  * attention run as one fused kernel (one thread-block cluster per (batch,
  * head)); other shapes run the per-stage kernels.  The fused kernel's waits
- * on tensor-core completion are bounded: if one gives up (it never should),
- * the kernel returns early, outputs are undefined, and a status word at the
- * start of ws is set; wf_workspace_status() reports it.
+ * (on copies, tensor-core completion and the cluster's exchanges) are
+ * bounded: if one gives up (it never should), the kernel returns early,
+ * outputs are undefined, and a status word in the first 4 bytes of ws is set;
+ * wf_workspace_status() reports and clears it.  wf_step never clears the word
+ * itself (so a failure stays visible across calls): zero those 4 bytes once
+ * before the first call (or call wf_workspace_status once).
  * ------------------------------------------------------------------------- */
 size_t wf_step_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
                                int n_g);

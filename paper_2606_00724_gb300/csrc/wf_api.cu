@@ -233,10 +233,9 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return WF_ERR_CUDA;
-  int* status = static_cast<int*>(ws);
+  int* status = static_cast<int*>(ws);  // set by the fused kernel on a timeout; read and cleared by wf_workspace_status
   void* scratch = static_cast<char*>(ws) + kStatusBytes;
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), s);
-  if (e != cudaSuccess) return WF_ERR_CUDA;
+  cudaError_t e = cudaSuccess;
   if (refresh_coeffs && (e = wf::launch_dwt(K, *kv, levels, coeffs, s)) != cudaSuccess) return WF_ERR_CUDA;
   const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, n_g, n_g > 0 ? g : nullptr, sms);
   if (fp.ok) {

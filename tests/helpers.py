@@ -50,7 +50,7 @@ class GpuRun:
         """One wf_step (fused kernel where it applies), with level sets."""
         if not hasattr(self, "ws_step"):
             ng = self.Kg.shape[2] if self.Kg is not None else 0
-            self.ws_step = torch.empty(wf.wf_step_workspace_bytes(self.Q, self.K, self.L, self.keep, ng),
+            self.ws_step = torch.zeros(wf.wf_step_workspace_bytes(self.Q, self.K, self.L, self.keep, ng),
                                        dtype=torch.uint8, device=self.K.device)
         wf.wf_step(self.Q, self.K, self.V, self.Kg, self.Vg, self.coeffs, refresh, self.L, self.keep, self.idx,
                    self.O, self.ws_step, level_sets=self.sets)

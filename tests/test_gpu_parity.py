@@ -136,7 +136,7 @@ def test_step_matches_separate_calls():
     idx = torch.empty_like(a.idx)
     O = torch.empty_like(a.O)
     coeffs = torch.empty_like(a.coeffs)
-    ws = torch.empty(wf.wf_step_workspace_bytes(batch.Q, batch.K, w.levels, w.keep, w.ng), dtype=torch.uint8,
+    ws = torch.zeros(wf.wf_step_workspace_bytes(batch.Q, batch.K, w.levels, w.keep, w.ng), dtype=torch.uint8,
                      device="cuda")
     wf.wf_step(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, coeffs, True, w.levels, w.keep, idx, O, ws)
     torch.cuda.synchronize()
