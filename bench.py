@@ -311,7 +311,8 @@ def main():
     config = {"workload": w.name, "batch": w.batch, "heads": w.heads, "head_dim": w.head_dim,
               "context": w.n, "query_block": w.q, "generation_rows": w.ng, "levels": w.levels, "k": w.k,
               "keep": list(w.keep), "layers": w.layers, "storage": w.dtype,
-              "step": "wf_filter + wf_sparse_attn per layer" + (
+              "step": ("wf_step (one fused filter + sparse-attention kernel) per layer" if fused_eligible(w) else
+                       "wf_step (per-stage filter and sparse-attention kernels) per layer") + (
                   f"; wf_dwt_build refresh every {w.refresh_every} steps" if w.refresh_every else
                   "; pyramid built once before timing"),
               "l2": "flushed before every timed step (256 MiB write)", "parallelism": f"replicas{args.gpus}"}
