@@ -291,6 +291,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=None, help="override the workload's batch (small profiling cases)")
     ap.add_argument("--heads", type=int, default=None, help="override the workload's head count")
+    ap.add_argument("--schedule", default="default", choices=["default", "level0"],
+                    help="kept counts: the default schedule, or the token level as its own selection step")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -304,6 +306,13 @@ def main():
         import dataclasses
         w = dataclasses.replace(w, batch=args.batch or w.batch, heads=args.heads or w.heads,
                                 name=f"{w.name}_B{args.batch or w.batch}_H{args.heads or w.heads}")
+        synth.WORKLOADS[cfg] = w
+    if args.schedule == "level0":
+        # The token level as its own selection step (one proportion over L+1 scans).
+        import dataclasses
+        from paper_2606_00724_gb300 import wf
+        keep = tuple(wf.wf_level0_schedule(w.n, w.levels, w.k))
+        w = dataclasses.replace(w, keep=keep, name=f"{w.name}_level0")
         synth.WORKLOADS[cfg] = w
     ub = unit_bytes(w)
     hbm_peak, peak_kind = peaks()

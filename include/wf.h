@@ -108,11 +108,18 @@ wf_status wf_dwt_build(const void* K, const void* V, const wf_tensor* kv, int le
  * wf_schedule_from_proportions: per-scale proportions m[l] in (0, 1]
  *   (m[0] unused): keep[l] = min(|C_l|, max(1, ceil(m[l] |C_l|))),
  *   keep[0] = 2 keep[1].
+ * wf_level0_schedule: the reading in which the token level is a selection
+ *   step of its own (Algorithm 1's last scan over raw keys): one proportion
+ *   m = (k/n)^(1/(L+1)) for the L pyramid scales and for the tokens,
+ *   keep[l] = min(|C_l|, max(1, ceil(m |C_l|))) for l = L..1, keep[0] = k
+ *   kept out of the 2 keep[1] token candidates (a level-0 selection
+ *   whenever k < 2 keep[1]).
  * "ceil" ignores a product that exceeds an integer by less than 1e-9.
  * Host-only; return WF_ERR_SCHEDULE if no feasible schedule exists.
  * ------------------------------------------------------------------------- */
 wf_status wf_default_schedule(int64_t n, int levels, int64_t k, int32_t* keep);
 wf_status wf_schedule_from_proportions(int64_t n, int levels, const double* m, int32_t* keep);
+wf_status wf_level0_schedule(int64_t n, int levels, int64_t k, int32_t* keep);
 
 /* ---------------------------------------------------------------------------
  * 2-3. Skim and scan (Eq. 7-11, Algorithm 1 inner loop).

@@ -59,6 +59,7 @@ def _load():
         "orc_round_bf16": (ctypes.c_float, [ctypes.c_float]),
         "orc_skim_weights_f64": (I, [P, I, I, P, I64, P]),
         "orc_default_schedule": (I, [I64, I, I64, P]),
+        "orc_level0_schedule": (I, [I64, I, I64, P]),
         "orc_schedule_from_proportions": (I, [I64, I, P, P]),
         "orc_filter_f64": (I, [P, I, I, P, P, I64, I, P, P, P, P]),
         "orc_filter_literal_f64": (I, [P, I, I, P, I64, I, P, P, P]),
@@ -155,6 +156,13 @@ def skim_weights(Q, rows):
 def default_schedule(n: int, L: int, k: int) -> np.ndarray:
     keep = np.zeros(L + 1, dtype=np.int32)
     _check(_load().orc_default_schedule(n, L, k, _p(keep)), "default_schedule")
+    return keep
+
+
+def level0_schedule(n: int, L: int, k: int) -> np.ndarray:
+    """The token level as its own selection step (m = (k/n)^(1/(L+1)))."""
+    keep = np.zeros(L + 1, dtype=np.int32)
+    _check(_load().orc_level0_schedule(n, L, k, _p(keep)), "level0_schedule")
     return keep
 
 

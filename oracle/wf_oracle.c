@@ -226,6 +226,25 @@ int orc_default_schedule(int64_t n, int L, int64_t k, int32_t* keep) {
   return 0;
 }
 
+/* Token level as a selection step of its own: the same proportion m for the
+ * L pyramid scans and for the scan over the 2 k_1 raw-key candidates
+ * (Algorithm 1 read with its last scan at level 0), m = (k/n)^(1/(L+1)). */
+int orc_level0_schedule(int64_t n, int L, int64_t k, int32_t* keep) {
+  if (!shape_ok(n, 1, L) || !keep || k < 1 || k > n) return -1;
+  double m = pow((double)k / (double)n, 1.0 / (double)(L + 1));
+  int64_t cnt = n >> L;
+  for (int b = L; b >= 1; --b) {
+    int64_t kb = ceil_guarded(m * (double)cnt);
+    if (kb < 1) kb = 1;
+    if (kb > cnt) kb = cnt;
+    keep[b] = (int32_t)kb;
+    cnt = 2 * kb;
+  }
+  if (k > cnt) return -1;
+  keep[0] = (int32_t)k;
+  return 0;
+}
+
 int orc_schedule_from_proportions(int64_t n, int L, const double* m, int32_t* keep) {
   if (!shape_ok(n, 1, L) || !m || !keep) return -1;
   int64_t cnt = n >> L;

@@ -68,6 +68,9 @@ int orc_default_schedule(int64_t n, int L, int64_t k, int32_t* keep);
 /* Kept counts from the per-scale proportions m_b of Eq. 9 (m[b], b = 1..L;
  * m[0] unused): keep[b] = ceil(m_b |C_b|) clamped to [1, |C_b|];
  * keep[0] = 2 keep[1] (no trim).  Returns 0, or -1 on a bad proportion. */
+/* Token level as its own selection step: m = (k/n)^(1/(L+1)) for the L
+ * pyramid scans and the token scan; keep[0] = k of the 2 keep[1] tokens. */
+int orc_level0_schedule(int64_t n, int L, int64_t k, int32_t* keep);
 int orc_schedule_from_proportions(int64_t n, int L, const double* m, int32_t* keep);
 
 /* Multi-scale recursive filtering (Sections 3.1-3.2, Algorithm 1 inner loop)

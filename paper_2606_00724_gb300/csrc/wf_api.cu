@@ -136,6 +136,22 @@ WF_API wf_status wf_default_schedule(int64_t n, int levels, int64_t k, int32_t* 
   return WF_OK;
 }
 
+WF_API wf_status wf_level0_schedule(int64_t n, int levels, int64_t k, int32_t* keep) {
+  if (!keep || levels < 1 || levels > 30 || n < 1 || k < 1 || k > n) return WF_ERR_INVALID_ARG;
+  if ((n >> levels) < 1 || ((n >> levels) << levels) != n) return WF_ERR_SHAPE;
+  const double m = pow((double)k / (double)n, 1.0 / (levels + 1));  // L pyramid scans + the token scan
+  int64_t cnt = n >> levels;
+  for (int l = levels; l >= 1; --l) {
+    int64_t kb = ceil_guarded(m * (double)cnt);
+    kb = kb < 1 ? 1 : (kb > cnt ? cnt : kb);
+    keep[l] = (int32_t)kb;
+    cnt = 2 * kb;
+  }
+  if (k > cnt) return WF_ERR_SCHEDULE;
+  keep[0] = (int32_t)k;
+  return WF_OK;
+}
+
 WF_API wf_status wf_schedule_from_proportions(int64_t n, int levels, const double* m, int32_t* keep) {
   if (!keep || !m || levels < 1 || levels > 30 || n < 1) return WF_ERR_INVALID_ARG;
   if ((n >> levels) < 1 || ((n >> levels) << levels) != n) return WF_ERR_SHAPE;

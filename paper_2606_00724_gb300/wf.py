@@ -45,6 +45,7 @@ SIGNATURES = {
     "wf_coeffs_bytes": (_SZ, [_T, _I]),
     "wf_dwt_build": (_I, [_P, _P, _T, _I, _P, _SZ, _P]),
     "wf_default_schedule": (_I, [_I64, _I, _I64, _P]),
+    "wf_level0_schedule": (_I, [_I64, _I, _I64, _P]),
     "wf_schedule_from_proportions": (_I, [_I64, _I, _P, _P]),
     "wf_filter_workspace_bytes": (_SZ, [_T, _T, _I, _P]),
     "wf_filter": (_I, [_P, _T, _P, _P, _T, _I, _P, _P, _P, _P, _SZ, _P]),
@@ -122,6 +123,12 @@ def wf_dwt_build(K: torch.Tensor, levels: int, coeffs: torch.Tensor, stream=None
 def wf_default_schedule(n: int, levels: int, k: int) -> list[int]:
     keep = (ctypes.c_int32 * (levels + 1))()
     _check(lib().wf_default_schedule(n, levels, k, keep), "wf_default_schedule")
+    return list(keep)
+
+
+def wf_level0_schedule(n: int, levels: int, k: int) -> list[int]:
+    keep = (ctypes.c_int32 * (levels + 1))()
+    _check(lib().wf_level0_schedule(n, levels, k, keep), "wf_level0_schedule")
     return list(keep)
 
 

@@ -64,6 +64,23 @@ def test_schedule_from_proportions_matches_oracle(lib):
         wf.wf_schedule_from_proportions(64, 2, [0, 0.5, 1.5])
 
 
+def test_level0_schedule_matches_oracle(lib):
+    r = np.random.default_rng(1)
+    for _ in range(60):
+        L = int(r.integers(1, 7))
+        n = int(r.integers(1, 256)) << L
+        k = int(r.integers(1, n + 1))
+        try:
+            want = oracle.level0_schedule(n, L, k).tolist()
+        except ValueError:
+            with pytest.raises(wf.WfError):
+                wf.wf_level0_schedule(n, L, k)
+            continue
+        assert wf.wf_level0_schedule(n, L, k) == want
+    for w in synth.WORKLOADS.values():
+        assert wf.wf_level0_schedule(w.n, w.levels, w.k) == oracle.level0_schedule(w.n, w.levels, w.k).tolist()
+
+
 def test_workload_schedules(lib):
     for w in synth.WORKLOADS.values():
         assert wf.wf_default_schedule(w.n, w.levels, w.k) == list(w.keep)

@@ -97,3 +97,23 @@ def test_step_random_shapes(B, H, n, q, ng, L, keep, bshd):
         assert np.all(np.diff(idx) > 0) and idx.min() >= 0 and idx.max() < n
         O = oracle.sparse_attn(Qn, Kn, Vn, idx, Kgn, Vgn)
         assert_close_out(f64(run.O[b, h]), O, torch.bfloat16)
+
+
+@pytest.mark.parametrize("cfg", ["c2", "c3", "c5"])
+def test_step_level0_schedule(cfg):
+    # The token level as its own selection step (wf_level0_schedule): the
+    # level-0 scan over raw keys keeps k of 2 keep[1] candidates.  Planted
+    # ladder built for that schedule; full-size layer in the fused kernel.
+    import dataclasses
+    w0 = synth.WORKLOADS[cfg]
+    keep = tuple(wf.wf_level0_schedule(w0.n, w0.levels, w0.k))
+    assert keep[0] < 2 * keep[1]
+    w = dataclasses.replace(w0, keep=keep, name=w0.name + "_level0")
+    batch = synth.make_batch(w, planted=True, device="cuda", cfg=cfg)
+    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, list(w.keep)).step()
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    _check(w, batch, run, [0, w.units // 2 + 1, w.units - 1])
+    idx = run.idx.cpu().numpy()
+    for u in range(w.units):
+        assert np.array_equal(idx[u], batch.targets[u][0].cpu().numpy()), f"unit {u} planted"

@@ -226,3 +226,49 @@ def test_table3_default_scale_schedule(orc):
                              math.ceil(0.6 * 1024)]
     with pytest.raises(ValueError):
         orc.schedule_from_proportions(4096, B, [0.0, 0.0, 0.5])
+
+
+@pytest.mark.parametrize("cfg", list(synth.WORKLOADS))
+def test_level0_schedule(orc, cfg):
+    # The token level as its own selection step: one proportion m over the
+    # L pyramid scans and the token scan.  Each scale keeps between m and
+    # m + 1/|C_b| of its candidates, the product of the kept fractions lands
+    # on k/n, and m lies in the range the hot-path survey gives for these
+    # shapes (about 0.50-0.57).
+    w = synth.WORKLOADS[cfg]
+    keep = orc.level0_schedule(w.n, w.levels, w.k)
+    m = (w.k / w.n) ** (1.0 / (w.levels + 1))
+    assert 0.49 <= m <= 0.58
+    assert keep[0] == w.k
+    cnt = w.n >> w.levels
+    frac = 1.0
+    for b in range(w.levels, 0, -1):
+        assert 1 <= keep[b] <= cnt
+        assert m - 1e-12 <= keep[b] / cnt <= m + 1.0 / cnt
+        frac *= keep[b] / cnt
+        cnt = 2 * int(keep[b])
+    assert w.k <= cnt                       # the token scan keeps k of 2 keep[1]
+    frac *= w.k / cnt
+    assert abs(frac - w.k / w.n) / (w.k / w.n) < 0.05 * (w.levels + 1)
+    with pytest.raises(ValueError):
+        orc.level0_schedule(w.n, w.levels, w.n + 1)
+
+
+@pytest.mark.parametrize("cfg", ["c1", "c2", "c3"])
+def test_planted_ladder_level0_schedule(orc, cfg):
+    # With the token level as its own selection step, the planted ladder
+    # (built for that schedule, including the level-0 scan over raw keys)
+    # is still what the oracle finds at every scale.
+    import dataclasses
+    w0 = synth.WORKLOADS[cfg]
+    keep = tuple(int(x) for x in orc.level0_schedule(w0.n, w0.levels, w0.k))
+    w = dataclasses.replace(w0, keep=keep, name=w0.name + "_level0")
+    dt = synth.storage_dtype(w)
+    u = synth.make_unit(w, 0, w.heads - 1, planted=True, cfg=cfg)
+    Q = u.Q.to(dt).float().numpy()
+    K = u.K.to(dt).float().numpy()
+    pyr = orc.haar_pyramid_spec32(K, w.levels, w.dtype == "bf16")
+    mu0, sets = orc.filter(Q, pyr, K, w.n, w.levels, np.array(w.keep), want_sets=True)
+    for b, tgt in u.targets.items():
+        assert np.array_equal(sets[b], tgt.numpy()), (cfg, b)
+    assert np.array_equal(mu0, u.targets[0].numpy())
