@@ -97,6 +97,28 @@ wf_status wf_dwt_build(const void* K, const void* V, const wf_tensor* kv, int le
                        size_t coeffs_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Cache update with an incremental pyramid refresh (the step before the build
+ * in Algorithm 1 when only part of the cached prompt changed, Eq. 4's cache
+ * refresh applied to a window): writes the count = nt->seq new key rows Knew
+ * (and value rows Vnew) into K (and V) at token positions [pos, pos + count),
+ * and in the same kernel recomputes every pyramid coefficient whose block
+ * contains one of those positions (Eq. 5-6): coeffs then equals wf_dwt_build
+ * of the updated K, bit for bit.  The kernel reads the aligned 2^L-token
+ * blocks that hold the new rows, writes the new rows and those blocks'
+ * coefficients, and touches nothing else.
+ *   Knew, Vnew: device, [B, H, count, d] (nt: same batch, heads, head_dim and
+ *               dtype as kv); Vnew and V are both NULL to update keys only.
+ *               They must not overlap K, V or coeffs.
+ *   K, V: the caches (kv), updated in place; coeffs: the pyramid of K.
+ * Errors: WF_ERR_INVALID_ARG for a missing pointer, Vnew/V given alone, or a
+ * window outside [0, n); shape, dtype, alignment and size errors as in
+ * wf_dwt_build.  Nothing is enqueued on an error.
+ * ------------------------------------------------------------------------- */
+wf_status wf_cache_update(const void* Knew, const void* Vnew, const wf_tensor* nt, void* K, void* V,
+                          const wf_tensor* kv, int64_t pos, int levels, void* coeffs, size_t coeffs_bytes,
+                          void* stream);
+
+/* ---------------------------------------------------------------------------
  * Kept counts (Eq. 9 "proportion m_B").  keep has levels+1 entries: keep[l]
  * = number of level-l coefficients kept (l = 1..levels), keep[0] = final
  * number of prompt tokens k.  Feasible iff 1 <= keep[L] <= n/2^L,

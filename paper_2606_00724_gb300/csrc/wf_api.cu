@@ -118,6 +118,24 @@ WF_API wf_status wf_dwt_build(const void* K, const void* V, const wf_tensor* kv,
   return cuda_status(wf::launch_dwt(K, *kv, levels, coeffs, static_cast<cudaStream_t>(stream)));
 }
 
+WF_API wf_status wf_cache_update(const void* Knew, const void* Vnew, const wf_tensor* nt, void* K, void* V,
+                                 const wf_tensor* kv, int64_t pos, int levels, void* coeffs, size_t coeffs_bytes,
+                                 void* stream) {
+  wf_status st;
+  if ((st = check_desc(kv, false)) != WF_OK) return st;
+  if ((st = check_desc(nt, false)) != WF_OK) return st;
+  if ((st = check_levels(kv, levels)) != WF_OK) return st;
+  if (!same_units(kv, nt)) return WF_ERR_SHAPE;
+  if (kv->dtype != nt->dtype) return WF_ERR_DTYPE;
+  if (!Knew || !K || !coeffs || (!Vnew) != (!V)) return WF_ERR_INVALID_ARG;
+  if (pos < 0 || pos + (int64_t)nt->seq > (int64_t)kv->seq) return WF_ERR_INVALID_ARG;
+  if (!aligned16(Knew) || !aligned16(K) || !aligned16(coeffs) || (V && (!aligned16(V) || !aligned16(Vnew))))
+    return WF_ERR_ALIGN;
+  if (coeffs_bytes < wf_coeffs_bytes(kv, levels)) return WF_ERR_WORKSPACE;
+  return cuda_status(
+      wf::launch_cache_update(Knew, Vnew, *nt, K, V, *kv, pos, levels, coeffs, static_cast<cudaStream_t>(stream)));
+}
+
 WF_API wf_status wf_default_schedule(int64_t n, int levels, int64_t k, int32_t* keep) {
   if (!keep || levels < 1 || levels > 30 || n < 1 || k < 1 || k > n) return WF_ERR_INVALID_ARG;
   if ((n >> levels) < 1 || ((n >> levels) << levels) != n) return WF_ERR_SHAPE;

@@ -8,29 +8,47 @@
 // share a row are adjacent, so each warp reads and writes whole 256-byte row
 // segments.  The arithmetic is the fp32 add-then-multiply of wf_dwt_build
 // (no fused multiply-add: __fadd_rn / __fmul_rn).
+//
+// The update mode (wf_cache_update) runs the same cascade over only the blocks
+// that contain token positions [pos, pos + count): a thread takes its slice of
+// a new row from the update buffer, writes it into the cache (and the value
+// slice too), and takes every other row of the block from the cache, so the
+// coefficients it writes equal those of a full build of the updated keys.
 #include "wf_internal.cuh"
 
 namespace wf {
 namespace {
 
-template <typename T, int L>
-__global__ void __launch_bounds__(256) dwt_kernel(const T* __restrict__ K, int64_t sb, int64_t sh, int64_t ss,
-                                                  int H, int n, int D, T* __restrict__ coeffs,
-                                                  int64_t rows_total, int64_t total_items) {
+// Rows [pos, pos + count) of the cache, replaced by an update buffer.
+template <typename T>
+struct Update {
+  const T* Kn;  // [B, H, count, D] new key rows
+  const T* Vn;  // new value rows, or null
+  T* V;         // value cache (null with Vn)
+  int64_t nsb, nsh, nss;  // strides of the update buffers
+  int64_t pos, count;
+  int64_t blk0;           // first block of the unit that holds a new row
+};
+
+template <typename T, int L, bool UPDATE>
+__global__ void __launch_bounds__(256) dwt_kernel(const T* K_in, T* K_out, int64_t sb, int64_t sh,
+                                                  int64_t ss, int H, int n, int D, T* __restrict__ coeffs,
+                                                  int64_t rows_total, int64_t nblk, int64_t total_items,
+                                                  Update<T> up) {
   constexpr int VEC = Vec<T>::N;
   constexpr int LC = L < 3 ? L : 3;
   constexpr int CH = 1 << LC;
   constexpr int NP = L > LC ? L - LC : 1;
   const int lanes = D / VEC;
-  const int64_t nblk = (int64_t)n >> L;
   const int64_t item = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (item >= total_items) return;
   const int lane = (int)(item % lanes);
   const int64_t rest = item / lanes;
-  const int64_t blk = rest % nblk;
+  const int64_t blk = rest % nblk + (UPDATE ? up.blk0 : 0);
   const int64_t u = rest / nblk;
   const int64_t bb = u / H, hh = u % H;
-  const T* src = K + bb * sb + hh * sh + (blk << L) * ss + (int64_t)lane * VEC;
+  const int64_t tok0 = blk << L;
+  const T* src = K_in + bb * sb + hh * sh + tok0 * ss + (int64_t)lane * VEC;
   T* dst = coeffs + u * rows_total * D + (int64_t)lane * VEC;
   const float c = 0.70710678118654752440f;  // fl32(1/sqrt 2)
 
@@ -39,7 +57,24 @@ __global__ void __launch_bounds__(256) dwt_kernel(const T* __restrict__ K, int64
   for (int ch = 0; ch < (1 << (L - LC)); ++ch) {
     float v[CH][VEC];
 #pragma unroll
-    for (int t = 0; t < CH; ++t) ld_vec(src + (int64_t)(ch * CH + t) * ss, v[t]);
+    for (int t = 0; t < CH; ++t) {
+      const int64_t tok = tok0 + ch * CH + t;
+      if (UPDATE && tok >= up.pos && tok < up.pos + up.count) {
+        // A new row: read it from the update buffer, store it into the cache.
+        const int64_t r = tok - up.pos;
+        const int64_t no = bb * up.nsb + hh * up.nsh + r * up.nss + (int64_t)lane * VEC;
+        const int64_t co = bb * sb + hh * sh + tok * ss + (int64_t)lane * VEC;
+        ld_vec(up.Kn + no, v[t]);
+        st_vec(K_out + co, v[t]);
+        if (up.Vn) {
+          float vv[VEC];
+          ld_vec(up.Vn + no, vv);
+          st_vec(up.V + co, vv);
+        }
+      } else {
+        ld_vec(src + (int64_t)(ch * CH + t) * ss, v[t]);
+      }
+    }
     const int64_t gc = (blk << (L - LC)) + ch;  // chunk index within the unit
 #pragma unroll
     for (int lev = 1; lev <= LC; ++lev) {
@@ -73,42 +108,76 @@ __global__ void __launch_bounds__(256) dwt_kernel(const T* __restrict__ K, int64
   }
 }
 
+// Full build (up.count == 0) or the update of the blocks holding the new rows.
 template <typename T, int L>
-cudaError_t run(const void* K, const wf_tensor& kv, void* coeffs, cudaStream_t s) {
+cudaError_t run(const void* K, void* K_out, const wf_tensor& kv, void* coeffs, const Update<T>& up, cudaStream_t s) {
   const int U = kv.batch * kv.heads;
   const int lanes = kv.head_dim / Vec<T>::N;
   const int64_t rows_total = (int64_t)kv.seq - ((int64_t)kv.seq >> L);
-  const int64_t items = (int64_t)U * ((int64_t)kv.seq >> L) * lanes;
+  const int64_t nblk = up.count > 0 ? ((up.pos + up.count - 1) >> L) - (up.pos >> L) + 1 : ((int64_t)kv.seq >> L);
+  const int64_t items = (int64_t)U * nblk * lanes;
   const int threads = 256;
   const int64_t blocks = (items + threads - 1) / threads;
-  dwt_kernel<T, L><<<(unsigned)blocks, threads, 0, s>>>(
-      static_cast<const T*>(K), kv.stride_b, kv.stride_h, kv.stride_s, kv.heads, kv.seq, kv.head_dim,
-      static_cast<T*>(coeffs), rows_total, items);
+  if (up.count > 0) {
+    Update<T> u2 = up;
+    u2.blk0 = up.pos >> L;
+    dwt_kernel<T, L, true><<<(unsigned)blocks, threads, 0, s>>>(
+        static_cast<const T*>(K), static_cast<T*>(K_out), kv.stride_b, kv.stride_h, kv.stride_s, kv.heads, kv.seq,
+        kv.head_dim, static_cast<T*>(coeffs), rows_total, nblk, items, u2);
+  } else {
+    dwt_kernel<T, L, false><<<(unsigned)blocks, threads, 0, s>>>(
+        static_cast<const T*>(K), nullptr, kv.stride_b, kv.stride_h, kv.stride_s, kv.heads, kv.seq, kv.head_dim,
+        static_cast<T*>(coeffs), rows_total, nblk, items, up);
+  }
   return cudaGetLastError();
 }
 
 template <typename T>
-cudaError_t dispatch(const void* K, const wf_tensor& kv, int levels, void* coeffs, cudaStream_t s) {
+cudaError_t dispatch(const void* K, void* K_out, const wf_tensor& kv, int levels, void* coeffs, const Update<T>& up,
+                     cudaStream_t s) {
   switch (levels) {
-    case 1: return run<T, 1>(K, kv, coeffs, s);
-    case 2: return run<T, 2>(K, kv, coeffs, s);
-    case 3: return run<T, 3>(K, kv, coeffs, s);
-    case 4: return run<T, 4>(K, kv, coeffs, s);
-    case 5: return run<T, 5>(K, kv, coeffs, s);
-    case 6: return run<T, 6>(K, kv, coeffs, s);
-    case 7: return run<T, 7>(K, kv, coeffs, s);
-    case 8: return run<T, 8>(K, kv, coeffs, s);
-    case 9: return run<T, 9>(K, kv, coeffs, s);
-    case 10: return run<T, 10>(K, kv, coeffs, s);
+    case 1: return run<T, 1>(K, K_out, kv, coeffs, up, s);
+    case 2: return run<T, 2>(K, K_out, kv, coeffs, up, s);
+    case 3: return run<T, 3>(K, K_out, kv, coeffs, up, s);
+    case 4: return run<T, 4>(K, K_out, kv, coeffs, up, s);
+    case 5: return run<T, 5>(K, K_out, kv, coeffs, up, s);
+    case 6: return run<T, 6>(K, K_out, kv, coeffs, up, s);
+    case 7: return run<T, 7>(K, K_out, kv, coeffs, up, s);
+    case 8: return run<T, 8>(K, K_out, kv, coeffs, up, s);
+    case 9: return run<T, 9>(K, K_out, kv, coeffs, up, s);
+    case 10: return run<T, 10>(K, K_out, kv, coeffs, up, s);
     default: return cudaErrorInvalidValue;
   }
+}
+
+template <typename T>
+Update<T> make_update(const void* Kn, const void* Vn, void* V, const wf_tensor* nt, int64_t pos) {
+  Update<T> up{};
+  if (nt) {
+    up.Kn = static_cast<const T*>(Kn);
+    up.Vn = static_cast<const T*>(Vn);
+    up.V = static_cast<T*>(V);
+    up.nsb = nt->stride_b;
+    up.nsh = nt->stride_h;
+    up.nss = nt->stride_s;
+    up.pos = pos;
+    up.count = nt->seq;
+  }
+  return up;
 }
 
 }  // namespace
 
 cudaError_t launch_dwt(const void* K, const wf_tensor& kv, int levels, void* coeffs, cudaStream_t s) {
-  if (kv.dtype == WF_BF16) return dispatch<bf16>(K, kv, levels, coeffs, s);
-  return dispatch<float>(K, kv, levels, coeffs, s);
+  if (kv.dtype == WF_BF16) return dispatch<bf16>(K, nullptr, kv, levels, coeffs, make_update<bf16>(0, 0, 0, 0, 0), s);
+  return dispatch<float>(K, nullptr, kv, levels, coeffs, make_update<float>(0, 0, 0, 0, 0), s);
+}
+
+cudaError_t launch_cache_update(const void* Kn, const void* Vn, const wf_tensor& nt, void* K, void* V,
+                                const wf_tensor& kv, int64_t pos, int levels, void* coeffs, cudaStream_t s) {
+  if (kv.dtype == WF_BF16)
+    return dispatch<bf16>(K, K, kv, levels, coeffs, make_update<bf16>(Kn, Vn, V, &nt, pos), s);
+  return dispatch<float>(K, K, kv, levels, coeffs, make_update<float>(Kn, Vn, V, &nt, pos), s);
 }
 
 }  // namespace wf

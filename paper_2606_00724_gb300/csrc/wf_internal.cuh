@@ -63,6 +63,9 @@ struct RowSrc {
 
 // DWT pyramid of the keys: see wf_dwt_build.
 cudaError_t launch_dwt(const void* K, const wf_tensor& kv, int levels, void* coeffs, cudaStream_t s);
+// Cache update with the refresh of the touched pyramid blocks: see wf_cache_update.
+cudaError_t launch_cache_update(const void* Kn, const void* Vn, const wf_tensor& nt, void* K, void* V,
+                                const wf_tensor& kv, int64_t pos, int levels, void* coeffs, cudaStream_t s);
 
 // Filter workspace plan for one call.
 struct FilterPlan {

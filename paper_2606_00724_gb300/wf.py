@@ -46,6 +46,7 @@ SIGNATURES = {
     "wf_dwt_build": (_I, [_P, _P, _T, _I, _P, _SZ, _P]),
     "wf_default_schedule": (_I, [_I64, _I, _I64, _P]),
     "wf_level0_schedule": (_I, [_I64, _I, _I64, _P]),
+    "wf_cache_update": (_I, [_P, _P, _T, _P, _P, _T, _I64, _I, _P, _SZ, _P]),
     "wf_schedule_from_proportions": (_I, [_I64, _I, _P, _P]),
     "wf_filter_workspace_bytes": (_SZ, [_T, _T, _I, _P]),
     "wf_filter": (_I, [_P, _T, _P, _P, _T, _I, _P, _P, _P, _P, _SZ, _P]),
@@ -118,6 +119,16 @@ def wf_dwt_build(K: torch.Tensor, levels: int, coeffs: torch.Tensor, stream=None
     d = desc(K)
     _check(lib().wf_dwt_build(_ptr(K), None, ctypes.byref(d), levels, _ptr(coeffs),
                               coeffs.numel() * coeffs.element_size(), _stream(stream)), "wf_dwt_build")
+
+
+def wf_cache_update(Knew: torch.Tensor, Vnew, K: torch.Tensor, V, pos: int, levels: int, coeffs: torch.Tensor,
+                    stream=None) -> None:
+    """Write Knew (and Vnew) into the caches at [pos, pos + count) and refresh
+    the touched pyramid blocks (see the C header)."""
+    dn, dk = desc(Knew), desc(K)
+    _check(lib().wf_cache_update(_ptr(Knew), _ptr(Vnew) if Vnew is not None else None, ctypes.byref(dn), _ptr(K),
+                                 _ptr(V) if V is not None else None, ctypes.byref(dk), pos, levels, _ptr(coeffs),
+                                 coeffs.numel() * coeffs.element_size(), _stream(stream)), "wf_cache_update")
 
 
 def wf_default_schedule(n: int, levels: int, k: int) -> list[int]:

@@ -136,6 +136,27 @@ def test_dwt_build_rejects(lib):
 
 
 @no_gpu
+def test_cache_update_rejects(lib):
+    kv = _desc(1, 2, 64, 128)
+    nt = _desc(1, 2, 8, 128)
+    need = lib.wf_coeffs_bytes(ctypes.byref(kv), 2)
+    F3 = ctypes.c_void_p(0x30000)
+
+    def call(Kn, Vn, n_desc, K, V, pos, L=2, nbytes=need, kv_desc=kv):
+        return lib.wf_cache_update(Kn, Vn, ctypes.byref(n_desc), K, V, ctypes.byref(kv_desc), pos, L, F3, nbytes,
+                                   None)
+    assert call(FAKE, None, nt, FAKE2, None, 57) == -1                     # window past the end
+    assert call(FAKE, None, nt, FAKE2, None, -1) == -1
+    assert call(FAKE, FAKE, nt, FAKE2, None, 0) == -1                      # Vnew without V
+    assert call(None, None, nt, FAKE2, None, 0) == -1
+    assert call(FAKE, None, _desc(1, 3, 8, 128), FAKE2, None, 0) == -2     # other heads
+    assert call(FAKE, None, _desc(1, 2, 8, 128, dtype=wf.WF_F32), FAKE2, None, 0) == -3
+    assert call(ctypes.c_void_p(0x10008), None, nt, FAKE2, None, 0) == -4  # misaligned rows
+    assert call(FAKE, None, nt, FAKE2, None, 0, nbytes=need - 1) == -5
+    assert call(FAKE, None, nt, FAKE2, None, 0, L=0) == -8
+
+
+@no_gpu
 def test_filter_rejects(lib):
     q = _desc(1, 2, 32, 128)
     kv = _desc(1, 2, 1024, 128)
