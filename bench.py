@@ -191,6 +191,55 @@ def make_inputs(w, cfg, device, rank):
     return [synth.make_batch(w, layer=rank, planted=False, device=device, cfg=cfg)]
 
 
+def measure_cache_update(args, w, cfg, device, hbm_peak, peak_kind):
+    """wf_cache_update of R new rows per unit (written into the K/V caches with
+    the touched pyramid blocks refreshed) against a full wf_dwt_build, on one
+    layer of the workload; the window moves by R rows every call."""
+    from paper_2606_00724_gb300 import wf
+    R = args.update_rows
+    lay = (synth.make_batch_fast(w, layer=0, device=device) if cfg == "c5" else
+           synth.make_batch(w, layer=0, planted=False, device=device, cfg=cfg))
+    K, V = lay.K, lay.V
+    dt = K.dtype
+    coeffs = torch.empty(wf.wf_coeffs_bytes(K, w.levels), dtype=torch.uint8, device=device)
+    wf.wf_dwt_build(K, w.levels, coeffs)
+    g = torch.Generator(device=device).manual_seed(7)
+    Kn = torch.randn(w.batch, w.heads, R, w.head_dim, generator=g, device=device).to(dt)
+    Vn = torch.randn(w.batch, w.heads, R, w.head_dim, generator=g, device=device).to(dt)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    row = w.head_dim * K.element_size()
+    blk = 1 << w.levels
+
+    def timed(fn, steps):
+        t = 0.0
+        for i in range(args.warmup + steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn(i)
+            b.record()
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                t += a.elapsed_time(b)
+        return t / steps * 1e3  # us
+
+    assert w.n % R == 0, "--update-rows must divide the context"
+    pos_of = lambda i: (i * R) % w.n  # windows aligned to R
+    upd_us = timed(lambda i: wf.wf_cache_update(Kn, Vn, K, V, pos_of(i), w.levels, coeffs), args.steps)
+    full_us = timed(lambda i: wf.wf_dwt_build(K, w.levels, coeffs), max(3, args.steps // 10))
+    nblk = ((R - 1) >> w.levels) + 1  # 2^L-token blocks an aligned window of R rows touches
+    upd_bytes = w.units * (4 * R * row + (nblk * blk - R) * row + nblk * (blk - 1) * row)
+    full_bytes = w.units * (w.n * row + (w.n - (w.n >> w.levels)) * row)
+    return {"metric": "cache update + incremental pyramid refresh latency (us)", "value": upd_us, "unit": "us",
+            "higher_is_better": False, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "dtype": "bf16" if dt == torch.bfloat16 else "f32", "data": "synthetic",
+            "config": {"workload": w.name, "batch": w.batch, "heads": w.heads, "context": w.n, "levels": w.levels,
+                       "update_rows": R, "l2": "flushed before every timed call (256 MiB write)"},
+            "bytes_per_call": upd_bytes, "achieved_gbs": upd_bytes / upd_us / 1e3,
+            "full_rebuild": {"us": full_us, "bytes": full_bytes, "achieved_gbs": full_bytes / full_us / 1e3,
+                             "peak_gbs": hbm_peak, "peak_kind": peak_kind}}
+
+
 def run_gpu(args, cfg, rank, world, device):
     from paper_2606_00724_gb300 import wf
 
@@ -293,6 +342,10 @@ def main():
     ap.add_argument("--heads", type=int, default=None, help="override the workload's head count")
     ap.add_argument("--schedule", default="default", choices=["default", "level0"],
                     help="kept counts: the default schedule, or the token level as its own selection step")
+    ap.add_argument("--measure", default="step", choices=["step", "cache-update"],
+                    help="step: the filter + sparse-attention step (the metric); cache-update: wf_cache_update of "
+                         "--update-rows rows per unit against a full pyramid rebuild")
+    ap.add_argument("--update-rows", type=int, default=32)
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -360,6 +413,11 @@ def main():
     torch.cuda.set_device(device)
     from paper_2606_00724_gb300 import build as wf_build
     wf_build.build()
+
+    if args.measure == "cache-update":
+        if rank == 0:
+            print(json.dumps(measure_cache_update(args, w, cfg, device, hbm_peak, peak_kind)))
+        return
 
     r = run_gpu(args, cfg, rank, world, device)
     total_ms = r["total_ms"]
