@@ -261,3 +261,26 @@ def sparse_attn(Q, K, V, mu0, Kg=None, Vg=None):
                                        _p(Kg) if Kg.shape[0] else None, _p(Vg) if Vg.shape[0] else None,
                                        Kg.shape[0], _p(O)), "sparse_attn")
     return O
+
+
+def filter_gqa(Qh, pyr, K, n: int, L: int, keep, want_sets: bool = False, want_w: bool = False):
+    """Filtering for one KV head shared by G query heads (grouped-query
+    attention, as in the Dream base model the paper evaluates, Section 4.1).
+
+    Eq. 7's softmax is taken for every query row of every head of the group,
+    and Eq. 8's column sum runs over all of those rows: the KV head's
+    importance W is the sum of its heads' W.  Qh is [G, q, d] (head after
+    head) or already [G*q, d]; the rows are stacked and filtered as one query
+    block, which is that sum.  Same outputs as ``filter``.
+    """
+    Qh = _f64(Qh)
+    Qs = np.ascontiguousarray(Qh.reshape(-1, Qh.shape[-1]))
+    return filter(Qs, pyr, K, n, L, keep, want_sets=want_sets, want_w=want_w)
+
+
+def sparse_attn_gqa(Qh, K, V, mu0, Kg=None, Vg=None):
+    """Final attention of each query head of a group over the rows its KV head
+    kept (Algorithm 1, final step, once per query head).  Qh: [G, q, d];
+    returns [G, q, d]."""
+    Qh = _f64(Qh)
+    return np.stack([sparse_attn(Qh[g], K, V, mu0, Kg, Vg) for g in range(Qh.shape[0])])

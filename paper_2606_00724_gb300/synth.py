@@ -37,10 +37,15 @@ class Workload:
     layers: int = 1
     refresh_every: int = 0
     extra: dict = field(default_factory=dict)
+    group: int = 1    # query heads per KV head (grouped-query attention); `heads` counts KV heads
 
     @property
     def k(self) -> int:
         return int(self.keep[0])
+
+    @property
+    def q_heads(self) -> int:
+        return self.heads * self.group
 
     @property
     def units(self) -> int:
@@ -62,9 +67,14 @@ WORKLOADS = {
                    "drift", extra={"period": 4096, "needles": 128, "gap_growth": 2.0 ** 0.5}),
     "c5": Workload("c5_llada_32layer_n32k_b4", 4, 32, 128, 32768, 32, 32, 4, (1638, 819, 868, 917, 969), "bf16",
                    "iid", layers=32, refresh_every=8),
+    # Grouped-query attention with the Dream-7B head layout (28 query heads
+    # sharing 4 KV heads, head_dim 128): one selection per KV head.
+    "g1": Workload("g1_dream_gqa_n32k_b8", 8, 4, 128, 32768, 32, 32, 4, (2048, 1024, 1024, 1024, 1024), "bf16",
+                   "clusters", extra={"centroids": 64, "seg_min": 256, "seg_max": 2048, "needle_frac": 0.001,
+                                      "gap_growth": 2.0 ** 0.5}, group=7),
 }
 
-CONFIG_NUMBER = {"c1": 1, "c2": 2, "c3": 3, "c4": 4, "c5": 5}
+CONFIG_NUMBER = {"c1": 1, "c2": 2, "c3": 3, "c4": 4, "c5": 5, "g1": 6}
 
 # Planted ladder constants: every query gets a component PLANT_C along the
 # unit direction u; each chosen scale-b block gets a bonus that lifts its
@@ -82,8 +92,8 @@ def unit_seed(cfg: str, layer: int, b: int, h: int, salt: int = 0) -> int:
 
 @dataclass
 class Unit:
-    """One (batch, head) unit, fp32 tensors before storage rounding."""
-    Q: torch.Tensor       # [q, d]
+    """One (batch, KV head) unit, fp32 tensors before storage rounding."""
+    Q: torch.Tensor       # [group * q, d]: the q rows of each query head of the group, head after head
     K: torch.Tensor       # [n, d]
     V: torch.Tensor       # [n, d]
     Kg: torch.Tensor      # [ng, d]
@@ -118,6 +128,7 @@ def make_unit(w: Workload, b: int, h: int, layer: int = 0, planted: bool = True,
     g = torch.Generator(device=dev)
     g.manual_seed(unit_seed(cfg, layer, b, h))
     d, n, q, ng = w.head_dim, w.n, w.q, w.ng
+    qr = q * w.group  # query rows of the unit
     f32 = torch.float32
 
     def randn(*shape):
@@ -126,7 +137,7 @@ def make_unit(w: Workload, b: int, h: int, layer: int = 0, planted: bool = True,
     def randint(lo, hi, shape):
         return torch.randint(lo, hi, shape, generator=g, device=dev)
 
-    Q = randn(q, d)
+    Q = randn(qr, d)
     V = randn(n, d)
     Kg = randn(ng, d)
     Vg = randn(ng, d)
@@ -138,7 +149,7 @@ def make_unit(w: Workload, b: int, h: int, layer: int = 0, planted: bool = True,
         omega = (10000.0 ** (-2.0 * torch.arange(d // 2, device=dev, dtype=torch.float64) / d)) * (
             0.5 + torch.rand(d // 2, generator=g, device=dev, dtype=torch.float64))
         K = _rope(K, torch.arange(n, device=dev), omega)
-        Q = _rope(Q, torch.arange(n, n + q, device=dev), omega)
+        Q = _rope(Q, torch.arange(n, n + q, device=dev).repeat(w.group), omega)
         Kg = _rope(Kg, torch.arange(n, n + ng, device=dev), omega)
     elif w.kind == "clusters":
         cent = randn(w.extra["centroids"], d)
@@ -174,7 +185,7 @@ def make_unit(w: Workload, b: int, h: int, layer: int = 0, planted: bool = True,
         starts = starts.clamp(max=n - span)
         needles = (starts[:, None] + torch.arange(span, device=dev)[None, :]).reshape(-1).unique()
     if needles.numel():
-        rows = randint(0, q, (needles.numel(),))
+        rows = randint(0, qr, (needles.numel(),))
         K[needles] = _needle_keys(Q, rows, d)
 
     targets = None
@@ -273,11 +284,13 @@ class Batch:
 
 def make_batch(w: Workload, layer: int = 0, planted: bool = True, device="cpu", cfg: str | None = None,
                units: list | None = None) -> Batch:
-    """Draw every unit (or only `units`, others left zero) of one layer."""
+    """Draw every unit (or only `units`, others left zero) of one layer.  Q
+    has heads * group query heads; query head h * group + g belongs to KV
+    head h."""
     dt = storage_dtype(w)
-    B, H, d = w.batch, w.heads, w.head_dim
+    B, H, d, G = w.batch, w.heads, w.head_dim, w.group
     dev = torch.device(device)
-    Q = torch.zeros(B, H, w.q, d, dtype=dt, device=dev)
+    Q = torch.zeros(B, H * G, w.q, d, dtype=dt, device=dev)
     K = torch.zeros(B, H, w.n, d, dtype=dt, device=dev)
     V = torch.zeros(B, H, w.n, d, dtype=dt, device=dev)
     Kg = torch.zeros(B, H, w.ng, d, dtype=dt, device=dev)
@@ -288,7 +301,7 @@ def make_batch(w: Workload, layer: int = 0, planted: bool = True, device="cpu", 
             if units is not None and b * H + h not in units:
                 continue
             u = make_unit(w, b, h, layer, planted, dev, cfg)
-            Q[b, h] = u.Q.to(dt)
+            Q[b, h * G:(h + 1) * G] = u.Q.to(dt).view(G, w.q, d)
             K[b, h] = u.K.to(dt)
             V[b, h] = u.V.to(dt)
             Kg[b, h] = u.Kg.to(dt)
@@ -306,7 +319,7 @@ def make_batch_fast(w: Workload, layer: int = 0, device="cuda", seed_salt: int =
     g.manual_seed(unit_seed("c5", layer, 0, 0, 1 + seed_salt))
     B, H, d = w.batch, w.heads, w.head_dim
 
-    def rn(rows):
-        return torch.randn(B, H, rows, d, generator=g, device=dev, dtype=torch.float32).to(dt)
+    def rn(rows, heads=H):
+        return torch.randn(B, heads, rows, d, generator=g, device=dev, dtype=torch.float32).to(dt)
 
-    return Batch(rn(w.q), rn(w.n), rn(w.n), rn(w.ng), rn(w.ng), [None] * (B * H))
+    return Batch(rn(w.q, w.q_heads), rn(w.n), rn(w.n), rn(w.ng), rn(w.ng), [None] * (B * H))
