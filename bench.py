@@ -62,7 +62,7 @@ def unit_bytes(w: synth.Workload) -> dict:
     cands = [w.n >> L] + [2 * keep[b + 1] for b in range(L - 1, 0, -1)]
     trim = 2 * keep[1] if keep[0] < 2 * keep[1] else 0
     k = keep[0]
-    q = w.q * row
+    q = w.q * w.group * row  # the query rows (and output rows) of every query head of the unit's group
     coeff = sum(cands) * row
     filt = q + coeff + trim * row + 4 * k
     attn = q + 4 * k + 2 * k * row + 2 * w.ng * row + q
@@ -72,8 +72,9 @@ def unit_bytes(w: synth.Workload) -> dict:
 
 
 def fused_eligible(w: synth.Workload) -> bool:
-    """wf_step runs its single fused kernel for bf16, head_dim 128, <= 32 query rows."""
-    return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32
+    """wf_step runs its single fused kernel for bf16, head_dim 128, <= 32 query
+    rows and one query head per key head."""
+    return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group == 1
 
 
 def recorded_traffic(w: synth.Workload):
@@ -173,8 +174,13 @@ def oracle_units_seconds(w: synth.Workload, cfg: str, budget_s: float, max_units
         Q, K, V, Kg, Vg = (t.to(dt).double().numpy() for t in (unit.Q, unit.K, unit.V, unit.Kg, unit.Vg))
         pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, w.dtype == "bf16").astype(np.float64)
         t0 = time.perf_counter()
-        mu0 = oracle.filter(Q, pyr, K, w.n, w.levels, np.array(w.keep))
-        oracle.sparse_attn(Q, K, V, mu0, Kg, Vg)
+        if w.group > 1:
+            Qh = Q.reshape(w.group, w.q, w.head_dim)
+            mu0 = oracle.filter_gqa(Qh, pyr, K, w.n, w.levels, np.array(w.keep))
+            oracle.sparse_attn_gqa(Qh, K, V, mu0, Kg, Vg)
+        else:
+            mu0 = oracle.filter(Q, pyr, K, w.n, w.levels, np.array(w.keep))
+            oracle.sparse_attn(Q, K, V, mu0, Kg, Vg)
         spent += time.perf_counter() - t0
         done += 1
         u += 1
@@ -370,7 +376,8 @@ def main():
     ub = unit_bytes(w)
     hbm_peak, peak_kind = peaks()
 
-    config = {"workload": w.name, "batch": w.batch, "heads": w.heads, "head_dim": w.head_dim,
+    config = {"workload": w.name, "batch": w.batch, "heads": w.heads, "query_heads": w.q_heads,
+              "head_dim": w.head_dim,
               "context": w.n, "query_block": w.q, "generation_rows": w.ng, "levels": w.levels, "k": w.k,
               "keep": list(w.keep), "layers": w.layers, "storage": w.dtype,
               "step": ("wf_step (one fused filter + sparse-attention kernel) per layer" if fused_eligible(w) else

@@ -155,8 +155,14 @@ wf_status wf_level0_schedule(int64_t n, int levels, int64_t k, int32_t* keep);
  * C_0 holds 2 keep[1] token positions; if keep[0] < 2 keep[1] the same
  * scoring on the raw keys K[C_0] keeps the top keep[0] of them.
  *
- * Inputs: Q [B,H,q,d] (descriptor q), coeffs from wf_dwt_build on K with the
- * same levels, K [B,H,n,d] (descriptor kv; read only by the level-0 trim).
+ * Inputs: Q [B,Hq,q,d] (descriptor q), coeffs from wf_dwt_build on K with
+ * the same levels, K [B,H,n,d] (descriptor kv; read only by the level-0 trim).
+ * Grouped-query attention: Hq may be any multiple G of the H key heads.
+ * Query head h G + g (g < G) belongs to key head h. A unit is one (batch,
+ * key head), and its query rows i are the q rows of each of its G query
+ * heads: Eq. 7's softmax is per row, and Eq. 8's sum runs over all G q rows,
+ * so one selection serves the whole group. Limits: q <= 64 and G q <= 256
+ * (else WF_ERR_UNSUPPORTED); Hq not a multiple of H gives WF_ERR_SHAPE.
  * keep: host array of levels+1 counts (e.g. from wf_default_schedule).
  * Outputs: idx int32 [B*H][keep[0]] token positions, ascending per unit.
  * level_sets (optional, NULL to skip): int32
@@ -172,11 +178,14 @@ wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const
 /* ---------------------------------------------------------------------------
  * 4. Sparse attention (Algorithm 1, final step; Eq. 3 form).
  *
- * For every unit: K_s = [K[idx[0..k)]; Kg], V_s = [V[idx[0..k)]; Vg] and
+ * For every query head (b, hq), with key head h = hq / G (G = Hq / H, as in
+ * wf_filter): K_s = [K[idx[b H + h][0..k)]; Kg], V_s likewise from V and Vg
+ * (both at key head h), and
  *   O = softmax(Q K_s^T * scale) V_s      (fp32 logits, softmax, accumulation)
  * with scale = 1/sqrt(d) when the argument is 0.  No mask (the DLMs attend
- * bidirectionally).  idx: int32 [B*H][k], each entry in [0, n) (any order).
- * Kg, Vg: [B,H,n_g,d] (descriptor g, may be NULL when n_g = 0).  O: [B,H,q,d]
+ * bidirectionally).  Q: [B,Hq,q,d], q <= 64.  K, V: [B,H,n,d].
+ * idx: int32 [B*H][k], each entry in [0, n) (any order).
+ * Kg, Vg: [B,H,n_g,d] (descriptor g, may be NULL when n_g = 0).  O: [B,Hq,q,d]
  * (descriptor o: same shape and dtype as Q), written rounded to that dtype.
  * ws: device scratch of at least wf_attn_workspace_bytes() bytes.
  * Out-of-range idx entries are clamped to [0, n) (never read out of bounds).
@@ -222,9 +231,10 @@ wf_status wf_sparse_attn_noalloc(const void* Q, const wf_tensor* q, const void* 
  * NULL) and O exactly as wf_filter + wf_sparse_attn define them.  Same
  * arguments and rules as those calls; ws must hold wf_step_workspace_bytes().
  *
- * For bf16 with head_dim 128 and at most 32 query rows the filter and the
- * attention run as one fused kernel (one thread-block cluster per (batch,
- * head)); other shapes run the per-stage kernels.  The fused kernel's waits
+ * For bf16 with head_dim 128, at most 32 query rows and one query head per
+ * key head, the filter and the attention run as one fused kernel (one
+ * thread-block cluster per (batch, head)); other shapes, grouped query
+ * heads included, run the per-stage kernels.  The fused kernel's waits
  * (on copies, tensor-core completion and the cluster's exchanges) are
  * bounded: if one gives up (it never should), the kernel returns early,
  * outputs are undefined, and a status word in the first 4 bytes of ws is set;

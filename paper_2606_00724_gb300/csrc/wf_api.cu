@@ -32,6 +32,13 @@ bool same_units(const wf_tensor* a, const wf_tensor* b) {
   return a->batch == b->batch && a->heads == b->heads && a->head_dim == b->head_dim;
 }
 
+// Query heads per KV head (grouped-query attention), or 0 if the query
+// descriptor q cannot be grouped onto kv.
+int group_of(const wf_tensor* q, const wf_tensor* kv) {
+  if (q->batch != kv->batch || q->head_dim != kv->head_dim || q->heads % kv->heads) return 0;
+  return q->heads / kv->heads;
+}
+
 wf_status check_levels(const wf_tensor* kv, int levels) {
   if (levels < 1 || levels > 10) return WF_ERR_UNSUPPORTED;
   const int64_t n = kv->seq;
@@ -58,9 +65,10 @@ wf_status check_filter_args(const wf_tensor* q, const wf_tensor* kv, int levels,
   wf_status st;
   if ((st = check_desc(q, false)) != WF_OK) return st;
   if ((st = check_desc(kv, false)) != WF_OK) return st;
-  if (!same_units(q, kv)) return WF_ERR_SHAPE;
+  const int G = group_of(q, kv);
+  if (!G) return WF_ERR_SHAPE;
   if (q->dtype != kv->dtype) return WF_ERR_DTYPE;
-  if (q->seq > wf::kMaxQ) return WF_ERR_UNSUPPORTED;
+  if (q->seq > wf::kMaxQ || (int64_t)G * q->seq > wf::kMaxQR) return WF_ERR_UNSUPPORTED;
   if ((st = check_levels(kv, levels)) != WF_OK) return st;
   return check_keep(kv->seq, levels, keep);
 }
@@ -71,13 +79,13 @@ wf_status check_attn_args(const wf_tensor* q, const wf_tensor* kv, int k, const 
   if ((st = check_desc(q, false)) != WF_OK) return st;
   if ((st = check_desc(kv, false)) != WF_OK) return st;
   if ((st = check_desc(o, false)) != WF_OK) return st;
-  if (!same_units(q, kv) || !same_units(q, o) || o->seq != q->seq) return WF_ERR_SHAPE;
+  if (!group_of(q, kv) || !same_units(q, o) || o->seq != q->seq) return WF_ERR_SHAPE;
   if (q->dtype != kv->dtype || o->dtype != q->dtype) return WF_ERR_DTYPE;
   if (q->seq > wf::kMaxQ) return WF_ERR_UNSUPPORTED;
   if (k < 1 || k > kv->seq || n_g < 0) return WF_ERR_INVALID_ARG;
   if (n_g > 0) {
     if ((st = check_desc(g, true)) != WF_OK) return st;
-    if (!same_units(q, g) || g->seq != n_g) return WF_ERR_SHAPE;
+    if (!same_units(kv, g) || g->seq != n_g) return WF_ERR_SHAPE;
     if (g->dtype != q->dtype) return WF_ERR_DTYPE;
   }
   return WF_OK;
@@ -208,7 +216,7 @@ WF_API wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs
 
 WF_API size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g) {
   if (check_desc(q, false) != WF_OK || k < 1 || n_g < 0 || q->seq > wf::kMaxQ) return 0;
-  return wf::plan_attn(*q, k, n_g).total;
+  return wf::plan_attn(*q, k, n_g, 1).total;  // the size does not depend on the grouping
 }
 
 WF_API wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const void* V,
@@ -225,7 +233,7 @@ WF_API wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || (reinterpret_cast<uintptr_t>(idx) & 3u) != 0)
     return WF_ERR_ALIGN;
   if (!(scale >= 0.f) || isinf(scale)) return WF_ERR_INVALID_ARG;
-  const wf::AttnPlan p = wf::plan_attn(*q, k, n_g);
+  const wf::AttnPlan p = wf::plan_attn(*q, k, n_g, group_of(q, kv));
   if (ws_bytes < p.total) return WF_ERR_WORKSPACE;
   const float sc = scale == 0.f ? 1.0f / sqrtf((float)q->head_dim) : scale;
   return cuda_status(wf::launch_attn(p, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, ws,
@@ -241,7 +249,7 @@ WF_API size_t wf_step_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, i
                                       int n_g) {
   if (check_filter_args(q, kv, levels, keep) != WF_OK || n_g < 0) return 0;
   const size_t f = wf::plan_filter(*q, *kv, levels, keep).total;
-  const size_t a = wf::plan_attn(*q, keep[0], n_g).total;
+  const size_t a = wf::plan_attn(*q, keep[0], n_g, 1).total;
   return kStatusBytes + (f > a ? f : a);
 }
 
@@ -271,8 +279,9 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   void* scratch = static_cast<char*>(ws) + kStatusBytes;
   cudaError_t e = cudaSuccess;
   if (refresh_coeffs && (e = wf::launch_dwt(K, *kv, levels, coeffs, s)) != cudaSuccess) return WF_ERR_CUDA;
+  // The fused kernel takes one query head per KV head; grouped heads run the per-stage kernels.
   const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, n_g, n_g > 0 ? g : nullptr, sms);
-  if (fp.ok) {
+  if (fp.ok && q->heads == kv->heads) {
     e = wf::launch_fused(fp, Q, *q, K, V, *kv, Kg, Vg, n_g > 0 ? g : nullptr, coeffs, levels, keep, idx,
                          level_sets, O, *o, status, s);
     return cuda_status(e);
@@ -280,7 +289,7 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
   if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, s)) != cudaSuccess)
     return WF_ERR_CUDA;
-  const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g);
+  const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g, group_of(q, kv));
   const float sc = 1.0f / sqrtf((float)q->head_dim);
   e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, s);
   return cuda_status(e);

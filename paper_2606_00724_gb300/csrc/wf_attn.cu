@@ -22,7 +22,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
     const T* __restrict__ Q, int64_t qsb, int64_t qsh, int64_t qss, const T* __restrict__ K,
     const T* __restrict__ V, int64_t ksb, int64_t ksh, int64_t kss, int n, const int32_t* __restrict__ idx, int k,
     const T* __restrict__ Kg, const T* __restrict__ Vg, int64_t gsb, int64_t gsh, int64_t gss, int ng, int q, int H,
-    float scale, int nsplit, float* __restrict__ Opart, float2* __restrict__ ML) {
+    int G, float scale, int nsplit, float* __restrict__ Opart, float2* __restrict__ ML) {
   constexpr int VEC = Vec<T>::N;
   constexpr int KS = D + 4;
   extern __shared__ __align__(16) float smem[];
@@ -36,6 +36,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
   const int total = k + ng;
   const int cnt = min(CH, total - t0);
   const int64_t bb = u / H, hh = u % H;
+  const int64_t hk = hh / G;  // the KV head of this query head
   const int tid = threadIdx.x;
 
   const T* qbase = Q + bb * qsb + hh * qsh;
@@ -49,7 +50,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
 #pragma unroll
     for (int x = 0; x < VEC; ++x) Qs[i * D + c + x] = v[x];
   }
-  const int32_t* ui = idx + (int64_t)u * k;
+  const int32_t* ui = idx + (bb * (H / G) + hk) * k;
   for (int e = tid; e < CH * (D / VEC); e += blockDim.x) {
     const int j = e / (D / VEC), c = (e % (D / VEC)) * VEC;
     float kv[VEC], vv[VEC];
@@ -59,10 +60,10 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
       if (t < k) {
         int r = ui[t];
         r = r < 0 ? 0 : (r >= n ? n - 1 : r);
-        const int64_t o = bb * ksb + hh * ksh + (int64_t)r * kss + c;
+        const int64_t o = bb * ksb + hk * ksh + (int64_t)r * kss + c;
         kp = K + o; vp = V + o;
       } else {
-        const int64_t o = bb * gsb + hh * gsh + (int64_t)(t - k) * gss + c;
+        const int64_t o = bb * gsb + hk * gsh + (int64_t)(t - k) * gss + c;
         kp = Kg + o; vp = Vg + o;
       }
       ld_vec(kp, kv);
@@ -169,7 +170,7 @@ cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const voi
   attn_split_kernel<T, D><<<dim3(p.nsplit, p.U), 256, smem, s>>>(
       static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, static_cast<const T*>(K),
       static_cast<const T*>(V), kv.stride_b, kv.stride_h, kv.stride_s, kv.seq, idx, p.k, static_cast<const T*>(Kg),
-      static_cast<const T*>(Vg), gsb, gsh, gss, p.ng, p.q, p.H, scale, p.nsplit, Opart, ML);
+      static_cast<const T*>(Vg), gsb, gsh, gss, p.ng, p.q, p.H, p.G, scale, p.nsplit, Opart, ML);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   attn_combine_kernel<T><<<p.U, 256, 0, s>>>(Opart, ML, p.nsplit, p.q, D, p.H, static_cast<T*>(O), od.stride_b,
                                              od.stride_h, od.stride_s);
@@ -178,10 +179,11 @@ cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const voi
 
 }  // namespace
 
-AttnPlan plan_attn(const wf_tensor& q, int k, int ng) {
+AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group) {
   AttnPlan p{};
   p.U = q.batch * q.heads;
   p.H = q.heads;
+  p.G = group;
   p.q = q.seq;
   p.d = q.head_dim;
   p.k = k;

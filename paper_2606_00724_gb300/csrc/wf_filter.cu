@@ -22,9 +22,18 @@ namespace {
 constexpr int TILE = kScoreTile;
 constexpr int QMAX = kMaxQ;
 
+// Query row i of unit (b, h): row i % qs of query head h G + i / qs.
+template <typename T>
+__device__ __forceinline__ const T* query_row(const T* Q, int64_t qsb, int64_t qsh, int64_t qss, int64_t bb,
+                                              int64_t hh, int G, int qs, int i) {
+  return Q + bb * qsb + (hh * G + i / qs) * qsh + (int64_t)(i % qs) * qss;
+}
+
+// Grid (candidate tiles, units, query chunks of QMAX rows).
 template <typename T, int D>
 __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int64_t qsb, int64_t qsh, int64_t qss,
-                                                    int q, int H, RowSrc src, const int32_t* __restrict__ cand,
+                                                    int q, int G, int qs, int H, RowSrc src,
+                                                    const int32_t* __restrict__ cand,
                                                     int64_t cand_stride, int m, float scale,
                                                     float* __restrict__ logits, int64_t lg_unit, int64_t lg_row,
                                                     float2* __restrict__ part, int64_t part_unit) {
@@ -35,14 +44,14 @@ __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int
   float* Rs = smem + QMAX * D;   // [TILE][RS]
   const int u = blockIdx.y;
   const int j0 = blockIdx.x * TILE;
+  const int i0 = blockIdx.z * QMAX;  // first query row of this chunk
   const int64_t bb = u / H, hh = u % H;
   const int tid = threadIdx.x;
 
-  const T* qbase = Q + bb * qsb + hh * qsh;
   for (int e = tid; e < QMAX * (D / VEC); e += blockDim.x) {
     const int i = e / (D / VEC), c = (e % (D / VEC)) * VEC;
     float v[VEC];
-    if (i < q) ld_vec(qbase + (int64_t)i * qss + c, v);
+    if (i0 + i < q) ld_vec(query_row(Q, qsb, qsh, qss, bb, hh, G, qs, i0 + i) + c, v);
     else
 #pragma unroll
       for (int x = 0; x < VEC; ++x) v[x] = 0.f;
@@ -88,7 +97,7 @@ __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int
   float2* pt = part + (int64_t)u * part_unit + (int64_t)blockIdx.x * q;
 #pragma unroll
   for (int r = 0; r < QMAX / 8; ++r) {
-    const int i = warp + 8 * r;
+    const int i = i0 + warp + 8 * r;
     if (i >= q) break;
     const float s = acc[r] * scale;
     if (valid) lg[(int64_t)i * lg_row + jj] = s;
@@ -111,7 +120,7 @@ __global__ void __launch_bounds__(256) weights_kernel(const float* __restrict__ 
   // log W_j = log sum_i exp(s_ij - M_i - log S_i), evaluated as a
   // log-sum-exp over the query rows: the same order as W_j, without the
   // underflow that would turn very small weights into ties.
-  __shared__ float Ms[QMAX];
+  __shared__ float Ms[kMaxQR];
   const int u = blockIdx.y;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float2* pt = part + (int64_t)u * part_unit;
@@ -133,19 +142,12 @@ __global__ void __launch_bounds__(256) weights_kernel(const float* __restrict__ 
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= m) return;
   const float* lg = logits + (int64_t)u * lg_unit + j;
-  float t[QMAX];
   float mx = -INFINITY;
-#pragma unroll
-  for (int i = 0; i < QMAX; ++i) {
-    if (i < q) {
-      t[i] = lg[(int64_t)i * lg_row] - Ms[i];
-      mx = fmaxf(mx, t[i]);
-    }
-  }
+#pragma unroll 8
+  for (int i = 0; i < q; ++i) mx = fmaxf(mx, lg[(int64_t)i * lg_row] - Ms[i]);
   float z = 0.f;
-#pragma unroll
-  for (int i = 0; i < QMAX; ++i)
-    if (i < q) z += expf(t[i] - mx);
+#pragma unroll 8
+  for (int i = 0; i < q; ++i) z += expf((lg[(int64_t)i * lg_row] - Ms[i]) - mx);
   W[(int64_t)u * w_unit + j] = mx + logf(z);
 }
 
@@ -253,9 +255,9 @@ cudaError_t run_score(const FilterPlan& p, const void* Q, const wf_tensor& qd, R
   const size_t smem = sizeof(float) * (size_t)(QMAX * D + TILE * (D + 4));
   cudaError_t e = cudaFuncSetAttribute(score_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((m + TILE - 1) / TILE, p.U);
+  dim3 grid((m + TILE - 1) / TILE, p.U, (p.q + QMAX - 1) / QMAX);
   score_kernel<T, D><<<grid, 256, smem, s>>>(static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, p.q,
-                                             p.H, src, cand, p.cmax, m, 1.0f / sqrtf((float)D), logits,
+                                             p.G, p.qs, p.H, src, cand, p.cmax, m, 1.0f / sqrtf((float)D), logits,
                                              (int64_t)p.q * p.cmax, p.cmax, part, (int64_t)p.tiles_max * p.q);
   return cudaGetLastError();
 }
@@ -276,7 +278,9 @@ FilterPlan plan_filter(const wf_tensor& q, const wf_tensor& kv, int levels, cons
   FilterPlan p{};
   p.U = kv.batch * kv.heads;
   p.H = kv.heads;
-  p.q = q.seq;
+  p.G = q.heads / kv.heads;
+  p.qs = q.seq;
+  p.q = p.G * q.seq;
   p.d = kv.head_dim;
   p.n = kv.seq;
   p.L = levels;

@@ -67,9 +67,11 @@ cudaError_t launch_dwt(const void* K, const wf_tensor& kv, int levels, void* coe
 cudaError_t launch_cache_update(const void* Kn, const void* Vn, const wf_tensor& nt, void* K, void* V,
                                 const wf_tensor& kv, int64_t pos, int levels, void* coeffs, cudaStream_t s);
 
-// Filter workspace plan for one call.
+// Filter workspace plan for one call.  A unit is one (batch, KV head); its
+// query block is the qs rows of each of its G query heads, q = G qs rows.
 struct FilterPlan {
   int U, H, q, d, n, L, dtype;
+  int G, qs;
   int32_t keep[16];
   int cmax;        // largest candidate count over the scales (and the trim)
   int tiles_max;   // ceil(cmax / kScoreTile)
@@ -77,19 +79,22 @@ struct FilterPlan {
   size_t off_cand_a, off_cand_b, off_w, off_logits, off_part, total;
 };
 constexpr int kScoreTile = 32;
-constexpr int kMaxQ = 64;
+constexpr int kMaxQ = 64;    // query rows per query head
+constexpr int kMaxQR = 256;  // query rows per KV head (all heads of a group)
 FilterPlan plan_filter(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep);
 cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* coeffs,
                           const void* K, const wf_tensor& kv, int32_t* idx, int32_t* level_sets, void* ws,
                           cudaStream_t s);
 
-// Sparse attention workspace plan.
+// Sparse attention workspace plan.  A unit is one (batch, query head); it
+// reads KV head h / G and that head's index row.
 struct AttnPlan {
   int U, H, q, d, k, ng, nsplit, dtype;
+  int G;
   size_t off_o, off_ml, total;
 };
 constexpr int kAttnChunk = 64;
-AttnPlan plan_attn(const wf_tensor& q, int k, int ng);
+AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group);
 cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                         const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
                         const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s);

@@ -101,6 +101,10 @@ def test_sizes(lib):
     assert wf.wf_filter_workspace_bytes(Q, K, 4, [2049, 1024, 1024, 1024, 1024]) == 0  # infeasible
     assert wf.wf_filter_workspace_bytes(_meta((2, 32, 65, 128)), K, 4, keep) == 0       # > 64 query rows
     assert wf.wf_attn_workspace_bytes(Q, 2048, 32) > 0
+    # Grouped query heads: 7 per key head (224 rows) fit, 9 (288 rows) do not.
+    assert wf.wf_filter_workspace_bytes(_meta((2, 224, 32, 128)), K, 4, keep) > 0
+    assert wf.wf_filter_workspace_bytes(_meta((2, 288, 32, 128)), K, 4, keep) == 0
+    assert wf.wf_filter_workspace_bytes(_meta((2, 48, 32, 128)), K, 4, keep) == 0   # 48 % 32 != 0
 
 
 # Argument validation returns before any CUDA call.  The pointers below are
@@ -170,6 +174,8 @@ def test_filter_rejects(lib):
     assert call(keep=(ctypes.c_int32 * 3)(129, 64, 91)) == -9    # k > 2 keep[1]
     assert call(keep=(ctypes.c_int32 * 3)(128, 64, 257)) == -9   # keep[2] > n/4
     assert call(q=_desc(1, 3, 32, 128)) == -2                     # heads disagree
+    assert call(q=_desc(1, 18, 32, 128)) == -8                    # 9 heads x 32 rows per key head > 256
+    assert call(q=_desc(2, 4, 32, 128)) == -2                     # batch disagrees
     assert call(q=_desc(1, 2, 32, 128, dtype=wf.WF_F32)) == -3    # dtypes disagree
     assert call(q=_desc(1, 2, 65, 128)) == -8                     # too many query rows
     assert call(L=11) == -8

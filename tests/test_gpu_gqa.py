@@ -1,0 +1,101 @@
+"""GPU parity of grouped-query attention (GQA): one selection per key head
+from the stacked query rows of its G query heads, then every query head
+attends over its key head's selected rows.
+
+Bars: indices bit-exact on planted inputs at every scale (against the planted
+answer and the oracle), outputs within the dtype's bound (fp32 max-abs 1e-5;
+bf16 max-abs 2e-2, rel-L2 1e-2); wf_step gives what wf_filter +
+wf_sparse_attn give."""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import GpuRun, assert_close_out, f64
+from paper_2606_00724_gb300 import synth, wf
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a GPU", allow_module_level=True)
+
+
+def _workload(base, k=None, **kw):
+    w = dataclasses.replace(synth.WORKLOADS[base], **kw)
+    keep = oracle.default_schedule(w.n, w.levels, w.k if k is None else k)
+    return dataclasses.replace(w, keep=tuple(int(x) for x in keep), name=w.name + "_variant")
+
+
+def _check_units(w, batch, run, units, dtype):
+    G = w.group
+    for u in units:
+        b, h = divmod(u, w.heads)
+        Qh = f64(batch.Q[b, h * G:(h + 1) * G])
+        K, V, Kg, Vg = (f64(t[b, h]) for t in (batch.K, batch.V, batch.Kg, batch.Vg))
+        pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, dtype == torch.bfloat16)
+        assert np.array_equal(run.pyramid(u), pyr.astype(np.float64)), f"pyramid unit {u}"
+        mu0, sets = oracle.filter_gqa(Qh, pyr, K, w.n, w.levels, np.array(w.keep), want_sets=True)
+        if run.sets is not None:
+            gsets = run.level_sets(u)
+            for lev in range(w.levels, -1, -1):
+                assert np.array_equal(gsets[lev], sets[lev]), f"unit {u} scale {lev}"
+                assert np.array_equal(gsets[lev], batch.targets[u][lev].cpu().numpy()), f"unit {u} planted {lev}"
+        assert np.array_equal(run.idx[u].cpu().numpy(), mu0), f"unit {u} mu0"
+        O = oracle.sparse_attn_gqa(Qh, K, V, mu0, Kg, Vg)
+        assert_close_out(f64(run.O[b, h * G:(h + 1) * G]), O, dtype)
+
+
+@pytest.mark.parametrize("base,kw,dtype", [
+    # Dream-7B grouping (7 query heads per key head), shorter context.
+    ("g1", dict(batch=2, heads=2, n=4096, levels=3, k=512), torch.bfloat16),
+    # Two heads per key head, head_dim 64, fp32 (the fp32 bar: max-abs 1e-5).
+    ("c1", dict(heads=2, group=2), torch.float32),
+    # Eight heads per key head: 8 x 32 = 256 query rows per key head (the limit).
+    ("g1", dict(batch=1, heads=1, group=8, n=2048, levels=2, k=256), torch.bfloat16),
+])
+def test_gqa_per_stage(base, kw, dtype):
+    w = _workload(base, **kw)
+    cfg = base
+    batch = synth.make_batch(w, planted=True, device="cuda", cfg=cfg)
+    assert batch.Q.dtype == dtype and batch.Q.shape[1] == w.heads * w.group
+    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    torch.cuda.synchronize()
+    _check_units(w, batch, run, range(w.units), dtype)
+    # wf_step takes the per-stage path for grouped heads: same indices, same output.
+    step = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
+    step.step()
+    torch.cuda.synchronize()
+    assert torch.equal(step.idx, run.idx)
+    assert torch.equal(step.sets, run.sets)
+    assert torch.equal(step.O, run.O)
+
+
+def test_gqa_dream_shape_sampled_units():
+    # The full Dream-shaped layer (B8, 28 query heads on 4 key heads, 32K
+    # context): wf_step on the whole layer; sampled units against the oracle.
+    w = synth.WORKLOADS["g1"]
+    units = [0, 13, w.units - 1]
+    batch = synth.make_batch(w, planted=True, device="cuda", cfg="g1", units=units)
+    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().step(refresh=False)
+    torch.cuda.synchronize()
+    _check_units(w, batch, run, units, torch.bfloat16)
+
+
+def test_gqa_attention_equals_repeated_key_heads():
+    # The head mapping of the grouped attention (query head h G + g reads key
+    # head h and its index row) against the ungrouped call on key heads
+    # repeated G times, with the same selection: identical outputs.
+    w = _workload("g1", batch=2, heads=2, group=3, n=2048, levels=2, k=256)
+    batch = synth.make_batch(w, planted=True, device="cuda", cfg="g1")
+    G = w.group
+    grouped = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    rep = lambda t: t.repeat_interleave(G, dim=1).contiguous()
+    K1, V1, Kg1, Vg1 = rep(batch.K), rep(batch.V), rep(batch.Kg), rep(batch.Vg)
+    idx1 = grouped.idx.repeat_interleave(G, dim=0).contiguous()
+    O1 = torch.empty_like(batch.Q)
+    ws = torch.empty(wf.wf_attn_workspace_bytes(batch.Q, w.k, w.ng), dtype=torch.uint8, device="cuda")
+    wf.wf_sparse_attn(batch.Q, K1, V1, idx1, w.k, Kg1, Vg1, O1, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(O1, grouped.O)
