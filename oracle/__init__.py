@@ -63,6 +63,11 @@ def _load():
         "orc_schedule_from_proportions": (I, [I64, I, P, P]),
         "orc_filter_f64": (I, [P, I, I, P, P, I64, I, P, P, P, P]),
         "orc_filter_literal_f64": (I, [P, I, I, P, I64, I, P, P, P]),
+        "orc_wavelet_taps": (I, [I, P, P]),
+        "orc_wavelet_analysis_f64": (I, [P, I64, I, I, I, P, P]),
+        "orc_wavelet_synthesis_f64": (I, [P, P, I64, I, I, I, P]),
+        "orc_wavelet_approx_spec32": (I, [P, I64, I, I, I, I, P]),
+        "orc_filter_wavelet_f64": (I, [P, I, I, P, I64, I, I, P, I, I, P, P]),
         "orc_attention_f64": (I, [P, I, I, P, P, I64, P]),
         "orc_sparse_attn_f64": (I, [P, I, I, P, P, P, I64, P, P, I64, P]),
     }
@@ -284,3 +289,66 @@ def sparse_attn_gqa(Qh, K, V, mu0, Kg=None, Vg=None):
     returns [G, q, d]."""
     Qh = _f64(Qh)
     return np.stack([sparse_attn(Qh[g], K, V, mu0, Kg, Vg) for g in range(Qh.shape[0])])
+
+
+# Other wavelet bases (Eq. 6 / Eq. 11 with a generic psi), periodized.
+HAAR, DB2 = 0, 1
+
+
+def wavelet_taps(wavelet: int):
+    """(h, g) of the orthogonal filter bank: Haar or db2."""
+    h = np.zeros(4)
+    g = np.zeros(4)
+    taps = _load().orc_wavelet_taps(wavelet, _p(h), _p(g))
+    if taps < 0:
+        raise ValueError(f"unknown wavelet {wavelet}")
+    return h[:taps].copy(), g[:taps].copy()
+
+
+def wavelet_analysis(x, wavelet: int, L: int):
+    """L periodized analysis levels: (A, D) in the pyramid layout."""
+    x = _f64(x)
+    n, d = x.shape
+    rows = pyramid_rows(n, L)
+    A = np.zeros((rows, d))
+    D = np.zeros((rows, d))
+    _check(_load().orc_wavelet_analysis_f64(_p(x), n, d, wavelet, L, _p(A), _p(D)), "wavelet_analysis")
+    return A, D
+
+
+def wavelet_synthesis(A, D, n: int, wavelet: int, L: int):
+    A = _f64(A)
+    D = _f64(D)
+    d = A.shape[1]
+    x = np.zeros((n, d))
+    _check(_load().orc_wavelet_synthesis_f64(_p(A), _p(D), n, d, wavelet, L, _p(x)), "wavelet_synthesis")
+    return x
+
+
+def wavelet_approx_spec32(x, wavelet: int, level: int, store_bf16: bool):
+    """Level-`level` approximation rows of x under the library's fp32 storage rule."""
+    x = _f32(x)
+    n, d = x.shape
+    out = np.zeros((n >> level, d), dtype=np.float32)
+    _check(_load().orc_wavelet_approx_spec32(_p(x), n, d, wavelet, level, int(store_bf16), _p(out)),
+           "wavelet_approx_spec32")
+    return out
+
+
+def filter_wavelet(Q, K, L: int, keep, wavelet: int, spec32: bool = True, store_bf16: bool = False,
+                   want_sets: bool = False):
+    """Algorithm 1 with a generic psi, literally (Eq. 11's transform of the
+    gathered keys at every scale).  Returns mu0 (and {b: J_b})."""
+    Q = _f64(Q)
+    K = _f64(K)
+    keep = _i32(keep)
+    q, d = Q.shape
+    n = K.shape[0]
+    mu0 = np.zeros(int(keep[0]), dtype=np.int32)
+    sets = np.zeros(int(keep.sum()), dtype=np.int32) if want_sets else None
+    _check(_load().orc_filter_wavelet_f64(_p(Q), q, d, _p(K), n, L, wavelet, _p(keep), int(spec32),
+                                          int(store_bf16), _p(mu0), _p(sets) if sets is not None else None),
+           "filter_wavelet")
+    if want_sets:
+        return mu0, split_level_sets(sets, L, keep)
+    return mu0

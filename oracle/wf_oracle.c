@@ -424,3 +424,179 @@ int orc_sparse_attn_f64(const double* Q, int q, int d, const double* K, const do
   free(Vs);
   return rc;
 }
+
+/* ------------------------------------------------------------------------ */
+/* Other wavelet bases (Eq. 6, Eq. 11 with a generic psi), periodized.      */
+/* ------------------------------------------------------------------------ */
+int orc_wavelet_taps(int wavelet, double* h, double* g) {
+  if (!h || !g) return -1;
+  if (wavelet == ORC_HAAR) {
+    h[0] = HAAR_C; h[1] = HAAR_C;
+    g[0] = HAAR_C; g[1] = -HAAR_C;
+    return 2;
+  }
+  if (wavelet == ORC_DB2) {
+    const double r = sqrt(3.0), s = 4.0 * sqrt(2.0);
+    h[0] = (1.0 + r) / s; h[1] = (3.0 + r) / s; h[2] = (3.0 - r) / s; h[3] = (1.0 - r) / s;
+    for (int k = 0; k < 4; ++k) g[k] = ((k & 1) ? -1.0 : 1.0) * h[3 - k];
+    return 4;
+  }
+  return -1;
+}
+
+/* One periodized analysis level: len/2 approximation (and detail) rows. */
+static void wavelet_step_f64(const double* x, int64_t len, int d, const double* h, const double* g, int taps,
+                             double* a, double* det) {
+  for (int64_t j = 0; j < len / 2; ++j) {
+    for (int c = 0; c < d; ++c) {
+      double sa = 0.0, sd = 0.0;
+      for (int k = 0; k < taps; ++k) {
+        const double v = x[((2 * j + k) % len) * d + c];
+        sa += h[k] * v;
+        sd += g[k] * v;
+      }
+      a[j * d + c] = sa;
+      if (det) det[j * d + c] = sd;
+    }
+  }
+}
+
+int orc_wavelet_analysis_f64(const double* x, int64_t n, int d, int wavelet, int L, double* A, double* D) {
+  double h[4], g[4];
+  const int taps = orc_wavelet_taps(wavelet, h, g);
+  if (taps < 0 || !x || !A || !D || !shape_ok(n, d, L)) return -1;
+  double* cur = (double*)malloc(sizeof(double) * (size_t)n * d);
+  if (!cur) return -1;
+  memcpy(cur, x, sizeof(double) * (size_t)n * d);
+  int64_t len = n;
+  for (int b = 1; b <= L; ++b) {
+    double* a = A + orc_pyramid_row_offset(n, b) * d;
+    double* det = D + orc_pyramid_row_offset(n, b) * d;
+    wavelet_step_f64(cur, len, d, h, g, taps, a, det);
+    len /= 2;
+    memcpy(cur, a, sizeof(double) * (size_t)len * d);
+  }
+  free(cur);
+  return 0;
+}
+
+int orc_wavelet_synthesis_f64(const double* A, const double* D, int64_t n, int d, int wavelet, int L,
+                              double* x) {
+  double h[4], g[4];
+  const int taps = orc_wavelet_taps(wavelet, h, g);
+  if (taps < 0 || !x || !A || !D || !shape_ok(n, d, L)) return -1;
+  double* cur = (double*)malloc(sizeof(double) * (size_t)n * d);
+  double* nxt = (double*)malloc(sizeof(double) * (size_t)n * d);
+  if (!cur || !nxt) { free(cur); free(nxt); return -1; }
+  memcpy(cur, A + orc_pyramid_row_offset(n, L) * d, sizeof(double) * (size_t)(n >> L) * d);
+  for (int b = L; b >= 1; --b) {
+    const int64_t half = n >> b, len = 2 * half;
+    const double* det = D + orc_pyramid_row_offset(n, b) * d;
+    memset(nxt, 0, sizeof(double) * (size_t)len * d);
+    /* The transpose of the analysis map: every input row receives h[k] a[j] + g[k] det[j]. */
+    for (int64_t j = 0; j < half; ++j)
+      for (int k = 0; k < taps; ++k)
+        for (int c = 0; c < d; ++c)
+          nxt[((2 * j + k) % len) * d + c] += h[k] * cur[j * d + c] + g[k] * det[j * d + c];
+    memcpy(cur, nxt, sizeof(double) * (size_t)len * d);
+  }
+  memcpy(x, cur, sizeof(double) * (size_t)n * d);
+  free(cur);
+  free(nxt);
+  return 0;
+}
+
+int orc_wavelet_approx_spec32(const float* x, int64_t len, int d, int wavelet, int level, int store_bf16,
+                              float* out) {
+  double h[4], g[4];
+  const int taps = orc_wavelet_taps(wavelet, h, g);
+  if (taps < 0 || !x || !out || !shape_ok(len, d, level)) return -1;
+  float h32[4];
+  for (int k = 0; k < taps; ++k) h32[k] = (float)h[k];
+  const float c32 = (float)HAAR_C;
+  float* prev = (float*)malloc(sizeof(float) * (size_t)len * d);
+  float* cur = (float*)malloc(sizeof(float) * (size_t)(len / 2) * d);
+  if (!prev || !cur) { free(prev); free(cur); return -1; }
+  memcpy(prev, x, sizeof(float) * (size_t)len * d);
+  int64_t n = len;
+  for (int b = 1; b <= level; ++b) {
+    const int64_t half = n / 2;
+    for (int64_t j = 0; j < half; ++j) {
+      for (int c = 0; c < d; ++c) {
+        float v;
+        if (wavelet == ORC_HAAR) {
+          const float s = prev[(2 * j) * d + c] + prev[(2 * j + 1) * d + c];
+          v = s * c32;
+        } else {
+          v = h32[0] * prev[((2 * j) % n) * d + c];
+          for (int k = 1; k < taps; ++k) {
+            const float t = h32[k] * prev[((2 * j + k) % n) * d + c];
+            v = v + t;
+          }
+        }
+        cur[j * d + c] = v;
+      }
+    }
+    n = half;
+    memcpy(prev, cur, sizeof(float) * (size_t)n * d);
+  }
+  for (int64_t i = 0; i < n * d; ++i) out[i] = store_bf16 ? orc_round_bf16(prev[i]) : prev[i];
+  free(prev);
+  free(cur);
+  return 0;
+}
+
+int orc_filter_wavelet_f64(const double* Q, int q, int d, const double* K, int64_t n, int L, int wavelet,
+                           const int32_t* keep, int spec32, int store_bf16, int32_t* mu0, int32_t* level_sets) {
+  double h[4], g[4];
+  if (orc_wavelet_taps(wavelet, h, g) < 0) return -1;
+  if (!Q || !K || !keep || !mu0 || q <= 0 || !shape_ok(n, d, L) || !schedule_ok(n, L, keep)) return -1;
+  int64_t cap = n >> L;
+  for (int b = 1; b <= L; ++b) cap = cap > 2 * (int64_t)keep[b] ? cap : 2 * (int64_t)keep[b];
+  int32_t* cand = (int32_t*)malloc(sizeof(int32_t) * (size_t)cap);
+  int32_t* chosen = (int32_t*)malloc(sizeof(int32_t) * (size_t)cap);
+  double* sub = (double*)malloc(sizeof(double) * (size_t)n * d);   /* K[mu^b] */
+  double* A = (double*)malloc(sizeof(double) * (size_t)n * d);
+  double* D = (double*)malloc(sizeof(double) * (size_t)n * d);
+  float* sub32 = (float*)malloc(sizeof(float) * (size_t)n * d);
+  float* a32 = (float*)malloc(sizeof(float) * (size_t)cap * d);
+  double* rows = (double*)malloc(sizeof(double) * (size_t)cap * d);
+  double* W = (double*)malloc(sizeof(double) * (size_t)cap);
+  if (!cand || !chosen || !sub || !A || !D || !sub32 || !a32 || !rows || !W) {
+    free(cand); free(chosen); free(sub); free(A); free(D); free(sub32); free(a32); free(rows); free(W);
+    return -1;
+  }
+  int64_t m = n >> L, set_pos = 0;
+  for (int64_t j = 0; j < m; ++j) cand[j] = (int32_t)j;
+  for (int b = L; b >= 1; --b) {
+    /* Eq. 10-11: the candidates' blocks of 2^b tokens, in candidate order. */
+    const int64_t len = m << b, blk = (int64_t)1 << b;
+    for (int64_t p = 0; p < len; ++p)
+      memcpy(sub + p * d, K + (((int64_t)cand[p >> b] << b) + (p & (blk - 1))) * d, sizeof(double) * d);
+    if (spec32) {
+      for (int64_t i = 0; i < len * d; ++i) sub32[i] = (float)sub[i];
+      orc_wavelet_approx_spec32(sub32, len, d, wavelet, b, store_bf16, a32);
+      for (int64_t i = 0; i < m * d; ++i) rows[i] = (double)a32[i];
+    } else {
+      orc_wavelet_analysis_f64(sub, len, d, wavelet, b, A, D);
+      memcpy(rows, A + orc_pyramid_row_offset(len, b) * d, sizeof(double) * (size_t)m * d);
+    }
+    orc_skim_weights_f64(Q, q, d, rows, m, W);                         /* Eq. 7-8 */
+    topk_ascending(W, cand, m, keep[b], chosen);                       /* Eq. 9 */
+    if (level_sets) { memcpy(level_sets + set_pos, chosen, sizeof(int32_t) * keep[b]); set_pos += keep[b]; }
+    for (int64_t j = 0; j < keep[b]; ++j) { cand[2 * j] = 2 * chosen[j]; cand[2 * j + 1] = 2 * chosen[j] + 1; }
+    m = 2 * (int64_t)keep[b];
+  }
+  /* mu^0: the 2 keep[1] tokens, trimmed to keep[0] on the raw keys. */
+  if (keep[0] < m) {
+    for (int64_t j = 0; j < m; ++j) memcpy(rows + j * d, K + (int64_t)cand[j] * d, sizeof(double) * d);
+    orc_skim_weights_f64(Q, q, d, rows, m, W);
+    topk_ascending(W, cand, m, keep[0], chosen);
+    memcpy(mu0, chosen, sizeof(int32_t) * keep[0]);
+  } else {
+    memcpy(mu0, cand, sizeof(int32_t) * keep[0]);
+  }
+  if (level_sets) memcpy(level_sets + set_pos, mu0, sizeof(int32_t) * keep[0]);
+  free(cand); free(chosen); free(sub); free(A); free(D); free(sub32); free(a32); free(rows); free(W);
+  return 0;
+}

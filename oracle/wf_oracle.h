@@ -91,6 +91,46 @@ int orc_filter_f64(const double* Q, int q, int d, const double* pyr, const doubl
 int orc_filter_literal_f64(const double* Q, int q, int d, const double* K, int64_t n, int L,
                            const int32_t* keep, int32_t* mu0, int32_t* level_sets);
 
+/* Other wavelet bases (Eq. 6 and Eq. 11 with a generic psi), periodized.
+ * An orthogonal two-channel filter bank of `taps` coefficients: low-pass h,
+ * high-pass g.  One analysis level of a periodic signal x of even length len:
+ *   a[j] = sum_k h[k] x[(2j + k) mod len],   det[j] = sum_k g[k] x[(2j + k) mod len]
+ * (periodization keeps the n / 2^B rows of Eq. 6 for every basis).
+ *   ORC_HAAR: h = (1, 1) / sqrt 2, g = (1, -1) / sqrt 2.
+ *   ORC_DB2 (Daubechies, two vanishing moments): h = (1 + r, 3 + r, 3 - r, 1 - r) / (4 sqrt 2),
+ *     r = sqrt 3, and g[k] = (-1)^k h[3 - k].
+ * orc_wavelet_taps fills h and g (4 entries each at most) and returns taps, or -1. */
+#define ORC_HAAR 0
+#define ORC_DB2 1
+int orc_wavelet_taps(int wavelet, double* h, double* g);
+
+/* L periodized analysis levels: A and D in the pyramid layout.  fp64. */
+int orc_wavelet_analysis_f64(const double* x, int64_t n, int d, int wavelet, int L, double* A, double* D);
+/* Inverse of orc_wavelet_analysis_f64 (each level is an orthogonal map; its
+ * inverse is the transpose).  fp64. */
+int orc_wavelet_synthesis_f64(const double* A, const double* D, int64_t n, int d, int wavelet, int L,
+                              double* x);
+
+/* Level-`level` approximation rows (len >> level of them) of the periodized
+ * transform of x under the library's storage rule: an fp32 cascade (Haar:
+ * fl32(x0 + x1) * fl32(1 / sqrt 2), as the stored pyramid; other bases: the
+ * products fl32(fl32(h[k]) * x) added left to right in fp32, no fused
+ * multiply-add), only the last level rounded (bfloat16, nearest even, when
+ * store_bf16; returned widened to float). */
+int orc_wavelet_approx_spec32(const float* x, int64_t len, int d, int wavelet, int level, int store_bf16,
+                              float* out);
+
+/* Algorithm 1 with a generic psi, taken literally: C_L = all level-L blocks;
+ * for b = L..1 the keys of the candidates' blocks, K[mu^b] (2^b tokens per
+ * candidate, in candidate order), are transformed (b periodized levels of the
+ * gathered sequence, Eq. 11; the whole prompt at b = L, Eq. 6) and the
+ * approximation rows scored (Eq. 7-9); C_{b-1} = {2j, 2j+1 : j in J_b}.  Then
+ * the level-0 trim as orc_filter_f64.  spec32 = 0: fp64 transform; 1: the
+ * storage rule of orc_wavelet_approx_spec32 (keys taken as fp32).  Scoring is
+ * fp64.  Outputs as orc_filter_f64 (global block indices per scale). */
+int orc_filter_wavelet_f64(const double* Q, int q, int d, const double* K, int64_t n, int L, int wavelet,
+                           const int32_t* keep, int spec32, int store_bf16, int32_t* mu0, int32_t* level_sets);
+
 /* softmax(Q Ks^T / sqrt(d)) Vs over m key rows (Eq. 1 / Eq. 3 form).  fp64. */
 int orc_attention_f64(const double* Q, int q, int d, const double* Ks, const double* Vs, int64_t m,
                       double* O);
