@@ -42,6 +42,7 @@ from paper_2606_00724_gb300 import synth  # noqa: E402
 
 METRIC = "fused filter+sparse-attn step latency (us) & achieved HBM GB/s vs roofline, 1 GB300"
 DEFAULT_WORKLOAD = "c3"
+WAVELET = None  # None: the Haar pyramid path (wf_step); "haar" / "db2": the literal path (wf_filter_wavelet)
 
 
 def peaks():
@@ -68,13 +69,31 @@ def unit_bytes(w: synth.Workload) -> dict:
     attn = q + 4 * k + 2 * k * row + 2 * w.ng * row + q
     step = q + coeff + trim * row + 2 * k * row + 2 * w.ng * row + q + 4 * k
     dwt = w.n * row + (w.n - (w.n >> L)) * row
+    if WAVELET:
+        step = wavelet_unit_bytes(w)
+        dwt = w.n * row + (w.n >> L) * row  # the scale-L rows of the whole prompt
     return {"filter": filt, "attn": attn, "step": step, "dwt": dwt}
+
+
+def wavelet_unit_bytes(w: synth.Workload) -> int:
+    """Algorithmic bytes of one unit's step on the literal path (Eq. 11 for a
+    generic basis): the cached scale-L rows, the keys of every finer scale's
+    gathered candidate blocks (2 keep[b+1] blocks of 2^b tokens, read once),
+    the level-0 trim rows, the sparse K/V rows, Q, O and the indices."""
+    e = 4 if w.dtype == "f32" else 2
+    row = w.head_dim * e
+    L, keep = w.levels, [int(x) for x in w.keep]
+    gathered = sum(2 * keep[b + 1] << b for b in range(L - 1, 0, -1))
+    trim = 2 * keep[1] if keep[0] < 2 * keep[1] else 0
+    k = keep[0]
+    q = w.q * w.group * row
+    return q + ((w.n >> L) + gathered + trim + 2 * k + 2 * w.ng) * row + q + 4 * k
 
 
 def fused_eligible(w: synth.Workload) -> bool:
     """wf_step runs its single fused kernel for bf16, head_dim 128, <= 32 query
-    rows and one query head per key head."""
-    return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group == 1
+    rows and one query head per key head (the Haar pyramid path)."""
+    return WAVELET is None and w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group == 1
 
 
 def recorded_traffic(w: synth.Workload):
@@ -100,6 +119,8 @@ def launches_per_step(w: synth.Workload) -> int:
     if fused_eligible(w):
         return 1
     trim = int(w.keep[0]) < 2 * int(w.keep[1])
+    if WAVELET:  # one transform kernel per scale below the top
+        return 3 * w.levels + (w.levels - 1) + 3 * trim + 2
     return 3 * w.levels + 3 * trim + 2
 
 
@@ -174,7 +195,11 @@ def oracle_units_seconds(w: synth.Workload, cfg: str, budget_s: float, max_units
         Q, K, V, Kg, Vg = (t.to(dt).double().numpy() for t in (unit.Q, unit.K, unit.V, unit.Kg, unit.Vg))
         pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, w.dtype == "bf16").astype(np.float64)
         t0 = time.perf_counter()
-        if w.group > 1:
+        if WAVELET:
+            basis = oracle.DB2 if WAVELET == "db2" else oracle.HAAR
+            mu0 = oracle.filter_wavelet(Q, K, w.levels, np.array(w.keep), basis, spec32=False)
+            oracle.sparse_attn(Q, K, V, mu0, Kg, Vg)
+        elif w.group > 1:
             Qh = Q.reshape(w.group, w.q, w.head_dim)
             mu0 = oracle.filter_gqa(Qh, pyr, K, w.n, w.levels, np.array(w.keep))
             oracle.sparse_attn_gqa(Qh, K, V, mu0, Kg, Vg)
@@ -253,13 +278,32 @@ def run_gpu(args, cfg, rank, world, device):
     keep = [int(x) for x in w.keep]
     layers = make_inputs(w, cfg, device, rank)
     bufs = []
+    basis = {"haar": wf.WF_WAVELET_HAAR, "db2": wf.WF_WAVELET_DB2}.get(WAVELET)
     for lay in layers:
-        coeffs = torch.empty(wf.wf_coeffs_bytes(lay.K, w.levels), dtype=torch.uint8, device=device)
-        wf.wf_dwt_build(lay.K, w.levels, coeffs)
-        ws = torch.zeros(wf.wf_step_workspace_bytes(lay.Q, lay.K, w.levels, keep, w.ng), dtype=torch.uint8,
-                         device=device)
+        if WAVELET:
+            # The literal path: the scale-L rows of the whole prompt once (like
+            # the pyramid), the finer scales' transforms inside every step.
+            coeffs = torch.empty(w.batch, w.heads, w.n >> w.levels, w.head_dim, dtype=lay.K.dtype, device=device)
+            wf.wf_wavelet_approx(lay.K, w.levels, basis, coeffs)
+            ws = torch.empty(max(wf.wf_filter_wavelet_workspace_bytes(lay.Q, lay.K, w.levels, keep, basis),
+                                 wf.wf_attn_workspace_bytes(lay.Q, w.k, w.ng)), dtype=torch.uint8, device=device)
+        else:
+            coeffs = torch.empty(wf.wf_coeffs_bytes(lay.K, w.levels), dtype=torch.uint8, device=device)
+            wf.wf_dwt_build(lay.K, w.levels, coeffs)
+            ws = torch.zeros(wf.wf_step_workspace_bytes(lay.Q, lay.K, w.levels, keep, w.ng), dtype=torch.uint8,
+                             device=device)
         bufs.append(dict(coeffs=coeffs, ws=ws, idx=torch.empty(w.units, w.k, dtype=torch.int32, device=device),
                          O=torch.empty_like(lay.Q)))
+
+    def one(lay, bf, Q, Kg, Vg, refresh):
+        if WAVELET:
+            if refresh:
+                wf.wf_wavelet_approx(lay.K, w.levels, basis, bf["coeffs"], stream=stream)
+            wf.wf_filter_wavelet(Q, bf["coeffs"], lay.K, w.levels, keep, basis, bf["idx"], bf["ws"], stream=stream)
+            wf.wf_sparse_attn(Q, lay.K, lay.V, bf["idx"], w.k, Kg, Vg, bf["O"], bf["ws"], stream=stream)
+        else:
+            wf.wf_step(Q, lay.K, lay.V, Kg, Vg, bf["coeffs"], refresh, w.levels, keep, bf["idx"], bf["O"], bf["ws"],
+                       stream)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
     stream = torch.cuda.current_stream()
     refresh_every = w.refresh_every
@@ -267,8 +311,7 @@ def run_gpu(args, cfg, rank, world, device):
     def step(i):
         for lay, bf in zip(layers, bufs):
             refresh = bool(refresh_every) and (i % refresh_every == 0)
-            wf.wf_step(lay.Q, lay.K, lay.V, lay.Kg, lay.Vg, bf["coeffs"], refresh, w.levels, keep, bf["idx"],
-                       bf["O"], bf["ws"], stream)
+            one(lay, bf, lay.Q, lay.Kg, lay.Vg, refresh)
 
     for i in range(args.warmup):
         step(i)
@@ -321,8 +364,7 @@ def run_gpu(args, cfg, rank, world, device):
         dQ.copy_(hQ, non_blocking=True)
         dKg.copy_(hKg, non_blocking=True)
         dVg.copy_(hVg, non_blocking=True)
-        wf.wf_step(dQ, lay.K, lay.V, dKg, dVg, bf["coeffs"], False, w.levels, keep, bf["idx"], bf["O"], bf["ws"],
-                   stream)
+        one(lay, bf, dQ, dKg, dVg, False)
         hO.copy_(bf["O"], non_blocking=True)
         hidx.copy_(bf["idx"], non_blocking=True)
         b.record(stream)
@@ -335,6 +377,7 @@ def run_gpu(args, cfg, rank, world, device):
 
 
 def main():
+    global WAVELET
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
@@ -346,6 +389,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=None, help="override the workload's batch (small profiling cases)")
     ap.add_argument("--heads", type=int, default=None, help="override the workload's head count")
+    ap.add_argument("--wavelet", default=None, choices=["haar", "db2"],
+                    help="time the literal path for a generic basis (wf_filter_wavelet + wf_sparse_attn): the "
+                         "transform of the gathered candidate blocks at every scale")
     ap.add_argument("--schedule", default="default", choices=["default", "level0"],
                     help="kept counts: the default schedule, or the token level as its own selection step")
     ap.add_argument("--measure", default="step", choices=["step", "cache-update"],
@@ -366,6 +412,11 @@ def main():
         w = dataclasses.replace(w, batch=args.batch or w.batch, heads=args.heads or w.heads,
                                 name=f"{w.name}_B{args.batch or w.batch}_H{args.heads or w.heads}")
         synth.WORKLOADS[cfg] = w
+    if args.wavelet:
+        import dataclasses
+        WAVELET = args.wavelet
+        w = dataclasses.replace(w, name=f"{w.name}_{args.wavelet}_literal")
+        synth.WORKLOADS[cfg] = w
     if args.schedule == "level0":
         # The token level as its own selection step (one proportion over L+1 scans).
         import dataclasses
@@ -381,9 +432,11 @@ def main():
               "context": w.n, "query_block": w.q, "generation_rows": w.ng, "levels": w.levels, "k": w.k,
               "keep": list(w.keep), "layers": w.layers, "storage": w.dtype,
               "step": ("wf_step (one fused filter + sparse-attention kernel) per layer" if fused_eligible(w) else
+                       f"wf_filter_wavelet ({WAVELET}, periodized; the gathered candidate blocks transformed at every "
+                       "scale) + wf_sparse_attn per layer" if WAVELET else
                        "wf_step (per-stage filter and sparse-attention kernels) per layer") + (
                   f"; wf_dwt_build refresh every {w.refresh_every} steps" if w.refresh_every else
-                  "; pyramid built once before timing"),
+                  ("; scale-L rows built once before timing" if WAVELET else "; pyramid built once before timing")),
               "l2": "flushed before every timed step (256 MiB write)", "parallelism": f"replicas{args.gpus}"}
     step_bytes = ub["step"] * w.units * w.layers
     if w.refresh_every:
@@ -444,7 +497,9 @@ def main():
     achieved = ub["step"] * w.units / (per_layer_ms * 1e-3) / 1e9
     if w.refresh_every:
         achieved = step_bytes / w.layers / (per_layer_ms * 1e-3) / 1e9
-    kname = "wf_fused_kernel" if fused_eligible(w) else "per-stage kernels (score/weights/select/attn)"
+    kname = "wf_fused_kernel" if fused_eligible(w) else (
+        "per-stage kernels (approx/score/weights/select/attn)" if WAVELET else
+        "per-stage kernels (score/weights/select/attn)")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                 "traffic": recorded_traffic(w) if fused_eligible(w) else None, "kernel": kname,
                 "peak_kind": peak_kind,

@@ -176,6 +176,50 @@ wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const
                     size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * 2-3'. Other wavelet bases (Eq. 6 and Eq. 11 with a generic psi).
+ *
+ * With a basis other than Haar the transform of the gathered sub-sequence in
+ * Eq. 11 is no longer the pyramid indexed at the candidates, so these calls
+ * take Algorithm 1 literally: at scale b the keys of the candidates' blocks
+ * (2^b tokens each, in candidate order) form one sequence, taken as
+ * periodic, and b levels of the periodized DWT give one approximation row
+ * per candidate.  Periodization keeps the n / 2^B rows of Eq. 6 for every
+ * basis.  One analysis level is a[j] = sum_k h[k] x[(2j + k) mod len] with
+ *   WF_WAVELET_HAAR: h = (1, 1) / sqrt 2;
+ *   WF_WAVELET_DB2:  Daubechies' filter with two vanishing moments,
+ *                    h = (1 + r, 3 + r, 3 - r, 1 - r) / (4 sqrt 2), r = sqrt 3.
+ * Arithmetic: an fp32 cascade (Haar: fl32(x0 + x1) * fl32(1 / sqrt 2), the
+ * rule of wf_dwt_build; db2: the products fl32(fl32(h[k]) x) added left to
+ * right, no fused multiply-add), the last level rounded to the key dtype.
+ *
+ * wf_wavelet_approx: the level-`level` rows of the keys of blocks
+ * [2^level c, 2^level (c + 1)) for the m candidates c of every unit.
+ * cand: device int32 [B*H][m] block indices at that scale (the sequence
+ * follows their order; entries outside [0, n >> level) are clamped), or NULL
+ * for all m = n >> level blocks in order (the whole prompt, Eq. 6).
+ * out: device [B*H][m][d] in the key dtype, at least B*H*m*d elements.
+ * level: 1..10 for Haar, 1..8 for db2; n a multiple of 2^level.
+ *
+ * wf_filter_wavelet: Eq. 7-11 with the basis `wavelet`.  The scale-L rows are
+ * `top` (wf_wavelet_approx with cand = NULL and level = levels, i.e.
+ * [B*H][n >> levels][d], recomputed whenever K changes); the rows of every
+ * finer scale are the transform of its candidates' gathered blocks.  Scores,
+ * Top-K, children and the level-0 trim, the query grouping rules, limits and
+ * outputs are those of wf_filter; with WF_WAVELET_HAAR the results equal
+ * wf_filter's.  ws: at least wf_filter_wavelet_workspace_bytes() bytes,
+ * 256-byte aligned.
+ * ------------------------------------------------------------------------- */
+#define WF_WAVELET_HAAR 0
+#define WF_WAVELET_DB2 1
+wf_status wf_wavelet_approx(const void* K, const wf_tensor* kv, const int32_t* cand, int m, int level, int wavelet,
+                            void* out, size_t out_bytes, void* stream);
+size_t wf_filter_wavelet_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
+                                         int wavelet);
+wf_status wf_filter_wavelet(const void* Q, const wf_tensor* q, const void* top, const void* K, const wf_tensor* kv,
+                            int levels, const int32_t* keep, int wavelet, int32_t* idx, int32_t* level_sets,
+                            void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
  * 4. Sparse attention (Algorithm 1, final step; Eq. 3 form).
  *
  * For every query head (b, hq), with key head h = hq / G (G = Hq / H, as in

@@ -214,6 +214,43 @@ WF_API wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs
                                        static_cast<cudaStream_t>(stream)));
 }
 
+WF_API wf_status wf_wavelet_approx(const void* K, const wf_tensor* kv, const int32_t* cand, int m, int level,
+                                   int wavelet, void* out, size_t out_bytes, void* stream) {
+  wf_status st;
+  if ((st = check_desc(kv, false)) != WF_OK) return st;
+  if (!wf::wavelet_taps(wavelet) || level < 1 || level > wf::wavelet_max_level(wavelet)) return WF_ERR_UNSUPPORTED;
+  if ((st = check_levels(kv, level)) != WF_OK) return st;
+  if (!K || !out || m < 1 || (!cand && m != (kv->seq >> level))) return WF_ERR_INVALID_ARG;
+  if (!aligned16(K) || !aligned16(out) || (reinterpret_cast<uintptr_t>(cand) & 3u) != 0) return WF_ERR_ALIGN;
+  if (out_bytes < (size_t)kv->batch * kv->heads * m * kv->head_dim * elem_size(kv->dtype)) return WF_ERR_WORKSPACE;
+  return cuda_status(wf::launch_wavelet_approx(K, *kv, cand, m, m, level, wavelet, out, (int64_t)m * kv->head_dim,
+                                               static_cast<cudaStream_t>(stream)));
+}
+
+WF_API size_t wf_filter_wavelet_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels,
+                                                const int32_t* keep, int wavelet) {
+  if (check_filter_args(q, kv, levels, keep) != WF_OK) return 0;
+  if (!wf::wavelet_taps(wavelet) || levels > wf::wavelet_max_level(wavelet)) return 0;
+  return wf::wavelet_filter_bytes(wf::plan_filter(*q, *kv, levels, keep));
+}
+
+WF_API wf_status wf_filter_wavelet(const void* Q, const wf_tensor* q, const void* top, const void* K,
+                                   const wf_tensor* kv, int levels, const int32_t* keep, int wavelet, int32_t* idx,
+                                   int32_t* level_sets, void* ws, size_t ws_bytes, void* stream) {
+  wf_status st = check_filter_args(q, kv, levels, keep);
+  if (st != WF_OK) return st;
+  if (!wf::wavelet_taps(wavelet) || levels > wf::wavelet_max_level(wavelet)) return WF_ERR_UNSUPPORTED;
+  if (!Q || !top || !K || !idx || !ws) return WF_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(top) || !aligned16(K)) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(idx) & 3u) != 0 || (reinterpret_cast<uintptr_t>(level_sets) & 3u) != 0)
+    return WF_ERR_ALIGN;
+  const wf::FilterPlan p = wf::plan_filter(*q, *kv, levels, keep);
+  if (ws_bytes < wf::wavelet_filter_bytes(p)) return WF_ERR_WORKSPACE;
+  return cuda_status(wf::launch_filter_wavelet(p, Q, *q, top, K, *kv, wavelet, idx, level_sets, ws,
+                                               static_cast<cudaStream_t>(stream)));
+}
+
 WF_API size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g) {
   if (check_desc(q, false) != WF_OK || k < 1 || n_g < 0 || q->seq > wf::kMaxQ) return 0;
   return wf::plan_attn(*q, k, n_g, 1).total;  // the size does not depend on the grouping

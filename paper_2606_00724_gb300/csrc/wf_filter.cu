@@ -368,4 +368,81 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
   return cudaSuccess;
 }
 
+size_t wavelet_filter_bytes(const FilterPlan& p) {
+  const size_t esz = p.dtype == WF_BF16 ? 2 : 4;
+  return align_up(p.total, 256) + (size_t)p.U * p.cmax * p.d * esz;
+}
+
+cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* top,
+                                  const void* K, const wf_tensor& kv, int wavelet, int32_t* idx, int32_t* level_sets,
+                                  void* ws, cudaStream_t s) {
+  // The same scan as launch_filter, except that the rows of scale l < L are
+  // the approximation rows of the transform of the candidates' gathered
+  // blocks (computed here, in candidate order) instead of pyramid rows.
+  char* base = static_cast<char*>(ws);
+  int32_t* cand_cur = reinterpret_cast<int32_t*>(base + p.off_cand_a);
+  int32_t* cand_nxt = reinterpret_cast<int32_t*>(base + p.off_cand_b);
+  float* W = reinterpret_cast<float*>(base + p.off_w);
+  float* logits = reinterpret_cast<float*>(base + p.off_logits);
+  float2* part = reinterpret_cast<float2*>(base + p.off_part);
+  void* arows = base + align_up(p.total, 256);
+  int64_t sets_stride = 0;
+  for (int l = 0; l <= p.L; ++l) sets_stride += p.keep[l];
+  int64_t sets_off = 0;
+  int m = p.n >> p.L;
+  cudaError_t e;
+  for (int l = p.L; l >= 1; --l) {
+    RowSrc src;
+    src.off = 0;
+    src.ss = p.d;
+    if (l == p.L) {
+      src.base = top;  // the whole prompt's level-L rows (Eq. 6), [units][m][d]
+      src.sh = (int64_t)m * p.d;
+    } else {
+      if ((e = launch_wavelet_approx(K, kv, cand_cur, p.cmax, m, l, wavelet, arows, (int64_t)p.cmax * p.d, s)) !=
+          cudaSuccess)
+        return e;
+      src.base = arows;
+      src.sh = (int64_t)p.cmax * p.d;
+    }
+    src.sb = src.sh * p.H;
+    if ((e = score(p, Q, qd, src, nullptr, m, logits, part, s)) != cudaSuccess) return e;
+    const int ntiles = (m + TILE - 1) / TILE;
+    weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
+                                                              (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const bool last = (l == 1) && !p.trim;
+    int32_t* out = last ? idx : cand_nxt;
+    const int64_t out_stride = last ? p.keep[0] : p.cmax;
+    const int32_t* cand = l == p.L ? nullptr : cand_cur;  // position -> block index at scale l
+    select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand, p.cmax, m, p.keep[l], 1, out, out_stride, level_sets,
+                                       sets_stride, sets_off);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    sets_off += p.keep[l];
+    m = 2 * p.keep[l];
+    int32_t* t = cand_cur; cand_cur = cand_nxt; cand_nxt = t;
+  }
+  if (p.trim) {
+    RowSrc src;
+    src.base = K;
+    src.sb = kv.stride_b;
+    src.sh = kv.stride_h;
+    src.ss = kv.stride_s;
+    src.off = 0;
+    if ((e = score(p, Q, qd, src, cand_cur, m, logits, part, s)) != cudaSuccess) return e;
+    const int ntiles = (m + TILE - 1) / TILE;
+    weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
+                                                              (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  if (level_sets) {
+    e = cudaMemcpy2DAsync(level_sets + sets_off, sizeof(int32_t) * sets_stride, idx, sizeof(int32_t) * p.keep[0],
+                          sizeof(int32_t) * p.keep[0], p.U, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 }  // namespace wf

@@ -86,6 +86,21 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
                           const void* K, const wf_tensor& kv, int32_t* idx, int32_t* level_sets, void* ws,
                           cudaStream_t s);
 
+// Approximation rows at scale `level` of the periodized transform (wavelet
+// WF_WAVELET_*) of the keys of blocks [2^level c, 2^level (c + 1)) for the m
+// candidates c of every unit (cand: [units][cand_stride], NULL = all blocks),
+// into out[unit * out_unit + j * head_dim + channel] in the key dtype.
+cudaError_t launch_wavelet_approx(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m,
+                                  int level, int wavelet, void* out, int64_t out_unit, cudaStream_t s);
+int wavelet_taps(int wavelet);       // 0 for an unknown basis
+int wavelet_max_level(int wavelet);  // deepest scale the approximation kernel supports
+// Filtering with a generic basis (Eq. 11 taken literally): the filter plan's
+// workspace followed by one block of approximation rows [units][cmax][d].
+size_t wavelet_filter_bytes(const FilterPlan& p);
+cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* top,
+                                  const void* K, const wf_tensor& kv, int wavelet, int32_t* idx, int32_t* level_sets,
+                                  void* ws, cudaStream_t s);
+
 // Sparse attention workspace plan.  A unit is one (batch, query head); it
 // reads KV head h / G and that head's index row.
 struct AttnPlan {

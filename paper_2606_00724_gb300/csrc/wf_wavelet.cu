@@ -1,0 +1,145 @@
+// Approximation rows of the periodized DWT of a gathered key sub-sequence
+// (Eq. 6 for the whole prompt, Eq. 11 for the blocks of the candidates kept
+// one scale up), for the Haar and db2 filter banks.
+//
+// The sequence of a unit is the keys of blocks [2^b c, 2^b (c + 1)) for the
+// unit's candidates c, in candidate order, taken as periodic.  One level of
+// analysis is a[j] = sum_k h[k] x[(2j + k) mod len]; b levels give one
+// approximation row per candidate.
+//
+// One CTA computes TO consecutive level-b rows for DS head-dim channels: it
+// gathers the TO 2^b input rows plus the (taps - 2)(2^b - 1) rows the filter
+// reaches past them (wrapping around the gathered sequence), widened to fp32
+// in shared memory, and runs the b levels of the cascade there (two buffers
+// alternating).  Arithmetic (the storage rule, shared with the Haar pyramid):
+// Haar: fl32(x0 + x1) * fl32(1 / sqrt 2); db2: the products
+// fl32(fl32(h[k]) * x) added left to right in fp32, no fused multiply-add.
+// Only the last level is rounded to the key dtype.
+#include <math.h>
+
+#include "wf_internal.cuh"
+
+namespace wf {
+namespace {
+
+constexpr int DS = 16;        // head-dim channels per CTA
+constexpr int NTH = 128;      // threads per CTA
+constexpr int IN_ROWS = 512;  // gathered rows per CTA before the filter's reach
+
+// Output rows per CTA at scale `level`.
+__host__ __device__ inline int outputs_per_cta(int level) { return (IN_ROWS >> level) > 0 ? (IN_ROWS >> level) : 1; }
+
+// Rows needed l levels below the output so that the output level yields `to`
+// rows: to 2^l + (taps - 2)(2^l - 1).
+__host__ __device__ inline int rows_needed(int to, int l, int taps) { return (to << l) + (taps - 2) * ((1 << l) - 1); }
+
+struct Taps {
+  float h[4];
+};
+
+template <typename T, int TAPS>
+__global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, int64_t ksb, int64_t ksh, int64_t kss,
+                                                     int64_t n, int H, const int32_t* __restrict__ cand,
+                                                     int64_t cand_stride, int m, int level, Taps taps, T* __restrict__ out,
+                                                     int64_t out_unit, int64_t out_row) {
+  extern __shared__ __align__(16) float buf[];
+  const int to = outputs_per_cta(level);
+  const int nin = rows_needed(to, level, TAPS);
+  float* X = buf;                     // [nin][DS]
+  float* Y = buf + (size_t)nin * DS;  // [nin / 2 + 1][DS]
+  const int u = blockIdx.y;
+  const int j0 = blockIdx.x * to;
+  const int c0 = blockIdx.z * DS;
+  const int64_t bb = u / H, hh = u % H;
+  const int64_t len = (int64_t)m << level;
+  const int64_t blk_mask = ((int64_t)1 << level) - 1;
+  const T* kb = K + bb * ksb + hh * ksh + c0;
+  const int32_t* cd = cand ? cand + (int64_t)u * cand_stride : nullptr;
+  const int tid = threadIdx.x;
+
+  // Gather: row r is gathered position (j0 2^b + r) mod len.
+  constexpr int VEC = Vec<T>::N;
+  constexpr int VPR = DS / VEC;  // 16-byte vectors per row
+  for (int e = tid; e < nin * VPR; e += NTH) {
+    const int r = e / VPR, v = e % VPR;
+    const int64_t p = (((int64_t)j0 << level) + r) % len;
+    int64_t tok = cd ? (((int64_t)cd[p >> level]) << level) + (p & blk_mask) : p;
+    tok = tok < 0 ? 0 : (tok >= n ? n - 1 : tok);  // out-of-range block indices are clamped
+    float x[VEC];
+    ld_vec(kb + tok * kss + v * VEC, x);
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) X[r * DS + v * VEC + i] = x[i];
+  }
+  __syncthreads();
+
+  const float c32 = 0.70710678118654752440f;  // fl32(1 / sqrt 2)
+  float* src = X;
+  float* dst = Y;
+#pragma unroll 1
+  for (int l = 1; l <= level; ++l) {
+    const int nout = rows_needed(to, level - l, TAPS);
+    for (int e = tid; e < nout * DS; e += NTH) {
+      const int j = e / DS, c = e % DS;
+      const float* x = src + (2 * j) * DS + c;
+      float v;
+      if (TAPS == 2) {
+        v = __fmul_rn(__fadd_rn(x[0], x[DS]), c32);
+      } else {
+        v = __fmul_rn(taps.h[0], x[0]);
+#pragma unroll
+        for (int k = 1; k < TAPS; ++k) v = __fadd_rn(v, __fmul_rn(taps.h[k], x[k * DS]));
+      }
+      dst[j * DS + c] = v;
+    }
+    __syncthreads();
+    float* t = src;
+    src = dst;
+    dst = t;
+  }
+
+  // The last level: rows j0 .. j0 + to - 1 (those below m), rounded to T.
+  T* ob = out + (int64_t)u * out_unit + c0;
+  for (int e = tid; e < to * DS; e += NTH) {
+    const int j = e / DS, c = e % DS;
+    if (j0 + j < m) from_f32(ob[(int64_t)(j0 + j) * out_row + c], src[j * DS + c]);
+  }
+}
+
+template <typename T, int TAPS>
+cudaError_t run(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m, int level,
+                const Taps& taps, void* out, int64_t out_unit, cudaStream_t s) {
+  const int to = outputs_per_cta(level);
+  const int nin = rows_needed(to, level, TAPS);
+  const size_t smem = sizeof(float) * DS * (size_t)(nin + nin / 2 + 1);
+  cudaError_t e = cudaFuncSetAttribute(approx_kernel<T, TAPS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads), (unsigned)(kv.head_dim / DS));
+  approx_kernel<T, TAPS><<<grid, NTH, smem, s>>>(static_cast<const T*>(K), kv.stride_b, kv.stride_h, kv.stride_s,
+                                                 kv.seq, kv.heads, cand, cand_stride, m, level, taps,
+                                                 static_cast<T*>(out),
+                                                 out_unit, kv.head_dim);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int wavelet_taps(int wavelet) { return wavelet == WF_WAVELET_HAAR ? 2 : (wavelet == WF_WAVELET_DB2 ? 4 : 0); }
+
+int wavelet_max_level(int wavelet) { return wavelet == WF_WAVELET_DB2 ? 8 : 10; }
+
+cudaError_t launch_wavelet_approx(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m,
+                                  int level, int wavelet, void* out, int64_t out_unit, cudaStream_t s) {
+  Taps taps{};
+  if (wavelet == WF_WAVELET_DB2) {
+    // Daubechies' two-vanishing-moment scaling filter, from its closed form.
+    const double r = sqrt(3.0), q = 4.0 * sqrt(2.0);
+    const double h[4] = {(1.0 + r) / q, (3.0 + r) / q, (3.0 - r) / q, (1.0 - r) / q};
+    for (int k = 0; k < 4; ++k) taps.h[k] = (float)h[k];
+    return kv.dtype == WF_BF16 ? run<bf16, 4>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s)
+                               : run<float, 4>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+  }
+  return kv.dtype == WF_BF16 ? run<bf16, 2>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s)
+                             : run<float, 2>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+}
+
+}  // namespace wf

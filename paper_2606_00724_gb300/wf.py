@@ -50,6 +50,9 @@ SIGNATURES = {
     "wf_schedule_from_proportions": (_I, [_I64, _I, _P, _P]),
     "wf_filter_workspace_bytes": (_SZ, [_T, _T, _I, _P]),
     "wf_filter": (_I, [_P, _T, _P, _P, _T, _I, _P, _P, _P, _P, _SZ, _P]),
+    "wf_wavelet_approx": (_I, [_P, _T, _P, _I, _I, _I, _P, _SZ, _P]),
+    "wf_filter_wavelet_workspace_bytes": (_SZ, [_T, _T, _I, _P, _I]),
+    "wf_filter_wavelet": (_I, [_P, _T, _P, _P, _T, _I, _P, _I, _P, _P, _P, _SZ, _P]),
     "wf_attn_workspace_bytes": (_SZ, [_T, _I, _I]),
     "wf_sparse_attn": (_I, [_P, _T, _P, _P, _T, _P, _I, _P, _P, _T, _P, _T, ctypes.c_float, _P, _SZ, _P]),
     "wf_step_workspace_bytes": (_SZ, [_T, _T, _I, _P, _I]),
@@ -161,6 +164,34 @@ def wf_filter(Q: torch.Tensor, coeffs: torch.Tensor, K: torch.Tensor, levels: in
     _check(lib().wf_filter(_ptr(Q), ctypes.byref(dq), _ptr(coeffs), _ptr(K), ctypes.byref(dk), levels,
                            _keep_arr(keep), _ptr(idx), _ptr(level_sets), _ptr(ws), ws.numel() * ws.element_size(),
                            _stream(stream)), "wf_filter")
+
+
+WF_WAVELET_HAAR, WF_WAVELET_DB2 = 0, 1
+
+
+def wf_wavelet_approx(K: torch.Tensor, level: int, wavelet: int, out: torch.Tensor, cand=None, m=None,
+                      stream=None):
+    """Level-`level` approximation rows of the gathered blocks of `cand`
+    ([B*H][m] int32, or None for the whole prompt) into out ([B, H, m, d])."""
+    dk = desc(K)
+    if m is None:
+        m = cand.shape[1] if cand is not None else K.shape[2] >> level
+    _check(lib().wf_wavelet_approx(_ptr(K), ctypes.byref(dk), _ptr(cand), int(m), level, wavelet, _ptr(out),
+                                   out.numel() * out.element_size(), _stream(stream)), "wf_wavelet_approx")
+
+
+def wf_filter_wavelet_workspace_bytes(Q: torch.Tensor, K: torch.Tensor, levels: int, keep, wavelet: int) -> int:
+    dq, dk = desc(Q), desc(K)
+    return int(lib().wf_filter_wavelet_workspace_bytes(ctypes.byref(dq), ctypes.byref(dk), levels, _keep_arr(keep),
+                                                       wavelet))
+
+
+def wf_filter_wavelet(Q: torch.Tensor, top: torch.Tensor, K: torch.Tensor, levels: int, keep, wavelet: int,
+                      idx: torch.Tensor, ws: torch.Tensor, level_sets: torch.Tensor | None = None, stream=None):
+    dq, dk = desc(Q), desc(K)
+    _check(lib().wf_filter_wavelet(_ptr(Q), ctypes.byref(dq), _ptr(top), _ptr(K), ctypes.byref(dk), levels,
+                                   _keep_arr(keep), wavelet, _ptr(idx), _ptr(level_sets), _ptr(ws),
+                                   ws.numel() * ws.element_size(), _stream(stream)), "wf_filter_wavelet")
 
 
 def wf_attn_workspace_bytes(Q: torch.Tensor, k: int, n_g: int) -> int:

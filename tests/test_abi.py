@@ -198,3 +198,22 @@ def test_attn_rejects(lib):
     assert call(Kg=None) == -1                                    # n_g > 0 needs Kg
     assert call(o=_desc(1, 2, 31, 128)) == -2
     assert call(scale=-1.0) == -1
+
+
+@no_gpu
+def test_wavelet_rejects(lib):
+    kv = _desc(1, 2, 64, 128)
+    need = 1 * 2 * 16 * 128 * 2
+    call = lambda K=FAKE, cand=None, m=16, level=2, wv=1, out=FAKE2, nb=need: lib.wf_wavelet_approx(
+        K, ctypes.byref(kv), cand, m, level, wv, out, nb, None)
+    assert call(wv=7) == -8                        # unknown basis
+    assert call(level=9) == -8                     # db2 deeper than 8 levels
+    assert call(m=15) == -1                        # whole prompt: m must be n >> level
+    assert call(nb=need - 1) == -5
+    assert call(K=ctypes.c_void_p(0x10008)) == -4
+    assert call(cand=ctypes.c_void_p(0x30002), m=3) == -4
+    q = _desc(1, 2, 32, 128)
+    keep = (ctypes.c_int32 * 3)(16, 8, 8)
+    assert lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1) > \
+        lib.wf_filter_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep)
+    assert lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 5) == 0
