@@ -17,7 +17,7 @@ namespace {
 constexpr int CH = kAttnChunk;
 constexpr int QMAX = kMaxQ;
 
-template <typename T, int D>
+template <typename T, int D, int QM>
 __global__ void __launch_bounds__(256) attn_split_kernel(
     const T* __restrict__ Q, int64_t qsb, int64_t qsh, int64_t qss, const T* __restrict__ K,
     const T* __restrict__ V, int64_t ksb, int64_t ksh, int64_t kss, int n, const int32_t* __restrict__ idx, int k,
@@ -26,10 +26,10 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
   constexpr int VEC = Vec<T>::N;
   constexpr int KS = D + 4;
   extern __shared__ __align__(16) float smem[];
-  float* Qs = smem;                // [QMAX][D]
-  float* Ks = Qs + QMAX * D;       // [CH][KS]
+  float* Qs = smem;                // [QM][D]
+  float* Ks = Qs + QM * D;         // [CH][KS]
   float* Vs = Ks + CH * KS;        // [CH][D]
-  float* P = Vs + CH * D;          // [QMAX][CH + 1]
+  float* P = Vs + CH * D;          // [QM][CH + 1]
   const int u = blockIdx.y;
   const int sp = blockIdx.x;
   const int t0 = sp * CH;
@@ -40,7 +40,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
   const int tid = threadIdx.x;
 
   const T* qbase = Q + bb * qsb + hh * qsh;
-  for (int e = tid; e < QMAX * (D / VEC); e += blockDim.x) {
+  for (int e = tid; e < QM * (D / VEC); e += blockDim.x) {
     const int i = e / (D / VEC), c = (e % (D / VEC)) * VEC;
     float v[VEC];
     if (i < q) ld_vec(qbase + (int64_t)i * qss + c, v);
@@ -79,23 +79,23 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
 
   // Logits: lane -> keys (lane, lane+32), warp -> query rows warp + 8r.
   const int lane = tid & 31, warp = tid >> 5;
-  float acc0[QMAX / 8], acc1[QMAX / 8];
+  float acc0[QM / 8], acc1[QM / 8];
 #pragma unroll
-  for (int r = 0; r < QMAX / 8; ++r) { acc0[r] = 0.f; acc1[r] = 0.f; }
+  for (int r = 0; r < QM / 8; ++r) { acc0[r] = 0.f; acc1[r] = 0.f; }
 #pragma unroll 2
   for (int c = 0; c < D; c += 4) {
     const float4 k0 = *reinterpret_cast<const float4*>(&Ks[lane * KS + c]);
     const float4 k1 = *reinterpret_cast<const float4*>(&Ks[(lane + 32) * KS + c]);
 #pragma unroll
-    for (int r = 0; r < QMAX / 8; ++r) {
+    for (int r = 0; r < QM / 8; ++r) {
       const float4 qv = *reinterpret_cast<const float4*>(&Qs[(warp + 8 * r) * D + c]);
       acc0[r] = fmaf(qv.x, k0.x, fmaf(qv.y, k0.y, fmaf(qv.z, k0.z, fmaf(qv.w, k0.w, acc0[r]))));
       acc1[r] = fmaf(qv.x, k1.x, fmaf(qv.y, k1.y, fmaf(qv.z, k1.z, fmaf(qv.w, k1.w, acc1[r]))));
     }
   }
-  float2* ml = ML + ((int64_t)u * nsplit + sp) * QMAX;
+  float2* ml = ML + ((int64_t)u * nsplit + sp) * QMAX;  // partials keep the workspace's QMAX-row stride
 #pragma unroll
-  for (int r = 0; r < QMAX / 8; ++r) {
+  for (int r = 0; r < QM / 8; ++r) {
     const int i = warp + 8 * r;
     if (i >= q) break;
     const float s0 = lane < cnt ? acc0[r] * scale : -INFINITY;
@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
 
   // Partial output: thread -> channel c, query rows [qg*QPT, (qg+1)*QPT).
   constexpr int GROUPS = 256 / D;
-  constexpr int QPT = QMAX / GROUPS;
+  constexpr int QPT = QM / GROUPS;
   const int c = tid % D, qg = tid / D;
   float o[QPT];
 #pragma unroll
@@ -134,46 +134,63 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
   }
 }
 
+// One CTA per unit: the weight exp(m_s - M) of every split s and query row
+// (and the denominator) is formed once in shared memory, then every output
+// element is one pass over the splits' partial outputs.
 template <typename T>
 __global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restrict__ Opart,
                                                            const float2* __restrict__ ML, int nsplit, int q, int D,
-                                                           int H, T* __restrict__ O, int64_t osb, int64_t osh,
-                                                           int64_t oss) {
+                                                           int H, int qstride, T* __restrict__ O, int64_t osb,
+                                                           int64_t osh, int64_t oss) {
+  extern __shared__ float fw[];  // [nsplit][q] weights, then the [q] denominators
+  float* den_s = fw + nsplit * q;
   const int u = blockIdx.x;
   const int64_t bb = u / H, hh = u % H;
+  const float2* ml = ML + (int64_t)u * nsplit * qstride;
+  for (int i = threadIdx.x; i < q; i += blockDim.x) {
+    float mx = -INFINITY;
+    for (int s = 0; s < nsplit; ++s) mx = fmaxf(mx, ml[(int64_t)s * qstride + i].x);
+    float den = 0.f;
+    for (int s = 0; s < nsplit; ++s) {
+      const float2 p = ml[(int64_t)s * qstride + i];
+      const float f = expf(p.x - mx);
+      fw[s * q + i] = f;
+      den = fmaf(p.y, f, den);
+    }
+    den_s[i] = den;
+  }
+  __syncthreads();
+  const float* op = Opart + (int64_t)u * nsplit * qstride * D;
   for (int e = threadIdx.x; e < q * D; e += blockDim.x) {
     const int i = e / D, c = e % D;
-    float mx = -INFINITY;
-    for (int s = 0; s < nsplit; ++s) mx = fmaxf(mx, ML[((int64_t)u * nsplit + s) * QMAX + i].x);
-    float num = 0.f, den = 0.f;
-    for (int s = 0; s < nsplit; ++s) {
-      const float2 p = ML[((int64_t)u * nsplit + s) * QMAX + i];
-      const float f = expf(p.x - mx);
-      den = fmaf(p.y, f, den);
-      num = fmaf(Opart[((int64_t)u * nsplit + s) * QMAX * D + (int64_t)i * D + c], f, num);
-    }
-    from_f32(O[bb * osb + hh * osh + (int64_t)i * oss + c], num / den);
+    float num = 0.f;
+    for (int s = 0; s < nsplit; ++s) num = fmaf(op[((int64_t)s * qstride + i) * D + c], fw[s * q + i], num);
+    from_f32(O[bb * osb + hh * osh + (int64_t)i * oss + c], num / den_s[i]);
   }
 }
 
-template <typename T, int D>
+template <typename T, int D, int QM>
 cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                 const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg, const wf_tensor* g,
                 void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s) {
   float* Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
   float2* ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
-  const size_t smem = sizeof(float) * (size_t)(QMAX * D + CH * (D + 4) + CH * D + QMAX * (CH + 1));
-  cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const size_t smem = sizeof(float) * (size_t)(QM * D + CH * (D + 4) + CH * D + QM * (CH + 1));
+  cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<T, D, QM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t gsb = g ? g->stride_b : 0, gsh = g ? g->stride_h : 0, gss = g ? g->stride_s : 0;
-  attn_split_kernel<T, D><<<dim3(p.nsplit, p.U), 256, smem, s>>>(
+  attn_split_kernel<T, D, QM><<<dim3(p.nsplit, p.U), 256, smem, s>>>(
       static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, static_cast<const T*>(K),
       static_cast<const T*>(V), kv.stride_b, kv.stride_h, kv.stride_s, kv.seq, idx, p.k, static_cast<const T*>(Kg),
       static_cast<const T*>(Vg), gsb, gsh, gss, p.ng, p.q, p.H, p.G, scale, p.nsplit, Opart, ML);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  attn_combine_kernel<T><<<p.U, 256, 0, s>>>(Opart, ML, p.nsplit, p.q, D, p.H, static_cast<T*>(O), od.stride_b,
-                                             od.stride_h, od.stride_s);
+  const size_t csmem = sizeof(float) * (size_t)(p.nsplit + 1) * p.q;
+  if ((e = cudaFuncSetAttribute(attn_combine_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem)) !=
+      cudaSuccess)
+    return e;
+  attn_combine_kernel<T><<<p.U, 256, csmem, s>>>(Opart, ML, p.nsplit, p.q, D, p.H, QMAX, static_cast<T*>(O),
+                                                 od.stride_b, od.stride_h, od.stride_s);
   return cudaGetLastError();
 }
 
@@ -200,12 +217,13 @@ AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group) {
 cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                         const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
                         const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s) {
-  if (p.dtype == WF_BF16) {
-    return p.d == 64 ? run<bf16, 64>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s)
-                     : run<bf16, 128>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s);
-  }
-  return p.d == 64 ? run<float, 64>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s)
-                   : run<float, 128>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s);
+  // Query blocks of up to 32 rows take the 32-row tile.
+#define WF_ATTN_RUN(T, DD)                                                                  \
+  (p.q <= 32 ? run<T, DD, 32>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s)     \
+             : run<T, DD, QMAX>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s))
+  if (p.dtype == WF_BF16) return p.d == 64 ? WF_ATTN_RUN(bf16, 64) : WF_ATTN_RUN(bf16, 128);
+  return p.d == 64 ? WF_ATTN_RUN(float, 64) : WF_ATTN_RUN(float, 128);
+#undef WF_ATTN_RUN
 }
 
 }  // namespace wf

@@ -29,8 +29,8 @@ __device__ __forceinline__ const T* query_row(const T* Q, int64_t qsb, int64_t q
   return Q + bb * qsb + (hh * G + i / qs) * qsh + (int64_t)(i % qs) * qss;
 }
 
-// Grid (candidate tiles, units, query chunks of QMAX rows).
-template <typename T, int D>
+// Grid (candidate tiles, units, query chunks of QM rows).
+template <typename T, int D, int QM>
 __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int64_t qsb, int64_t qsh, int64_t qss,
                                                     int q, int G, int qs, int H, RowSrc src,
                                                     const int32_t* __restrict__ cand,
@@ -40,15 +40,15 @@ __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int
   constexpr int VEC = Vec<T>::N;
   constexpr int RS = D + 4;  // padded row stride of the candidate tile (keeps 16-byte alignment)
   extern __shared__ __align__(16) float smem[];
-  float* Qs = smem;              // [QMAX][D]
-  float* Rs = smem + QMAX * D;   // [TILE][RS]
+  float* Qs = smem;              // [QM][D]
+  float* Rs = smem + QM * D;     // [TILE][RS]
   const int u = blockIdx.y;
   const int j0 = blockIdx.x * TILE;
-  const int i0 = blockIdx.z * QMAX;  // first query row of this chunk
+  const int i0 = blockIdx.z * QM;  // first query row of this chunk
   const int64_t bb = u / H, hh = u % H;
   const int tid = threadIdx.x;
 
-  for (int e = tid; e < QMAX * (D / VEC); e += blockDim.x) {
+  for (int e = tid; e < QM * (D / VEC); e += blockDim.x) {
     const int i = e / (D / VEC), c = (e % (D / VEC)) * VEC;
     float v[VEC];
     if (i0 + i < q) ld_vec(query_row(Q, qsb, qsh, qss, bb, hh, G, qs, i0 + i) + c, v);
@@ -76,14 +76,14 @@ __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int
   __syncthreads();
 
   const int lane = tid & 31, warp = tid >> 5;  // lane = candidate, warp = query phase
-  float acc[QMAX / 8];
+  float acc[QM / 8];
 #pragma unroll
-  for (int r = 0; r < QMAX / 8; ++r) acc[r] = 0.f;
+  for (int r = 0; r < QM / 8; ++r) acc[r] = 0.f;
 #pragma unroll 4
   for (int c = 0; c < D; c += 4) {
     const float4 rv = *reinterpret_cast<const float4*>(&Rs[lane * RS + c]);
 #pragma unroll
-    for (int r = 0; r < QMAX / 8; ++r) {
+    for (int r = 0; r < QM / 8; ++r) {
       const float4 qv = *reinterpret_cast<const float4*>(&Qs[(warp + 8 * r) * D + c]);
       acc[r] = fmaf(qv.x, rv.x, acc[r]);
       acc[r] = fmaf(qv.y, rv.y, acc[r]);
@@ -96,7 +96,7 @@ __global__ void __launch_bounds__(256) score_kernel(const T* __restrict__ Q, int
   float* lg = logits + (int64_t)u * lg_unit;
   float2* pt = part + (int64_t)u * part_unit + (int64_t)blockIdx.x * q;
 #pragma unroll
-  for (int r = 0; r < QMAX / 8; ++r) {
+  for (int r = 0; r < QM / 8; ++r) {
     const int i = i0 + warp + 8 * r;
     if (i >= q) break;
     const float s = acc[r] * scale;
@@ -249,17 +249,25 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   }
 }
 
-template <typename T, int D>
-cudaError_t run_score(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
-                      int m, float* logits, float2* part, cudaStream_t s) {
-  const size_t smem = sizeof(float) * (size_t)(QMAX * D + TILE * (D + 4));
-  cudaError_t e = cudaFuncSetAttribute(score_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+template <typename T, int D, int QM>
+cudaError_t run_score_q(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
+                        int m, float* logits, float2* part, cudaStream_t s) {
+  const size_t smem = sizeof(float) * (size_t)(QM * D + TILE * (D + 4));
+  cudaError_t e = cudaFuncSetAttribute(score_kernel<T, D, QM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((m + TILE - 1) / TILE, p.U, (p.q + QMAX - 1) / QMAX);
-  score_kernel<T, D><<<grid, 256, smem, s>>>(static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, p.q,
+  dim3 grid((m + TILE - 1) / TILE, p.U, (p.q + QM - 1) / QM);
+  score_kernel<T, D, QM><<<grid, 256, smem, s>>>(static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, p.q,
                                              p.G, p.qs, p.H, src, cand, p.cmax, m, 1.0f / sqrtf((float)D), logits,
                                              (int64_t)p.q * p.cmax, p.cmax, part, (int64_t)p.tiles_max * p.q);
   return cudaGetLastError();
+}
+
+// Query blocks of up to 32 rows take the 32-row tile; larger ones 64-row chunks.
+template <typename T, int D>
+cudaError_t run_score(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
+                      int m, float* logits, float2* part, cudaStream_t s) {
+  return p.q <= 32 ? run_score_q<T, D, 32>(p, Q, qd, src, cand, m, logits, part, s)
+                   : run_score_q<T, D, QMAX>(p, Q, qd, src, cand, m, logits, part, s);
 }
 
 cudaError_t score(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand, int m,
