@@ -168,7 +168,11 @@ wf_status wf_level0_schedule(int64_t n, int levels, int64_t k, int32_t* keep);
  * level_sets (optional, NULL to skip): int32
  * [B*H][keep[L] + .. + keep[1] + keep[0]] = J_L, .., J_1, mu^0 per unit.
  * ws: device scratch of at least wf_filter_workspace_bytes() bytes,
- * 256-byte aligned; its contents on entry do not matter.
+ * 256-byte aligned.  Its first 4 bytes are a status word: for bf16 keys with
+ * head_dim 128 the scores run on the tensor cores, and a kernel whose bounded
+ * wait gives up (it never should) sets the word and leaves the outputs
+ * undefined; wf_workspace_status() reads and clears it.  Zero the word once
+ * before the first call; the rest of ws may hold anything.
  * ------------------------------------------------------------------------- */
 size_t wf_filter_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep);
 wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const void* K, const wf_tensor* kv,
@@ -207,7 +211,7 @@ wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const
  * Top-K, children and the level-0 trim, the query grouping rules, limits and
  * outputs are those of wf_filter; with WF_WAVELET_HAAR the results equal
  * wf_filter's.  ws: at least wf_filter_wavelet_workspace_bytes() bytes,
- * 256-byte aligned.
+ * 256-byte aligned, with wf_filter's status word in its first 4 bytes.
  * ------------------------------------------------------------------------- */
 #define WF_WAVELET_HAAR 0
 #define WF_WAVELET_DB2 1
@@ -231,7 +235,10 @@ wf_status wf_filter_wavelet(const void* Q, const wf_tensor* q, const void* top, 
  * idx: int32 [B*H][k], each entry in [0, n) (any order).
  * Kg, Vg: [B,H,n_g,d] (descriptor g, may be NULL when n_g = 0).  O: [B,Hq,q,d]
  * (descriptor o: same shape and dtype as Q), written rounded to that dtype.
- * ws: device scratch of at least wf_attn_workspace_bytes() bytes.
+ * ws: device scratch of at least wf_attn_workspace_bytes() bytes, 256-byte
+ * aligned; as for wf_filter, its first 4 bytes are a status word set if a
+ * tensor-core kernel's bounded wait gives up (bf16 keys with head_dim 128 run
+ * on the tensor cores): zero it once, read it with wf_workspace_status().
  * Out-of-range idx entries are clamped to [0, n) (never read out of bounds).
  * ------------------------------------------------------------------------- */
 size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g);

@@ -210,7 +210,7 @@ WF_API wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs
     return WF_ERR_ALIGN;
   const wf::FilterPlan p = wf::plan_filter(*q, *kv, levels, keep);
   if (ws_bytes < p.total) return WF_ERR_WORKSPACE;
-  return cuda_status(wf::launch_filter(p, Q, *q, coeffs, K, *kv, idx, level_sets, ws,
+  return cuda_status(wf::launch_filter(p, Q, *q, coeffs, K, *kv, idx, level_sets, ws, static_cast<int*>(ws),
                                        static_cast<cudaStream_t>(stream)));
 }
 
@@ -248,7 +248,7 @@ WF_API wf_status wf_filter_wavelet(const void* Q, const wf_tensor* q, const void
   const wf::FilterPlan p = wf::plan_filter(*q, *kv, levels, keep);
   if (ws_bytes < wf::wavelet_filter_bytes(p)) return WF_ERR_WORKSPACE;
   return cuda_status(wf::launch_filter_wavelet(p, Q, *q, top, K, *kv, wavelet, idx, level_sets, ws,
-                                               static_cast<cudaStream_t>(stream)));
+                                               static_cast<int*>(ws), static_cast<cudaStream_t>(stream)));
 }
 
 WF_API size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g) {
@@ -274,7 +274,7 @@ WF_API wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K
   if (ws_bytes < p.total) return WF_ERR_WORKSPACE;
   const float sc = scale == 0.f ? 1.0f / sqrtf((float)q->head_dim) : scale;
   return cuda_status(wf::launch_attn(p, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, ws,
-                                     static_cast<cudaStream_t>(stream)));
+                                     static_cast<int*>(ws), static_cast<cudaStream_t>(stream)));
 }
 
 // wf_step keeps a 256-byte status block at the start of its workspace (the
@@ -324,11 +324,11 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
     return cuda_status(e);
   }
   const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
-  if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, s)) != cudaSuccess)
+  if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, status, s)) != cudaSuccess)
     return WF_ERR_CUDA;
   const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g, group_of(q, kv));
   const float sc = 1.0f / sqrtf((float)q->head_dim);
-  e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, s);
+  e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, status, s);
   return cuda_status(e);
 }
 

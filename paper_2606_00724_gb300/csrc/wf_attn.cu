@@ -169,6 +169,19 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restri
   }
 }
 
+// The combine of nsplit partials per query-head unit into O.
+template <typename T>
+cudaError_t combine(const AttnPlan& p, int nsplit, void* O, const wf_tensor& od, void* ws, cudaStream_t s) {
+  float* Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
+  float2* ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
+  const size_t csmem = sizeof(float) * (size_t)(nsplit + 1) * p.q;
+  cudaError_t e = cudaFuncSetAttribute(attn_combine_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem);
+  if (e != cudaSuccess) return e;
+  attn_combine_kernel<T><<<p.U, 256, csmem, s>>>(Opart, ML, nsplit, p.q, p.d, p.H, QMAX, static_cast<T*>(O),
+                                                 od.stride_b, od.stride_h, od.stride_s);
+  return cudaGetLastError();
+}
+
 template <typename T, int D, int QM>
 cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                 const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg, const wf_tensor* g,
@@ -185,13 +198,7 @@ cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const voi
       static_cast<const T*>(V), kv.stride_b, kv.stride_h, kv.stride_s, kv.seq, idx, p.k, static_cast<const T*>(Kg),
       static_cast<const T*>(Vg), gsb, gsh, gss, p.ng, p.q, p.H, p.G, scale, p.nsplit, Opart, ML);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const size_t csmem = sizeof(float) * (size_t)(p.nsplit + 1) * p.q;
-  if ((e = cudaFuncSetAttribute(attn_combine_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem)) !=
-      cudaSuccess)
-    return e;
-  attn_combine_kernel<T><<<p.U, 256, csmem, s>>>(Opart, ML, p.nsplit, p.q, D, p.H, QMAX, static_cast<T*>(O),
-                                                 od.stride_b, od.stride_h, od.stride_s);
-  return cudaGetLastError();
+  return combine<T>(p, p.nsplit, O, od, ws, s);
 }
 
 }  // namespace
@@ -207,7 +214,7 @@ AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group) {
   p.ng = ng;
   p.dtype = q.dtype;
   p.nsplit = (k + ng + CH - 1) / CH;
-  size_t off = 0;
+  size_t off = 256;  // status block
   p.off_o = off;  off = align_up(off + (size_t)p.U * p.nsplit * QMAX * p.d * sizeof(float), 256);
   p.off_ml = off; off = align_up(off + (size_t)p.U * p.nsplit * QMAX * sizeof(float2), 256);
   p.total = off;
@@ -216,7 +223,15 @@ AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group) {
 
 cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                         const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
-                        const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s) {
+                        const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, int* status,
+                        cudaStream_t s) {
+  // bf16 with head_dim 128: tensor cores.
+  if (tc_attn_supported(p, p.G * p.q)) {
+    int nsplit = 0;
+    cudaError_t e = launch_tc_attn(p, Q, qd, K, V, kv, idx, Kg, Vg, g, scale, status, ws, &nsplit, s);
+    if (e != cudaSuccess) return e;
+    return combine<bf16>(p, nsplit, O, od, ws, s);
+  }
   // Query blocks of up to 32 rows take the 32-row tile.
 #define WF_ATTN_RUN(T, DD)                                                                  \
   (p.q <= 32 ? run<T, DD, 32>(p, Q, qd, K, V, kv, idx, Kg, Vg, g, O, od, scale, ws, s)     \

@@ -300,7 +300,7 @@ FilterPlan plan_filter(const wf_tensor& q, const wf_tensor& kv, int levels, cons
   p.tiles_max = (cmax + TILE - 1) / TILE;
   p.trim = keep[0] < 2 * keep[1];
   const size_t U = (size_t)p.U;
-  size_t off = 0;
+  size_t off = 256;  // status block
   p.off_cand_a = off; off = align_up(off + U * cmax * sizeof(int32_t), 256);
   p.off_cand_b = off; off = align_up(off + U * cmax * sizeof(int32_t), 256);
   p.off_w = off;      off = align_up(off + U * cmax * sizeof(float), 256);
@@ -310,9 +310,24 @@ FilterPlan plan_filter(const wf_tensor& q, const wf_tensor& kv, int levels, cons
   return p;
 }
 
+namespace {
+// Eq. 7-8 for one scale: the ranking key of each of the m candidates into W
+// (tensor cores where they apply, else the fp32 score and weights kernels).
+cudaError_t skim(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand, int m,
+                 float* logits, float2* part, float* W, int* status, cudaStream_t s) {
+  if (tc_skim_supported(p)) return launch_tc_skim(p, Q, qd, src, cand, m, part, W, status, s);
+  cudaError_t e;
+  if ((e = score(p, Q, qd, src, cand, m, logits, part, s)) != cudaSuccess) return e;
+  const int ntiles = (m + TILE - 1) / TILE;
+  weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
+                                                            (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
+  return cudaGetLastError();
+}
+}  // namespace
+
 cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* coeffs,
                           const void* K, const wf_tensor& kv, int32_t* idx, int32_t* level_sets, void* ws,
-                          cudaStream_t s) {
+                          int* status, cudaStream_t s) {
   char* base = static_cast<char*>(ws);
   int32_t* cand_cur = reinterpret_cast<int32_t*>(base + p.off_cand_a);
   int32_t* cand_nxt = reinterpret_cast<int32_t*>(base + p.off_cand_b);
@@ -336,11 +351,7 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
     src.ss = p.d;
     src.off = ((int64_t)p.n - ((int64_t)p.n >> (l - 1))) * p.d;
     const int32_t* cand = first ? nullptr : cand_cur;
-    if ((e = score(p, Q, qd, src, cand, m, logits, part, s)) != cudaSuccess) return e;
-    const int ntiles = (m + TILE - 1) / TILE;
-    weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
-                                                              (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = skim(p, Q, qd, src, cand, m, logits, part, W, status, s)) != cudaSuccess) return e;
     const bool last = (l == 1) && !p.trim;
     int32_t* out = last ? idx : cand_nxt;
     const int64_t out_stride = last ? p.keep[0] : p.cmax;
@@ -359,11 +370,7 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
     src.sh = kv.stride_h;
     src.ss = kv.stride_s;
     src.off = 0;
-    if ((e = score(p, Q, qd, src, cand_cur, m, logits, part, s)) != cudaSuccess) return e;
-    const int ntiles = (m + TILE - 1) / TILE;
-    weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
-                                                              (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = skim(p, Q, qd, src, cand_cur, m, logits, part, W, status, s)) != cudaSuccess) return e;
     select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -383,7 +390,7 @@ size_t wavelet_filter_bytes(const FilterPlan& p) {
 
 cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* top,
                                   const void* K, const wf_tensor& kv, int wavelet, int32_t* idx, int32_t* level_sets,
-                                  void* ws, cudaStream_t s) {
+                                  void* ws, int* status, cudaStream_t s) {
   // The same scan as launch_filter, except that the rows of scale l < L are
   // the approximation rows of the transform of the candidates' gathered
   // blocks (computed here, in candidate order) instead of pyramid rows.
@@ -414,11 +421,7 @@ cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_t
       src.sh = (int64_t)p.cmax * p.d;
     }
     src.sb = src.sh * p.H;
-    if ((e = score(p, Q, qd, src, nullptr, m, logits, part, s)) != cudaSuccess) return e;
-    const int ntiles = (m + TILE - 1) / TILE;
-    weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
-                                                              (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = skim(p, Q, qd, src, nullptr, m, logits, part, W, status, s)) != cudaSuccess) return e;
     const bool last = (l == 1) && !p.trim;
     int32_t* out = last ? idx : cand_nxt;
     const int64_t out_stride = last ? p.keep[0] : p.cmax;
@@ -437,11 +440,7 @@ cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_t
     src.sh = kv.stride_h;
     src.ss = kv.stride_s;
     src.off = 0;
-    if ((e = score(p, Q, qd, src, cand_cur, m, logits, part, s)) != cudaSuccess) return e;
-    const int ntiles = (m + TILE - 1) / TILE;
-    weights_kernel<<<dim3((m + 255) / 256, p.U), 256, 0, s>>>(logits, (int64_t)p.q * p.cmax, p.cmax, part,
-                                                              (int64_t)p.tiles_max * p.q, ntiles, p.q, m, W, p.cmax);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = skim(p, Q, qd, src, cand_cur, m, logits, part, W, status, s)) != cudaSuccess) return e;
     select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

@@ -76,15 +76,22 @@ struct FilterPlan {
   int cmax;        // largest candidate count over the scales (and the trim)
   int tiles_max;   // ceil(cmax / kScoreTile)
   bool trim;
-  size_t off_cand_a, off_cand_b, off_w, off_logits, off_part, total;
+  size_t off_cand_a, off_cand_b, off_w, off_logits, off_part, total;  // a 256-byte status block precedes off_cand_a
 };
 constexpr int kScoreTile = 32;
 constexpr int kMaxQ = 64;    // query rows per query head
 constexpr int kMaxQR = 256;  // query rows per KV head (all heads of a group)
 FilterPlan plan_filter(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep);
+// status: the word a tensor-core kernel sets when a bounded wait gives up.
 cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* coeffs,
                           const void* K, const wf_tensor& kv, int32_t* idx, int32_t* level_sets, void* ws,
-                          cudaStream_t s);
+                          int* status, cudaStream_t s);
+// The tensor-core skim (bf16, head_dim 128, <= 256 query rows per unit): the
+// per-tile softmax partials and the ranking keys log2 W of one scale's m
+// candidates (rows from src, gathered through cand when not NULL).
+bool tc_skim_supported(const FilterPlan& p);
+cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
+                           int m, float2* part, float* W, int* status, cudaStream_t s);
 
 // Approximation rows at scale `level` of the periodized transform (wavelet
 // WF_WAVELET_*) of the keys of blocks [2^level c, 2^level (c + 1)) for the m
@@ -99,7 +106,7 @@ int wavelet_max_level(int wavelet);  // deepest scale the approximation kernel s
 size_t wavelet_filter_bytes(const FilterPlan& p);
 cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_tensor& qd, const void* top,
                                   const void* K, const wf_tensor& kv, int wavelet, int32_t* idx, int32_t* level_sets,
-                                  void* ws, cudaStream_t s);
+                                  void* ws, int* status, cudaStream_t s);
 
 // Sparse attention workspace plan.  A unit is one (batch, query head); it
 // reads KV head h / G and that head's index row.
@@ -110,9 +117,19 @@ struct AttnPlan {
 };
 constexpr int kAttnChunk = 64;
 AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group);
+// status: the word a tensor-core kernel sets when a bounded wait gives up.
 cudaError_t launch_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                         const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
-                        const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, cudaStream_t s);
+                        const wf_tensor* g, void* O, const wf_tensor& od, float scale, void* ws, int* status,
+                        cudaStream_t s);
+// The tensor-core split attention (bf16, head_dim 128, <= 256 query rows per
+// key unit): partials in the workspace's flash-decoding layout, split count
+// into *nsplit_out.
+bool tc_attn_supported(const AttnPlan& p, int kv_group_rows);
+cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
+                           const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
+                           const wf_tensor* g, float scale, int* status, void* ws, int* nsplit_out,
+                           cudaStream_t s);
 
 // Fused step (bf16, head_dim 128, <= 32 query rows): one cluster of cs CTAs
 // per P units.

@@ -1,0 +1,523 @@
+// Tensor-core skim for the per-stage filter (bf16 keys, head_dim 128): the
+// scores of one scale (Eq. 7 logits) as tcgen05 MMAs of 128 gathered
+// candidate rows against the unit's whole query block (up to 256 rows: the
+// grouped heads of a key head), in two passes over the same tiles.
+//   stats: per (tile, query row) the max and the sum of 2^(s - max) of the
+//          tile's logits (log2 units) -> part[unit][tile][row];
+//   keys:  the query rows' normalisers c_i = M_i + log2 S_i folded from all
+//          tiles' partials, then each candidate's ranking key
+//          log2 W_j = log2 sum_i 2^(s_ij - c_i) (Eq. 8 as a log-sum-exp)
+//          -> W[unit][j].
+// The keys pass recomputes the MMA instead of storing the logits: a tile's
+// rows are read twice (the second time mostly from L2) and no logit matrix
+// goes through memory.
+//
+// One CTA (four warps, one TMEM lane quarter each) per (tile, unit): all
+// threads gather the tile (16-byte cp.async into the 128-byte-swizzled
+// K-major layout) and the query block (K-major core matrices, zero rows up
+// to a multiple of 32), one thread issues the eight MMAs (K = 128) into TMEM
+// and commits them to an mbarrier, and every thread reads back its
+// candidate's row in chunks of 32 query columns.  The wait on the MMAs is
+// bounded (~1 s): on a timeout the CTA sets the status word, waits once more
+// with the same bound, frees its TMEM and leaves.
+#include <math.h>
+
+#include "wf_internal.cuh"
+#include "wf_sm100.cuh"
+
+namespace wf {
+namespace {
+
+using namespace sm100;
+
+constexpr int D = 128;
+constexpr int TM = 128;                // candidate rows per tile (MMA M)
+constexpr int NTH = 128;               // threads per CTA
+constexpr int HALF = TM * 128;         // one 64-column half of the tile
+constexpr int QGRP = (D / 8) * 128;    // bytes per 8-row group of the query block
+constexpr long long kWait = 1ll << 31;
+
+struct TcArgs {
+  const bf16* Q;
+  int64_t qsb, qsh, qss;
+  int q, G, qs, H;              // query rows per unit (G heads of qs rows), key heads
+  RowSrc src;                   // candidate rows (row index = cand[j] or j)
+  const int32_t* cand;
+  int64_t cand_stride;
+  int m;                        // candidates of the scale
+  int nq;                       // query columns of the MMA (q rounded up to 32)
+  uint32_t tcols;               // TMEM columns allocated
+  float2* part;                 // [unit][tile][q]
+  int64_t part_unit;
+  float* W;                     // [unit][w_unit]
+  int64_t w_unit;
+  int* status;
+  float sl2;                    // log2(e) / sqrt(d)
+};
+
+// Lane l of the warp ends with the reduction of column l over the warp's 32
+// lanes (31 shuffles).
+template <bool MAX>
+__device__ __forceinline__ float xpose_reduce32(float (&v)[32], int lane) {
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) {
+    const bool up = (lane & off) != 0;
+#pragma unroll
+    for (int j = 0; j < off; ++j) {
+      const float keep = up ? v[j + off] : v[j];
+      const float send = up ? v[j] : v[j + off];
+      const float recv = __shfl_xor_sync(0xffffffffu, send, off);
+      v[j] = MAX ? fmaxf(keep, recv) : keep + recv;
+    }
+  }
+  return v[0];
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ TcArgs a) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint8_t* tile = smem;                        // 2 x HALF, 1024-aligned
+  uint8_t* sq = smem + 2 * HALF;               // nq / 8 groups of QGRP
+  float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [4][32]
+  float* col = red + 4 * 32;                   // [256]: per-column max, or the normalisers c_i
+  unsigned long long* bar = reinterpret_cast<unsigned long long*>(col + 256);
+  uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 1);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int t = blockIdx.x, u = blockIdx.y;
+  const int64_t bb = u / a.H, hh = u % a.H;
+
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tbase), a.tcols);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    mbar_init(smem_u32(bar), 1);
+    fence_mbar_init();
+  }
+  // The tile: chunk c = tid % 16 of rows tid / 16 + 8 i, 128-byte swizzle.
+  {
+    const int c = tid & 15;
+    const bf16* rb = static_cast<const bf16*>(a.src.base) + bb * a.src.sb + hh * a.src.sh + a.src.off;
+    const int32_t* cd = a.cand ? a.cand + (int64_t)u * a.cand_stride : nullptr;
+    const uint32_t cbase = smem_u32(tile) + ((c >> 3) * HALF);
+#pragma unroll 4
+    for (int i = 0; i < TM / 8; ++i) {
+      const int r = (tid >> 4) + 8 * i;
+      const int j = min(t * TM + r, a.m - 1);  // rows past the list repeat its last row (finite, masked)
+      const int64_t row = cd ? (int64_t)cd[j] : (int64_t)j;
+      cp_async16(cbase + r * 128 + (((c & 7) ^ (r & 7)) << 4), rb + row * a.src.ss + c * 8);
+    }
+  }
+  // The query block, K-major core matrices; rows q .. nq - 1 zero.
+  for (int e = tid; e < a.nq * (D / 8); e += NTH) {
+    const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
+    const int i = g * 8 + rr;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (i < a.q) {
+      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + i / a.qs) * a.qsh + (int64_t)(i % a.qs) * a.qss;
+      v = __ldg(reinterpret_cast<const uint4*>(qp + ch * 8));
+    }
+    *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
+  }
+  cp_async_wait_all();
+  fence_proxy_async();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tbase;
+  const uint32_t idesc = idesc_bf16(TM, a.nq, 0, 0);
+  if (tid == 0) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        mma_bf16(tmem, smem_desc_sw128(smem_u32(tile) + h * HALF + kk * 32, 16, 1024),
+                 smem_desc(smem_u32(sq) + (4 * h + kk) * 256, 128, QGRP), idesc, (h | kk) != 0);
+    mma_commit(smem_u32(bar));
+  }
+  __syncwarp();
+  bool ok = mbar_wait_bounded(smem_u32(bar), 0u, kWait);
+  if (!ok) {
+    atomicExch(a.status, 1);
+    (void)mbar_wait_bounded(smem_u32(bar), 0u, kWait);
+  }
+  ok = __syncthreads_and(ok);
+  tc_fence_after();
+
+  const int j = t * TM + tid;  // this thread's candidate (TMEM lane tid)
+  const bool valid = j < a.m;
+  const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+  const int nch = a.nq / 32;
+  if (ok && MODE == 0) {
+    float2* pt = a.part + (int64_t)u * a.part_unit + (int64_t)t * a.q;
+#pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) {
+      float v[32], w[32];
+      tmem_ld32(lane_base + 32 * ch, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        v[i] = valid ? v[i] * a.sl2 : -INFINITY;
+        w[i] = v[i];
+      }
+      red[warp * 32 + lane] = xpose_reduce32<true>(w, lane);
+      __syncthreads();
+      if (tid < 32) col[tid] = fmaxf(fmaxf(red[tid], red[32 + tid]), fmaxf(red[64 + tid], red[96 + tid]));
+      __syncthreads();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) w[i] = valid ? ex2(v[i] - col[i]) : 0.f;
+      red[warp * 32 + lane] = xpose_reduce32<false>(w, lane);
+      __syncthreads();
+      if (tid < 32 && ch * 32 + tid < a.q)
+        pt[ch * 32 + tid] = make_float2(col[tid], (red[tid] + red[32 + tid]) + (red[64 + tid] + red[96 + tid]));
+      __syncthreads();
+    }
+  }
+  if (ok && MODE == 1) {
+    // c_i over all tiles of the scale (columns past q never count).
+    const int ntiles = (a.m + TM - 1) / TM;
+    const float2* pu = a.part + (int64_t)u * a.part_unit;
+    for (int i = tid; i < a.nq; i += NTH) {
+      float c = INFINITY;
+      if (i < a.q) {
+        float M = -INFINITY;
+        for (int tt = 0; tt < ntiles; ++tt) M = fmaxf(M, pu[(int64_t)tt * a.q + i].x);
+        float S = 0.f;
+        for (int tt = 0; tt < ntiles; ++tt) {
+          const float2 p = pu[(int64_t)tt * a.q + i];
+          S += p.y * ex2(p.x - M);
+        }
+        c = M + lg2(S);
+      }
+      col[i] = c;
+    }
+    __syncthreads();
+    float mx = -INFINITY;
+#pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) {
+      float v[32];
+      tmem_ld32(lane_base + 32 * ch, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (ch * 32 + i < a.q) mx = fmaxf(mx, fmaf(v[i], a.sl2, -col[ch * 32 + i]));
+    }
+    float z = 0.f;
+#pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) {
+      float v[32];
+      tmem_ld32(lane_base + 32 * ch, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (ch * 32 + i < a.q) z += ex2(fmaf(v[i], a.sl2, -col[ch * 32 + i]) - mx);
+    }
+    if (valid) a.W[(int64_t)u * a.w_unit + j] = mx + lg2(z);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, a.tcols);
+  }
+}
+
+}  // namespace
+
+bool tc_skim_supported(const FilterPlan& p) { return p.dtype == WF_BF16 && p.d == D && p.q <= 256; }
+
+cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
+                           int m, float2* part, float* W, int* status, cudaStream_t s) {
+  TcArgs a;
+  a.Q = static_cast<const bf16*>(Q);
+  a.qsb = qd.stride_b; a.qsh = qd.stride_h; a.qss = qd.stride_s;
+  a.q = p.q; a.G = p.G; a.qs = p.qs; a.H = p.H;
+  a.src = src;
+  a.cand = cand;
+  a.cand_stride = p.cmax;
+  a.m = m;
+  a.nq = (p.q + 31) / 32 * 32;
+  uint32_t cols = 32;
+  while ((int)cols < a.nq) cols *= 2;
+  a.tcols = cols;
+  a.part = part;
+  a.part_unit = (int64_t)p.tiles_max * p.q;
+  a.W = W;
+  a.w_unit = p.cmax;
+  a.status = status;
+  a.sl2 = 1.4426950408889634f / sqrtf((float)D);
+  // Shared memory: the tile, the query block, the reductions, the barrier.
+  // At most 512 / cols CTAs may share an SM (TMEM); the request is padded so
+  // that shared memory enforces it.
+  size_t smem = 2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (4 * 32 + 256) + 16;
+  const size_t per_sm = 228 * 1024;
+  const size_t cap = 512 / cols;  // CTAs per SM the TMEM allows
+  const size_t floor_smem = per_sm / (cap + 1) + 1;
+  if (cap < 16 && smem < floor_smem) smem = floor_smem;
+  const dim3 grid((unsigned)((m + TM - 1) / TM), (unsigned)p.U);
+  cudaError_t e = cudaFuncSetAttribute(tc_score_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_score_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  tc_score_kernel<0><<<grid, NTH, smem, s>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  tc_score_kernel<1><<<grid, NTH, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace wf
+
+// ---------------------------------------------------------------------------
+// Tensor-core sparse attention (Algorithm 1, final step) for the per-stage
+// path: one CTA per (key unit, split of 128 sparse keys).  The split's K and
+// V rows ([K[idx]; Kg] and [V[idx]; Vg]) are gathered into two
+// 128-byte-swizzled tiles, S^T = K Q^T goes to TMEM (keys on the lanes, the
+// unit's query rows on the columns), every thread turns its key's row into
+// P = 2^(s - m) with m the split's per-query max (bf16, stored as P^T in
+// MN-major core matrices), and O^T = V^T P^T goes to TMEM.  The partial
+// (O, m, l) of every query row lands in the flash-decoding layout of the
+// fp32 kernels, per query head, so the same combine kernel finishes it.
+// ---------------------------------------------------------------------------
+namespace wf {
+namespace {
+
+using namespace sm100;
+
+struct TcAttnArgs {
+  const bf16* Q;
+  int64_t qsb, qsh, qss;
+  const bf16* K;
+  const bf16* V;
+  int64_t ksb, ksh, kss;
+  const bf16* Kg;
+  const bf16* Vg;
+  int64_t gsb, gsh, gss;
+  const int32_t* idx;
+  int n, k, ng, q, G, qs, H;  // q = G qs query rows per key unit; H key heads
+  int nq;                     // MMA columns (q rounded up to 32)
+  uint32_t tcols;
+  int nsplit;
+  float* Opart;               // [query unit][nsplit][qstride][D]
+  float2* ML;                 // [query unit][nsplit][qstride]
+  int qstride;
+  int* status;
+  float sl2;
+};
+
+__global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ TcAttnArgs a) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint8_t* kt = smem;                          // K tile, 2 x HALF
+  uint8_t* vt = smem + 2 * HALF;               // V tile, 2 x HALF
+  uint8_t* sq = smem + 4 * HALF;               // query block, nq / 8 groups of QGRP
+  uint8_t* pb = sq + (a.nq / 8) * QGRP;        // P^T: 16 key groups of nq * 16 bytes
+  float* red = reinterpret_cast<float*>(pb + a.nq * 256);  // [4][32]
+  float* cm = red + 4 * 32;                    // [256] split max per query (log2 units)
+  float* cl = cm + 256;                        // [256] split row sums of P
+  unsigned long long* bar = reinterpret_cast<unsigned long long*>(cl + 256);  // [2]
+  uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 2);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int sp = blockIdx.x, u = blockIdx.y;
+  const int64_t bb = u / a.H, hh = u % a.H;
+  const int total = a.k + a.ng, t0 = sp * TM;
+
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tbase), a.tcols);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    mbar_init(smem_u32(&bar[0]), 1);
+    mbar_init(smem_u32(&bar[1]), 1);
+    fence_mbar_init();
+  }
+  // K and V rows of the split: chunk c = tid % 16 of rows tid / 16 + 8 i.
+  {
+    const int c = tid & 15;
+    const int32_t* ui = a.idx + (int64_t)u * a.k;
+    const uint32_t koff = smem_u32(kt) + ((c >> 3) * HALF), voff = smem_u32(vt) + ((c >> 3) * HALF);
+#pragma unroll 4
+    for (int i = 0; i < TM / 8; ++i) {
+      const int r = (tid >> 4) + 8 * i;
+      const int tt = min(t0 + r, total - 1);  // keys past the list repeat its last key (P = 0 there)
+      const bf16 *kp, *vp;
+      if (tt < a.k) {
+        int row = ui[tt];
+        row = row < 0 ? 0 : (row >= a.n ? a.n - 1 : row);
+        const int64_t o = bb * a.ksb + hh * a.ksh + (int64_t)row * a.kss + c * 8;
+        kp = a.K + o;
+        vp = a.V + o;
+      } else {
+        const int64_t o = bb * a.gsb + hh * a.gsh + (int64_t)(tt - a.k) * a.gss + c * 8;
+        kp = a.Kg + o;
+        vp = a.Vg + o;
+      }
+      const uint32_t so = r * 128 + (((c & 7) ^ (r & 7)) << 4);
+      cp_async16(koff + so, kp);
+      cp_async16(voff + so, vp);
+    }
+  }
+  for (int e = tid; e < a.nq * (D / 8); e += NTH) {
+    const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
+    const int i = g * 8 + rr;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (i < a.q) {
+      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + i / a.qs) * a.qsh + (int64_t)(i % a.qs) * a.qss;
+      v = __ldg(reinterpret_cast<const uint4*>(qp + ch * 8));
+    }
+    *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
+  }
+  cp_async_wait_all();
+  fence_proxy_async();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tbase;
+  const uint32_t ocol = tmem + (uint32_t)a.nq;  // O^T columns after S^T
+  if (tid == 0) {
+    const uint32_t idesc = idesc_bf16(TM, a.nq, 0, 0);
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        mma_bf16(tmem, smem_desc_sw128(smem_u32(kt) + h * HALF + kk * 32, 16, 1024),
+                 smem_desc(smem_u32(sq) + (4 * h + kk) * 256, 128, QGRP), idesc, (h | kk) != 0);
+    mma_commit(smem_u32(&bar[0]));
+  }
+  __syncwarp();
+  bool ok = mbar_wait_bounded(smem_u32(&bar[0]), 0u, kWait);
+  if (!ok) {
+    atomicExch(a.status, 1);
+    (void)mbar_wait_bounded(smem_u32(&bar[0]), 0u, kWait);
+  }
+  ok = __syncthreads_and(ok);
+  tc_fence_after();
+
+  const bool valid = t0 + tid < total;  // this thread's key (TMEM lane tid)
+  const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+  const int nch = a.nq / 32;
+  if (ok) {
+    uint8_t* prow = pb + (tid >> 3) * (a.nq * 16) + (tid & 7) * 16;
+#pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) {
+      float v[32], w[32];
+      tmem_ld32(lane_base + 32 * ch, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        v[i] = valid ? v[i] * a.sl2 : -INFINITY;
+        w[i] = v[i];
+      }
+      red[warp * 32 + lane] = xpose_reduce32<true>(w, lane);
+      __syncthreads();
+      if (tid < 32) cm[ch * 32 + tid] = fmaxf(fmaxf(red[tid], red[32 + tid]), fmaxf(red[64 + tid], red[96 + tid]));
+      __syncthreads();
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        const float p0 = valid ? ex2(v[i] - cm[ch * 32 + i]) : 0.f;
+        const float p1 = valid ? ex2(v[i + 1] - cm[ch * 32 + i + 1]) : 0.f;
+        const __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+        w[i] = __low2float(h2);
+        w[i + 1] = __high2float(h2);
+        pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h2);
+      }
+#pragma unroll
+      for (int c4 = 0; c4 < 4; ++c4)
+        *reinterpret_cast<uint4*>(prow + (ch * 4 + c4) * 128) =
+            make_uint4(pk[4 * c4], pk[4 * c4 + 1], pk[4 * c4 + 2], pk[4 * c4 + 3]);
+      red[warp * 32 + lane] = xpose_reduce32<false>(w, lane);
+      __syncthreads();
+      if (tid < 32) cl[ch * 32 + tid] = (red[tid] + red[32 + tid]) + (red[64 + tid] + red[96 + tid]);
+      __syncthreads();
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (tid == 0) {
+      const uint32_t idesc = idesc_bf16(D, a.nq, 1, 1);
+#pragma unroll
+      for (int kq = 0; kq < TM / 16; ++kq)
+        mma_bf16(ocol, smem_desc_sw128(smem_u32(vt) + kq * 2048, HALF, 1024),
+                 smem_desc(smem_u32(pb) + kq * 2 * (a.nq * 16), a.nq * 16, 128), idesc, kq > 0 ? 1u : 0u);
+      mma_commit(smem_u32(&bar[1]));
+    }
+    __syncwarp();
+    bool ok2 = mbar_wait_bounded(smem_u32(&bar[1]), 0u, kWait);
+    if (!ok2) {
+      atomicExch(a.status, 1);
+      (void)mbar_wait_bounded(smem_u32(&bar[1]), 0u, kWait);
+    }
+    ok2 = __syncthreads_and(ok2);
+    tc_fence_after();
+    if (ok2) {
+      // Thread tid holds head-dim row tid of O^T: query columns in chunks.
+      const float ln2 = 0.69314718055994531f;
+#pragma unroll 1
+      for (int ch = 0; ch < nch; ++ch) {
+        float o[32];
+        tmem_ld32(ocol + ((uint32_t)(warp * 32) << 16) + 32 * ch, o);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int col = ch * 32 + i;
+          if (col < a.q) {
+            const int64_t uq = bb * (a.H * a.G) + hh * a.G + col / a.qs;
+            const int iq = col % a.qs;
+            a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + tid] = o[i];
+          }
+        }
+      }
+      for (int col = tid; col < a.q; col += NTH) {
+        const int64_t uq = bb * (a.H * a.G) + hh * a.G + col / a.qs;
+        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + col % a.qs] = make_float2(cm[col] * ln2, cl[col]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, a.tcols);
+  }
+}
+
+}  // namespace
+
+bool tc_attn_supported(const AttnPlan& p, int kv_group_rows) {
+  return p.dtype == WF_BF16 && p.d == D && kv_group_rows <= 256;
+}
+
+cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd, const void* K, const void* V,
+                           const wf_tensor& kv, const int32_t* idx, const void* Kg, const void* Vg,
+                           const wf_tensor* g, float scale, int* status, void* ws, int* nsplit_out,
+                           cudaStream_t s) {
+  TcAttnArgs a;
+  a.Q = static_cast<const bf16*>(Q);
+  a.qsb = qd.stride_b; a.qsh = qd.stride_h; a.qss = qd.stride_s;
+  a.K = static_cast<const bf16*>(K);
+  a.V = static_cast<const bf16*>(V);
+  a.ksb = kv.stride_b; a.ksh = kv.stride_h; a.kss = kv.stride_s;
+  a.Kg = static_cast<const bf16*>(Kg);
+  a.Vg = static_cast<const bf16*>(Vg);
+  a.gsb = g ? g->stride_b : 0; a.gsh = g ? g->stride_h : 0; a.gss = g ? g->stride_s : 0;
+  a.idx = idx;
+  a.n = kv.seq; a.k = p.k; a.ng = p.ng;
+  a.G = p.G; a.qs = p.q; a.q = p.G * p.q; a.H = kv.heads;
+  a.nq = (a.q + 31) / 32 * 32;
+  uint32_t cols = 32;
+  while ((int)cols < 2 * a.nq) cols *= 2;
+  a.tcols = cols;
+  a.nsplit = (p.k + p.ng + TM - 1) / TM;
+  a.Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
+  a.ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
+  a.qstride = kMaxQ;
+  a.status = status;
+  a.sl2 = 1.4426950408889634f * scale;
+  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + (size_t)a.nq * 256 + sizeof(float) * (4 * 32 + 512) + 32;
+  const size_t per_sm = 228 * 1024;
+  const size_t cap = 512 / cols;
+  const size_t floor_smem = per_sm / (cap + 1) + 1;
+  if (cap < 16 && smem < floor_smem) smem = floor_smem;
+  cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  tc_attn_kernel<<<dim3((unsigned)a.nsplit, (unsigned)(kv.batch * kv.heads)), NTH, smem, s>>>(a);
+  *nsplit_out = a.nsplit;
+  return cudaGetLastError();
+}
+
+}  // namespace wf

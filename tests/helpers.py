@@ -25,7 +25,7 @@ class GpuRun:
         self.coeffs = torch.empty(wf.wf_coeffs_bytes(K, L), dtype=torch.uint8, device=dev)
         ws_bytes = max(wf.wf_filter_workspace_bytes(Q, K, L, self.keep),
                        wf.wf_attn_workspace_bytes(Q, self.keep[0], Kg.shape[2] if Kg is not None else 0))
-        self.ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+        self.ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)  # status word zeroed once
         self.idx = torch.empty(B * H, self.keep[0], dtype=torch.int32, device=dev)
         self.sets = torch.empty(B * H, sum(self.keep), dtype=torch.int32, device=dev) if want_sets else None
         self.O = torch.empty_like(Q)
@@ -36,6 +36,7 @@ class GpuRun:
 
     def filter(self):
         wf.wf_filter(self.Q, self.coeffs, self.K, self.L, self.keep, self.idx, self.ws, self.sets)
+        wf.wf_workspace_status(self.ws)  # raises if a bounded device wait gave up
         return self
 
     def attn(self, idx=None, scale=0.0):
