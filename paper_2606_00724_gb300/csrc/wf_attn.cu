@@ -134,38 +134,38 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
   }
 }
 
-// One CTA per unit: the weight exp(m_s - M) of every split s and query row
-// (and the denominator) is formed once in shared memory, then every output
+// One CTA per (unit, query row): the weight exp(m_s - M) of every split s
+// and the denominator are formed once in shared memory, then each output
 // element is one pass over the splits' partial outputs.
 template <typename T>
-__global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restrict__ Opart,
+__global__ void __launch_bounds__(128) attn_combine_kernel(const float* __restrict__ Opart,
                                                            const float2* __restrict__ ML, int nsplit, int q, int D,
                                                            int H, int qstride, T* __restrict__ O, int64_t osb,
                                                            int64_t osh, int64_t oss) {
-  extern __shared__ float fw[];  // [nsplit][q] weights, then the [q] denominators
-  float* den_s = fw + nsplit * q;
-  const int u = blockIdx.x;
+  extern __shared__ float fw[];  // [nsplit] weights, then the denominator
+  const int u = blockIdx.x, i = blockIdx.y;
   const int64_t bb = u / H, hh = u % H;
-  const float2* ml = ML + (int64_t)u * nsplit * qstride;
-  for (int i = threadIdx.x; i < q; i += blockDim.x) {
+  const float2* ml = ML + (int64_t)u * nsplit * qstride + i;
+  if (threadIdx.x < 32) {
     float mx = -INFINITY;
-    for (int s = 0; s < nsplit; ++s) mx = fmaxf(mx, ml[(int64_t)s * qstride + i].x);
-    float den = 0.f;
-    for (int s = 0; s < nsplit; ++s) {
-      const float2 p = ml[(int64_t)s * qstride + i];
-      const float f = expf(p.x - mx);
-      fw[s * q + i] = f;
-      den = fmaf(p.y, f, den);
+    for (int s = threadIdx.x; s < nsplit; s += 32) mx = fmaxf(mx, ml[(int64_t)s * qstride].x);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    for (int s = threadIdx.x; s < nsplit; s += 32) fw[s] = expf(ml[(int64_t)s * qstride].x - mx);
+    __syncwarp();
+    if (threadIdx.x == 0) {
+      float den = 0.f;
+      for (int s = 0; s < nsplit; ++s) den = fmaf(ml[(int64_t)s * qstride].y, fw[s], den);
+      fw[nsplit] = den;
     }
-    den_s[i] = den;
   }
   __syncthreads();
-  const float* op = Opart + (int64_t)u * nsplit * qstride * D;
-  for (int e = threadIdx.x; e < q * D; e += blockDim.x) {
-    const int i = e / D, c = e % D;
+  const float* op = Opart + ((int64_t)u * nsplit * qstride + i) * D;
+  const float den = fw[nsplit];
+  for (int c = threadIdx.x; c < D; c += blockDim.x) {
     float num = 0.f;
-    for (int s = 0; s < nsplit; ++s) num = fmaf(op[((int64_t)s * qstride + i) * D + c], fw[s * q + i], num);
-    from_f32(O[bb * osb + hh * osh + (int64_t)i * oss + c], num / den_s[i]);
+    for (int s = 0; s < nsplit; ++s) num = fmaf(op[(int64_t)s * qstride * D + c], fw[s], num);
+    from_f32(O[bb * osb + hh * osh + (int64_t)i * oss + c], num / den);
   }
 }
 
@@ -174,11 +174,11 @@ template <typename T>
 cudaError_t combine(const AttnPlan& p, int nsplit, void* O, const wf_tensor& od, void* ws, cudaStream_t s) {
   float* Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
   float2* ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
-  const size_t csmem = sizeof(float) * (size_t)(nsplit + 1) * p.q;
+  const size_t csmem = sizeof(float) * (size_t)(nsplit + 1);
   cudaError_t e = cudaFuncSetAttribute(attn_combine_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem);
   if (e != cudaSuccess) return e;
-  attn_combine_kernel<T><<<p.U, 256, csmem, s>>>(Opart, ML, nsplit, p.q, p.d, p.H, QMAX, static_cast<T*>(O),
-                                                 od.stride_b, od.stride_h, od.stride_s);
+  attn_combine_kernel<T><<<dim3((unsigned)p.U, (unsigned)p.q), 128, csmem, s>>>(
+      Opart, ML, nsplit, p.q, p.d, p.H, QMAX, static_cast<T*>(O), od.stride_b, od.stride_h, od.stride_s);
   return cudaGetLastError();
 }
 

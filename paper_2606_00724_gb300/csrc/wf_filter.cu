@@ -315,7 +315,9 @@ namespace {
 // (tensor cores where they apply, else the fp32 score and weights kernels).
 cudaError_t skim(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand, int m,
                  float* logits, float2* part, float* W, int* status, cudaStream_t s) {
-  if (tc_skim_supported(p)) return launch_tc_skim(p, Q, qd, src, cand, m, part, W, status, s);
+  // The fp32 logits buffer is not used by the tensor-core skim: its first
+  // U q floats hold the normalisers between the two passes.
+  if (tc_skim_supported(p)) return launch_tc_skim(p, Q, qd, src, cand, m, part, W, logits, status, s);
   cudaError_t e;
   if ((e = score(p, Q, qd, src, cand, m, logits, part, s)) != cudaSuccess) return e;
   const int ntiles = (m + TILE - 1) / TILE;

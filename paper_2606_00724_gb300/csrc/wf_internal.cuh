@@ -91,7 +91,7 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
 // candidates (rows from src, gathered through cand when not NULL).
 bool tc_skim_supported(const FilterPlan& p);
 cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
-                           int m, float2* part, float* W, int* status, cudaStream_t s);
+                           int m, float2* part, float* W, float* cvec, int* status, cudaStream_t s);
 
 // Approximation rows at scale `level` of the periodized transform (wavelet
 // WF_WAVELET_*) of the keys of blocks [2^level c, 2^level (c + 1)) for the m

@@ -4,8 +4,8 @@
 // grouped heads of a key head), in two passes over the same tiles.
 //   stats: per (tile, query row) the max and the sum of 2^(s - max) of the
 //          tile's logits (log2 units) -> part[unit][tile][row];
-//   keys:  the query rows' normalisers c_i = M_i + log2 S_i folded from all
-//          tiles' partials, then each candidate's ranking key
+//   keys:  the query rows' normalisers c_i = M_i + log2 S_i (folded from all
+//          tiles' partials by a small kernel in between), then each candidate's ranking key
 //          log2 W_j = log2 sum_i 2^(s_ij - c_i) (Eq. 8 as a log-sum-exp)
 //          -> W[unit][j].
 // The keys pass recomputes the MMA instead of storing the logits: a tile's
@@ -14,8 +14,8 @@
 //
 // One CTA (four warps, one TMEM lane quarter each) per (tile, unit): all
 // threads gather the tile (16-byte cp.async into the 128-byte-swizzled
-// K-major layout) and the query block (K-major core matrices, zero rows up
-// to a multiple of 32), one thread issues the eight MMAs (K = 128) into TMEM
+// K-major layout) and the query block (cp.async into K-major core matrices,
+// zero rows up to a multiple of 32), one thread issues the eight MMAs (K = 128) into TMEM
 // and commits them to an mbarrier, and every thread reads back its
 // candidate's row in chunks of 32 query columns.  The wait on the MMAs is
 // bounded (~1 s): on a timeout the CTA sets the status word, waits once more
@@ -51,9 +51,27 @@ struct TcArgs {
   int64_t part_unit;
   float* W;                     // [unit][w_unit]
   int64_t w_unit;
+  float* cvec;                  // [unit][q] normalisers c_i (folded between the passes)
   int* status;
   float sl2;                    // log2(e) / sqrt(d)
 };
+
+// c_i = M_i + log2 S_i of every query row from all tiles' partials.
+__global__ void __launch_bounds__(256) norm_kernel(const float2* __restrict__ part, int64_t part_unit, int ntiles,
+                                                   int q, float* __restrict__ cvec) {
+  const int u = blockIdx.y;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= q) return;
+  const float2* pu = part + (int64_t)u * part_unit + i;
+  float M = -INFINITY;
+  for (int tt = 0; tt < ntiles; ++tt) M = fmaxf(M, pu[(int64_t)tt * q].x);
+  float S = 0.f;
+  for (int tt = 0; tt < ntiles; ++tt) {
+    const float2 p = pu[(int64_t)tt * q];
+    S += p.y * ex2(p.x - M);
+  }
+  cvec[(int64_t)u * q + i] = M + lg2(S);
+}
 
 // Lane l of the warp ends with the reduction of column l over the warp's 32
 // lanes (31 shuffles).
@@ -112,12 +130,13 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
   for (int e = tid; e < a.nq * (D / 8); e += NTH) {
     const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
     const int i = g * 8 + rr;
-    uint4 v = make_uint4(0, 0, 0, 0);
+    const uint32_t dst = smem_u32(sq + g * QGRP + ch * 128 + rr * 16);
     if (i < a.q) {
       const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + i / a.qs) * a.qsh + (int64_t)(i % a.qs) * a.qss;
-      v = __ldg(reinterpret_cast<const uint4*>(qp + ch * 8));
+      cp_async16(dst, qp + ch * 8);
+    } else {
+      sts_v4(dst, make_uint4(0, 0, 0, 0));
     }
-    *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
   }
   cp_async_wait_all();
   fence_proxy_async();
@@ -173,23 +192,8 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
     }
   }
   if (ok && MODE == 1) {
-    // c_i over all tiles of the scale (columns past q never count).
-    const int ntiles = (a.m + TM - 1) / TM;
-    const float2* pu = a.part + (int64_t)u * a.part_unit;
-    for (int i = tid; i < a.nq; i += NTH) {
-      float c = INFINITY;
-      if (i < a.q) {
-        float M = -INFINITY;
-        for (int tt = 0; tt < ntiles; ++tt) M = fmaxf(M, pu[(int64_t)tt * a.q + i].x);
-        float S = 0.f;
-        for (int tt = 0; tt < ntiles; ++tt) {
-          const float2 p = pu[(int64_t)tt * a.q + i];
-          S += p.y * ex2(p.x - M);
-        }
-        c = M + lg2(S);
-      }
-      col[i] = c;
-    }
+    // The normalisers (columns past q never count).
+    for (int i = tid; i < a.nq; i += NTH) col[i] = i < a.q ? a.cvec[(int64_t)u * a.q + i] : INFINITY;
     __syncthreads();
     float mx = -INFINITY;
 #pragma unroll 1
@@ -224,7 +228,7 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
 bool tc_skim_supported(const FilterPlan& p) { return p.dtype == WF_BF16 && p.d == D && p.q <= 256; }
 
 cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
-                           int m, float2* part, float* W, int* status, cudaStream_t s) {
+                           int m, float2* part, float* W, float* cvec, int* status, cudaStream_t s) {
   TcArgs a;
   a.Q = static_cast<const bf16*>(Q);
   a.qsb = qd.stride_b; a.qsh = qd.stride_h; a.qss = qd.stride_s;
@@ -241,6 +245,7 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
   a.part_unit = (int64_t)p.tiles_max * p.q;
   a.W = W;
   a.w_unit = p.cmax;
+  a.cvec = cvec;
   a.status = status;
   a.sl2 = 1.4426950408889634f / sqrtf((float)D);
   // Shared memory: the tile, the query block, the reductions, the barrier.
@@ -257,6 +262,9 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
     e = cudaFuncSetAttribute(tc_score_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   tc_score_kernel<0><<<grid, NTH, smem, s>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  norm_kernel<<<dim3((unsigned)((p.q + 255) / 256), (unsigned)p.U), 256, 0, s>>>(part, a.part_unit,
+                                                                                (m + TM - 1) / TM, p.q, cvec);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   tc_score_kernel<1><<<grid, NTH, smem, s>>>(a);
   return cudaGetLastError();
@@ -355,12 +363,13 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   for (int e = tid; e < a.nq * (D / 8); e += NTH) {
     const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
     const int i = g * 8 + rr;
-    uint4 v = make_uint4(0, 0, 0, 0);
+    const uint32_t dst = smem_u32(sq + g * QGRP + ch * 128 + rr * 16);
     if (i < a.q) {
       const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + i / a.qs) * a.qsh + (int64_t)(i % a.qs) * a.qss;
-      v = __ldg(reinterpret_cast<const uint4*>(qp + ch * 8));
+      cp_async16(dst, qp + ch * 8);
+    } else {
+      sts_v4(dst, make_uint4(0, 0, 0, 0));
     }
-    *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
   }
   cp_async_wait_all();
   fence_proxy_async();

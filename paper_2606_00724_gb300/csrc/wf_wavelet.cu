@@ -9,9 +9,9 @@
 //
 // One CTA computes TO consecutive level-b rows for DS head-dim channels: it
 // gathers the TO 2^b input rows plus the (taps - 2)(2^b - 1) rows the filter
-// reaches past them (wrapping around the gathered sequence), widened to fp32
-// in shared memory, and runs the b levels of the cascade there (two buffers
-// alternating).  Arithmetic (the storage rule, shared with the Haar pyramid):
+// reaches past them (wrapping around the gathered sequence) into shared
+// memory with 16-byte cp.async copies, and runs the b levels of the cascade
+// there in fp32 (two buffers alternating).  Arithmetic (the storage rule, shared with the Haar pyramid):
 // Haar: fl32(x0 + x1) * fl32(1 / sqrt 2); db2: the products
 // fl32(fl32(h[k]) * x) added left to right in fp32, no fused multiply-add.
 // Only the last level is rounded to the key dtype.
@@ -22,9 +22,8 @@
 namespace wf {
 namespace {
 
-constexpr int DS = 16;        // head-dim channels per CTA
-constexpr int NTH = 128;      // threads per CTA
-constexpr int IN_ROWS = 512;  // gathered rows per CTA before the filter's reach
+constexpr int NTH = 256;      // threads per CTA
+constexpr int IN_ROWS = 256;  // gathered rows per CTA before the filter's reach
 
 // Output rows per CTA at scale `level`.
 __host__ __device__ inline int outputs_per_cta(int level) { return (IN_ROWS >> level) > 0 ? (IN_ROWS >> level) : 1; }
@@ -37,16 +36,23 @@ struct Taps {
   float h[4];
 };
 
-template <typename T, int TAPS>
+template <typename T>
+__device__ __forceinline__ float rd(const T* p) { return to_f32(*p); }
+
+// Shared memory: the gathered rows as loaded (T), then the fp32 levels
+// alternating between a second buffer and the first one (which holds at
+// least as many fp32 rows as the level after the first needs).
+template <typename T, int TAPS, int DS>
 __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, int64_t ksb, int64_t ksh, int64_t kss,
                                                      int64_t n, int H, const int32_t* __restrict__ cand,
                                                      int64_t cand_stride, int m, int level, Taps taps, T* __restrict__ out,
                                                      int64_t out_unit, int64_t out_row) {
-  extern __shared__ __align__(16) float buf[];
+  extern __shared__ __align__(16) uint8_t sbuf[];
   const int to = outputs_per_cta(level);
   const int nin = rows_needed(to, level, TAPS);
-  float* X = buf;                     // [nin][DS]
-  float* Y = buf + (size_t)nin * DS;  // [nin / 2 + 1][DS]
+  T* X0 = reinterpret_cast<T*>(sbuf);                                    // [nin][DS] raw
+  float* Y = reinterpret_cast<float*>(sbuf + (size_t)nin * DS * sizeof(T));  // [nin / 2 + 1][DS]
+  float* X = reinterpret_cast<float*>(sbuf);                             // fp32 levels >= 2
   const int u = blockIdx.y;
   const int j0 = blockIdx.x * to;
   const int c0 = blockIdx.z * DS;
@@ -57,68 +63,91 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   const int32_t* cd = cand ? cand + (int64_t)u * cand_stride : nullptr;
   const int tid = threadIdx.x;
 
-  // Gather: row r is gathered position (j0 2^b + r) mod len.
+  // Gather: row r is gathered position (j0 2^b + r) mod len, 16-byte copies.
   constexpr int VEC = Vec<T>::N;
   constexpr int VPR = DS / VEC;  // 16-byte vectors per row
+  const uint32_t xs = (uint32_t)__cvta_generic_to_shared(X0);
   for (int e = tid; e < nin * VPR; e += NTH) {
     const int r = e / VPR, v = e % VPR;
     const int64_t p = (((int64_t)j0 << level) + r) % len;
     int64_t tok = cd ? (((int64_t)cd[p >> level]) << level) + (p & blk_mask) : p;
     tok = tok < 0 ? 0 : (tok >= n ? n - 1 : tok);  // out-of-range block indices are clamped
-    float x[VEC];
-    ld_vec(kb + tok * kss + v * VEC, x);
-#pragma unroll
-    for (int i = 0; i < VEC; ++i) X[r * DS + v * VEC + i] = x[i];
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(xs + (uint32_t)((r * DS + v * VEC) * sizeof(T))),
+                 "l"(kb + tok * kss + v * VEC)
+                 : "memory");
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
 
   const float c32 = 0.70710678118654752440f;  // fl32(1 / sqrt 2)
-  float* src = X;
-  float* dst = Y;
 #pragma unroll 1
   for (int l = 1; l <= level; ++l) {
     const int nout = rows_needed(to, level - l, TAPS);
+    float* dst = (l & 1) ? Y : X;
+    const float* src = (l & 1) ? X : Y;  // fp32 input of levels >= 2
     for (int e = tid; e < nout * DS; e += NTH) {
       const int j = e / DS, c = e % DS;
-      const float* x = src + (2 * j) * DS + c;
+      float x[TAPS];
+      if (l == 1) {
+#pragma unroll
+        for (int k = 0; k < TAPS; ++k) x[k] = rd(X0 + (2 * j + k) * DS + c);
+      } else {
+#pragma unroll
+        for (int k = 0; k < TAPS; ++k) x[k] = src[(2 * j + k) * DS + c];
+      }
       float v;
       if (TAPS == 2) {
-        v = __fmul_rn(__fadd_rn(x[0], x[DS]), c32);
+        v = __fmul_rn(__fadd_rn(x[0], x[1]), c32);
       } else {
         v = __fmul_rn(taps.h[0], x[0]);
 #pragma unroll
-        for (int k = 1; k < TAPS; ++k) v = __fadd_rn(v, __fmul_rn(taps.h[k], x[k * DS]));
+        for (int k = 1; k < TAPS; ++k) v = __fadd_rn(v, __fmul_rn(taps.h[k], x[k]));
       }
       dst[j * DS + c] = v;
     }
     __syncthreads();
-    float* t = src;
-    src = dst;
-    dst = t;
   }
 
   // The last level: rows j0 .. j0 + to - 1 (those below m), rounded to T.
+  const float* fin = (level & 1) ? Y : X;
   T* ob = out + (int64_t)u * out_unit + c0;
   for (int e = tid; e < to * DS; e += NTH) {
     const int j = e / DS, c = e % DS;
-    if (j0 + j < m) from_f32(ob[(int64_t)(j0 + j) * out_row + c], src[j * DS + c]);
+    if (j0 + j < m) from_f32(ob[(int64_t)(j0 + j) * out_row + c], fin[j * DS + c]);
   }
 }
 
+// Shared memory of one CTA for DS channels: the raw rows, then the first
+// fp32 level (the raw buffer holds the later ones).
+template <typename T, int TAPS>
+size_t approx_smem(int level, int ds) {
+  const int nin = rows_needed(outputs_per_cta(level), level, TAPS);
+  return (size_t)nin * ds * sizeof(T) + sizeof(float) * ds * (size_t)(nin / 2 + 1);
+}
+
+template <typename T, int TAPS, int DS>
+cudaError_t run_ds(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m, int level,
+                   const Taps& taps, void* out, int64_t out_unit, cudaStream_t s) {
+  const int to = outputs_per_cta(level);
+  const size_t smem = approx_smem<T, TAPS>(level, DS);
+  cudaError_t e =
+      cudaFuncSetAttribute(approx_kernel<T, TAPS, DS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads), (unsigned)(kv.head_dim / DS));
+  approx_kernel<T, TAPS, DS><<<grid, NTH, smem, s>>>(static_cast<const T*>(K), kv.stride_b, kv.stride_h,
+                                                     kv.stride_s, kv.seq, kv.heads, cand, cand_stride, m, level, taps,
+                                                     static_cast<T*>(out), out_unit, kv.head_dim);
+  return cudaGetLastError();
+}
+
+// 64 channels per CTA (whole 128-byte lines of bf16) while the shared memory
+// allows, else 16 (the deepest scales).
 template <typename T, int TAPS>
 cudaError_t run(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m, int level,
                 const Taps& taps, void* out, int64_t out_unit, cudaStream_t s) {
-  const int to = outputs_per_cta(level);
-  const int nin = rows_needed(to, level, TAPS);
-  const size_t smem = sizeof(float) * DS * (size_t)(nin + nin / 2 + 1);
-  cudaError_t e = cudaFuncSetAttribute(approx_kernel<T, TAPS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  const dim3 grid((unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads), (unsigned)(kv.head_dim / DS));
-  approx_kernel<T, TAPS><<<grid, NTH, smem, s>>>(static_cast<const T*>(K), kv.stride_b, kv.stride_h, kv.stride_s,
-                                                 kv.seq, kv.heads, cand, cand_stride, m, level, taps,
-                                                 static_cast<T*>(out),
-                                                 out_unit, kv.head_dim);
-  return cudaGetLastError();
+  if (approx_smem<T, TAPS>(level, 64) <= 200 * 1024)
+    return run_ds<T, TAPS, 64>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+  return run_ds<T, TAPS, 16>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
 }
 
 }  // namespace
