@@ -195,24 +195,52 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   const float* w = W + (int64_t)u * w_unit;
   uint32_t prefix = 0, mask = 0;
   uint32_t need = (uint32_t)kk;
+  const int lane = tid & 31;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
     if (tid < 256) hist[tid] = 0;
     __syncthreads();
-    for (int j = tid; j < m; j += blockDim.x) {
-      const uint32_t key = order_key(w[j]);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    // Keys crowd into few bins (sign and exponent bits first): the lanes of a
+    // warp that share a bin add their count with one atomic.
+    for (int base = 0; base < m; base += blockDim.x) {
+      const int j = base + tid;
+      const uint32_t key = j < m ? order_key(w[j]) : 0u;
+      const bool in = j < m && (key & mask) == prefix;
+      const unsigned act = __ballot_sync(0xffffffffu, in);
+      if (in) {
+        const uint32_t bin = (key >> shift) & 255u;
+        const unsigned peers = __match_any_sync(act, bin);
+        if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], (uint32_t)__popc(peers));
+      }
     }
     __syncthreads();
-    if (tid == 0) {
-      uint32_t cum = 0;
-      int sel = 0;
-      for (int bin = 255; bin >= 0; --bin) {
-        if (cum + hist[bin] >= need) { sel = bin; break; }
-        cum += hist[bin];
+    if (tid < 32) {
+      // Warp 0: bins high to low, eight per lane; the lane whose run reaches
+      // `need` picks the bin.
+      uint32_t c[8], run = 0;
+#pragma unroll
+      for (int b = 0; b < 8; ++b) {
+        c[b] = hist[255 - (lane * 8 + b)];
+        run += c[b];
       }
-      s_need = need - cum;
-      s_prefix = prefix | ((uint32_t)sel << shift);
+      uint32_t incl = run;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      uint32_t cum = incl - run;  // keys in higher bins than this lane's
+      const bool mine = cum < need && incl >= need;
+      if (mine) {
+        int sel = 0;
+#pragma unroll 1
+        for (int b = 0; b < 8; ++b) {
+          if (cum + c[b] >= need) { sel = 255 - (lane * 8 + b); break; }
+          cum += c[b];
+        }
+        s_need = need - cum;
+        s_prefix = prefix | ((uint32_t)sel << shift);
+      }
     }
     __syncthreads();
     prefix = s_prefix;

@@ -79,31 +79,52 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
 
+  // The cascade: a thread owns a channel pair and a run of consecutive
+  // outputs, sliding its filter window two rows per output (each output is
+  // the same fp32 sequence of products and sums).
   const float c32 = 0.70710678118654752440f;  // fl32(1 / sqrt 2)
+  constexpr int PAIRS = DS / 2;
+  constexpr int GROUPS = NTH / PAIRS;
+  const int cp = tid % PAIRS, grp = tid / PAIRS;
 #pragma unroll 1
   for (int l = 1; l <= level; ++l) {
     const int nout = rows_needed(to, level - l, TAPS);
     float* dst = (l & 1) ? Y : X;
     const float* src = (l & 1) ? X : Y;  // fp32 input of levels >= 2
-    for (int e = tid; e < nout * DS; e += NTH) {
-      const int j = e / DS, c = e % DS;
-      float x[TAPS];
+    const int per = (nout + GROUPS - 1) / GROUPS;
+    const int jb = grp * per, je = min(nout, jb + per);
+    auto in = [&](int row) -> float2 {
       if (l == 1) {
-#pragma unroll
-        for (int k = 0; k < TAPS; ++k) x[k] = rd(X0 + (2 * j + k) * DS + c);
-      } else {
-#pragma unroll
-        for (int k = 0; k < TAPS; ++k) x[k] = src[(2 * j + k) * DS + c];
+        const T* p = X0 + row * DS + 2 * cp;
+        return make_float2(rd(p), rd(p + 1));
       }
-      float v;
-      if (TAPS == 2) {
-        v = __fmul_rn(__fadd_rn(x[0], x[1]), c32);
-      } else {
-        v = __fmul_rn(taps.h[0], x[0]);
+      return *reinterpret_cast<const float2*>(src + row * DS + 2 * cp);
+    };
+    if (jb < je) {
+      float2 x[TAPS];
 #pragma unroll
-        for (int k = 1; k < TAPS; ++k) v = __fadd_rn(v, __fmul_rn(taps.h[k], x[k]));
+      for (int k = 0; k < TAPS - 2; ++k) x[k + 2] = in(2 * jb + k);
+#pragma unroll 1
+      for (int j = jb; j < je; ++j) {
+#pragma unroll
+        for (int k = 0; k < TAPS - 2; ++k) x[k] = x[k + 2];
+        x[TAPS - 2] = in(2 * j + TAPS - 2);
+        x[TAPS - 1] = in(2 * j + TAPS - 1);
+        float2 v;
+        if (TAPS == 2) {
+          v.x = __fmul_rn(__fadd_rn(x[0].x, x[1].x), c32);
+          v.y = __fmul_rn(__fadd_rn(x[0].y, x[1].y), c32);
+        } else {
+          v.x = __fmul_rn(taps.h[0], x[0].x);
+          v.y = __fmul_rn(taps.h[0], x[0].y);
+#pragma unroll
+          for (int k = 1; k < TAPS; ++k) {
+            v.x = __fadd_rn(v.x, __fmul_rn(taps.h[k], x[k].x));
+            v.y = __fadd_rn(v.y, __fmul_rn(taps.h[k], x[k].y));
+          }
+        }
+        *reinterpret_cast<float2*>(dst + j * DS + 2 * cp) = v;
       }
-      dst[j * DS + c] = v;
     }
     __syncthreads();
   }
