@@ -193,8 +193,9 @@ wf_status wf_filter(const void* Q, const wf_tensor* q, const void* coeffs, const
  *   WF_WAVELET_DB2:  Daubechies' filter with two vanishing moments,
  *                    h = (1 + r, 3 + r, 3 - r, 1 - r) / (4 sqrt 2), r = sqrt 3.
  * Arithmetic: an fp32 cascade (Haar: fl32(x0 + x1) * fl32(1 / sqrt 2), the
- * rule of wf_dwt_build; db2: the products fl32(fl32(h[k]) x) added left to
- * right, no fused multiply-add), the last level rounded to the key dtype.
+ * rule of wf_dwt_build; db2: fl32(fl32(h[0]) x0), then fused multiply-adds
+ * with fl32(h[1]), fl32(h[2]), fl32(h[3]) in that order), the last level
+ * rounded to the key dtype.
  *
  * wf_wavelet_approx: the level-`level` rows of the keys of blocks
  * [2^level c, 2^level (c + 1)) for the m candidates c of every unit.

@@ -529,10 +529,7 @@ int orc_wavelet_approx_spec32(const float* x, int64_t len, int d, int wavelet, i
           v = s * c32;
         } else {
           v = h32[0] * prev[((2 * j) % n) * d + c];
-          for (int k = 1; k < taps; ++k) {
-            const float t = h32[k] * prev[((2 * j + k) % n) * d + c];
-            v = v + t;
-          }
+          for (int k = 1; k < taps; ++k) v = fmaf(h32[k], prev[((2 * j + k) % n) * d + c], v);
         }
         cur[j * d + c] = v;
       }

@@ -113,10 +113,10 @@ int orc_wavelet_synthesis_f64(const double* A, const double* D, int64_t n, int d
 
 /* Level-`level` approximation rows (len >> level of them) of the periodized
  * transform of x under the library's storage rule: an fp32 cascade (Haar:
- * fl32(x0 + x1) * fl32(1 / sqrt 2), as the stored pyramid; other bases: the
- * products fl32(fl32(h[k]) * x) added left to right in fp32, no fused
- * multiply-add), only the last level rounded (bfloat16, nearest even, when
- * store_bf16; returned widened to float). */
+ * fl32(x0 + x1) * fl32(1 / sqrt 2), as the stored pyramid; other bases:
+ * fl32(fl32(h[0]) x0), then fmaf(fl32(h[k]), x_k, acc) for k = 1.. in order,
+ * each fused multiply-add rounded once), only the last level rounded
+ * (bfloat16, nearest even, when store_bf16; returned widened to float). */
 int orc_wavelet_approx_spec32(const float* x, int64_t len, int d, int wavelet, int level, int store_bf16,
                               float* out);
 

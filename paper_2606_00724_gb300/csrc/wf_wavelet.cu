@@ -53,12 +53,14 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   T* X0 = reinterpret_cast<T*>(sbuf);                                    // [nin][DS] raw
   float* Y = reinterpret_cast<float*>(sbuf + (size_t)nin * DS * sizeof(T));  // [nin / 2 + 1][DS]
   float* X = reinterpret_cast<float*>(sbuf);                             // fp32 levels >= 2
-  const int u = blockIdx.y;
-  const int j0 = blockIdx.x * to;
-  const int c0 = blockIdx.z * DS;
+  // The channel slice varies fastest, so the slices of the same rows are read
+  // by neighbouring CTAs at about the same time.
+  const int u = blockIdx.z;
+  const int j0 = blockIdx.y * to;
+  const int c0 = blockIdx.x * DS;
   const int64_t bb = u / H, hh = u % H;
-  const int64_t len = (int64_t)m << level;
-  const int64_t blk_mask = ((int64_t)1 << level) - 1;
+  const int len = m << level;  // the gathered sequence (< 2^31 tokens)
+  const int blk_mask = (1 << level) - 1;
   const T* kb = K + bb * ksb + hh * ksh + c0;
   const int32_t* cd = cand ? cand + (int64_t)u * cand_stride : nullptr;
   const int tid = threadIdx.x;
@@ -67,9 +69,11 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   constexpr int VEC = Vec<T>::N;
   constexpr int VPR = DS / VEC;  // 16-byte vectors per row
   const uint32_t xs = (uint32_t)__cvta_generic_to_shared(X0);
+  const int base = (int)(((int64_t)j0 << level) % len);
   for (int e = tid; e < nin * VPR; e += NTH) {
     const int r = e / VPR, v = e % VPR;
-    const int64_t p = (((int64_t)j0 << level) + r) % len;
+    int p = base + r;
+    if (p >= len) p = p - len < len ? p - len : p % len;  // the filter's reach wraps around
     int64_t tok = cd ? (((int64_t)cd[p >> level]) << level) + (p & blk_mask) : p;
     tok = tok < 0 ? 0 : (tok >= n ? n - 1 : tok);  // out-of-range block indices are clamped
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(xs + (uint32_t)((r * DS + v * VEC) * sizeof(T))),
@@ -119,8 +123,8 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
           v.y = __fmul_rn(taps.h[0], x[0].y);
 #pragma unroll
           for (int k = 1; k < TAPS; ++k) {
-            v.x = __fadd_rn(v.x, __fmul_rn(taps.h[k], x[k].x));
-            v.y = __fadd_rn(v.y, __fmul_rn(taps.h[k], x[k].y));
+            v.x = __fmaf_rn(taps.h[k], x[k].x, v.x);
+            v.y = __fmaf_rn(taps.h[k], x[k].y, v.y);
           }
         }
         *reinterpret_cast<float2*>(dst + j * DS + 2 * cp) = v;
@@ -154,7 +158,7 @@ cudaError_t run_ds(const void* K, const wf_tensor& kv, const int32_t* cand, int6
   cudaError_t e =
       cudaFuncSetAttribute(approx_kernel<T, TAPS, DS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  const dim3 grid((unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads), (unsigned)(kv.head_dim / DS));
+  const dim3 grid((unsigned)(kv.head_dim / DS), (unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads));
   approx_kernel<T, TAPS, DS><<<grid, NTH, smem, s>>>(static_cast<const T*>(K), kv.stride_b, kv.stride_h,
                                                      kv.stride_s, kv.seq, kv.heads, cand, cand_stride, m, level, taps,
                                                      static_cast<T*>(out), out_unit, kv.head_dim);
