@@ -1214,25 +1214,38 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
     tmax = tmax > ta ? tmax : ta;
     return 32 * tmax;
   };
-  // Two units per cluster (copies of one overlap the other's exchanges and
-  // Top-K) unless that leaves most SMs idle; the largest cluster that still
-  // fits the grid in one wave.
-  const int P = (U >= 2 && U * MAXCS > num_sms) ? 2 : 1;
-  const int clusters = (U + P - 1) / P;
   const size_t kMaxSmem = 227 * 1024;
-  int stages = 4;
-  if (smem_layout(4, P, cmax, kmax).total > kMaxSmem) stages = 3;
-  const size_t smem = smem_layout(stages, P, cmax, kmax).total;
-  if (smem > kMaxSmem) return fp;
-  // The largest cluster (any size up to 8) whose grid fits the SMs in one
-  // wave, all clusters resident at once, and whose slices fit TMEM; else the
-  // smallest one that fits TMEM.
-  int cs = 0;
-  for (int c = MAXCS; c >= 1 && cs == 0; --c)
-    if (clusters * c <= num_sms && P * unit_cols(c) <= 512 && clusters <= max_active_clusters(stages, c, smem)) cs = c;
-  for (int c = 1; c <= MAXCS && cs == 0; ++c)
-    if (P * unit_cols(c) <= 512) cs = c;
-  if (cs == 0) return fp;
+  // For P units per cluster (1, or 2 so that one unit's copies overlap the
+  // other's exchanges and Top-K): the largest cluster (any size up to 8)
+  // whose grid fits the SMs in one wave, all clusters resident at once, and
+  // whose slices fit TMEM; else the smallest one that fits TMEM.
+  struct Choice {
+    int P, cs, stages;
+    size_t smem;
+  };
+  auto choose = [&](int P) {
+    Choice ch{P, 0, 4, 0};
+    const int clusters = (U + P - 1) / P;
+    if (smem_layout(4, P, cmax, kmax).total > kMaxSmem) ch.stages = 3;
+    ch.smem = smem_layout(ch.stages, P, cmax, kmax).total;
+    if (ch.smem > kMaxSmem) return ch;
+    for (int c = MAXCS; c >= 1 && ch.cs == 0; --c)
+      if (clusters * c <= num_sms && P * unit_cols(c) <= 512 && clusters <= max_active_clusters(ch.stages, c, ch.smem))
+        ch.cs = c;
+    for (int c = 1; c <= MAXCS && ch.cs == 0; ++c)
+      if (P * unit_cols(c) <= 512) ch.cs = c;
+    return ch;
+  };
+  // Units per SM (P / cs) set each SM's share of the rows: take the smaller,
+  // two units per cluster on a tie.
+  const Choice c2 = U >= 2 ? choose(2) : Choice{2, 0, 4, 0};
+  const Choice c1 = choose(1);
+  Choice best = c2;
+  if (c2.cs == 0 || (c1.cs > 0 && 1 * c2.cs < 2 * c1.cs)) best = c1;
+  if (best.cs == 0) return fp;
+  const int P = best.P, cs = best.cs, stages = best.stages;
+  const size_t smem = best.smem;
+  const int clusters = (U + P - 1) / P;
   const int ucols = unit_cols(cs);
   int cols = 32;
   while (cols < P * ucols) cols *= 2;
