@@ -214,6 +214,27 @@ def oracle_units_seconds(w: synth.Workload, cfg: str, budget_s: float, max_units
 
 
 # ---------------------------------------------------------------------------
+# Multi-rank aggregation (one replica per rank, weak scaling).
+# ---------------------------------------------------------------------------
+def max_over_ranks(values, device):
+    """Each value's MAX over the ranks of the default process group (the
+    values themselves on a single rank)."""
+    dist = torch.distributed
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t]
+
+
+def aggregate(world: int, step_bytes: float, total_ms: float, steps: int):
+    """(ms per step, whole-job GB/s): every rank moves step_bytes per step and
+    the slowest rank's time counts."""
+    ms_per_step = total_ms / steps
+    return ms_per_step, world * step_bytes / (ms_per_step * 1e-3) / 1e9
+
+
+# ---------------------------------------------------------------------------
 # GPU arm.
 # ---------------------------------------------------------------------------
 def make_inputs(w, cfg, device, rank):
@@ -482,12 +503,8 @@ def main():
     r = run_gpu(args, cfg, rank, world, device)
     total_ms = r["total_ms"]
     e2e_ms = r["e2e_ms"]
-    if world > 1:
-        t = torch.tensor([total_ms, e2e_ms], device=device, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms, e2e_ms = float(t[0]), float(t[1])
-    ms_per_step = total_ms / args.steps
-    value = world * step_bytes / (ms_per_step * 1e-3) / 1e9
+    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], device)
+    ms_per_step, value = aggregate(world, step_bytes, total_ms, args.steps)
 
     # Roofline of the dominant kernel: the fused step kernel is the only kernel
     # of a step (one launch per layer), so its algorithmic bytes per launch are
@@ -508,7 +525,7 @@ def main():
     line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "step_us": ms_per_step * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "bf16" if fused_eligible(w) else "f32",
+            "dtype": "bf16" if (w.dtype == "bf16" and w.head_dim == 128) else "f32",
             "data": "synthetic", "config": config, "roofline": roofline, "clocks": r["clocks"],
             "e2e": {"value": world * e2e_bytes_per_step / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                     "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"], "ms_per_step": e2e_ms,
