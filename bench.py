@@ -518,6 +518,7 @@ def main():
         "per-stage kernels (approx/score/weights/select/attn)" if WAVELET else
         "per-stage kernels (score/weights/select/attn)")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                "frac_of_nominal_7900": achieved / 7900.0,
                 "traffic": recorded_traffic(w) if fused_eligible(w) else None, "kernel": kname,
                 "peak_kind": peak_kind,
                 "bytes_per_launch": ub["step"] * w.units, "launch_us": per_layer_ms * 1e3}
