@@ -14,6 +14,12 @@
  *   4. attention of the query block over [K[mu^0]; K[I_g]], [V[mu^0]; V[I_g]]
  *      (Algorithm 1, final step)                             -> wf_sparse_attn
  * and wf_step runs 1 (optionally) + 2-3 + 4 as one stream-ordered call.
+ * Around them: wf_cache_update (new rows into the caches with the touched
+ * pyramid blocks refreshed), the kept-count schedules (wf_default_schedule,
+ * wf_level0_schedule, wf_schedule_from_proportions), other wavelet bases
+ * with Eq. 11 taken literally (wf_wavelet_approx, wf_filter_wavelet), grouped
+ * query heads (wf_filter, wf_sparse_attn, wf_step), and
+ * wf_sparse_attn_noalloc for callers that cannot pass a workspace.
  *
  * Conventions shared by every entry point
  * - A tensor is described by wf_tensor: [batch, heads, seq, head_dim] with
@@ -27,10 +33,12 @@
  *   outputs are valid once the stream reaches that point.
  * - Every argument is checked on the host before anything is launched; a
  *   failed check returns a negative wf_status and enqueues nothing.  A failed
- *   launch returns WF_ERR_CUDA.  The only device-side waits (in wf_step's
- *   fused kernel) are bounded, so no call can hang the device.
+ *   launch returns WF_ERR_CUDA.  Every device-side wait (the fused kernel's
+ *   and the tensor-core kernels') is bounded, so no call can hang the device;
+ *   a wait that gives up sets the status word read by wf_workspace_status.
  * - Supported: dtype WF_F32 or WF_BF16 (Q, K, V, Kg, Vg, coeffs and O all of
- *   the same dtype); head_dim 64 or 128; 1 <= query rows <= 64; prompt length
+ *   the same dtype); head_dim 64 or 128; 1 <= query rows <= 64 per query head
+ *   (at most 256 per key head when query heads are grouped); prompt length
  *   n a multiple of 2^levels with 1 <= levels <= 10; base pointers and the
  *   three strides (in bytes) 16-byte aligned.
  */
