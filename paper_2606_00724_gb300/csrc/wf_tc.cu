@@ -12,8 +12,9 @@
 // rows are read twice (the second time mostly from L2) and no logit matrix
 // goes through memory.
 //
-// One CTA (four warps, one TMEM lane quarter each) per (tile, unit): all
-// threads gather the tile (16-byte cp.async into the 128-byte-swizzled
+// One CTA of two warpgroups per (tile, unit); each warpgroup covers the 128
+// TMEM lanes (a warp per lane quarter) and takes every other 32-column chunk
+// of the query columns.  All threads gather the tile (16-byte cp.async into the 128-byte-swizzled
 // K-major layout) and the query block (cp.async into K-major core matrices,
 // zero rows up to a multiple of 32), one thread issues the eight MMAs (K = 128) into TMEM
 // and commits them to an mbarrier, and every thread reads back its
@@ -32,7 +33,8 @@ using namespace sm100;
 
 constexpr int D = 128;
 constexpr int TM = 128;                // candidate rows per tile (MMA M)
-constexpr int NTH = 128;               // threads per CTA
+constexpr int NTH = 256;               // threads per CTA: two warpgroups
+constexpr int NWG = NTH / 128;         // warpgroups; each covers all 128 TMEM lanes
 constexpr int HALF = TM * 128;         // one 64-column half of the tile
 constexpr int QGRP = (D / 8) * 128;    // bytes per 8-row group of the query block
 constexpr long long kWait = 1ll << 31;
@@ -73,6 +75,9 @@ __global__ void __launch_bounds__(256) norm_kernel(const float2* __restrict__ pa
   cvec[(int64_t)u * q + i] = M + lg2(S);
 }
 
+// Barrier of one warpgroup (named barriers 1, 2).
+__device__ __forceinline__ void wg_sync(int wg) { asm volatile("bar.sync %0, 128;" ::"r"(1 + wg) : "memory"); }
+
 // Lane l of the warp ends with the reduction of column l over the warp's 32
 // lanes (31 shuffles).
 template <bool MAX>
@@ -96,11 +101,13 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* tile = smem;                        // 2 x HALF, 1024-aligned
   uint8_t* sq = smem + 2 * HALF;               // nq / 8 groups of QGRP
-  float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [4][32]
-  float* col = red + 4 * 32;                   // [256]: per-column max, or the normalisers c_i
-  unsigned long long* bar = reinterpret_cast<unsigned long long*>(col + 256);
+  float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [NWG][4][32]
+  float* col = red + NWG * 4 * 32;             // [256]: per-warpgroup column maxima ([NWG][32]), or the c_i
+  float2* xch = reinterpret_cast<float2*>(col + 256);  // [128]: the second warpgroup's (max, sum) per row
+  unsigned long long* bar = reinterpret_cast<unsigned long long*>(xch + 128);
   uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 1);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int wg = tid >> 7, wt = tid & 127, quarter = warp & 3;
   const int t = blockIdx.x, u = blockIdx.y;
   const int64_t bb = u / a.H, hh = u % a.H;
 
@@ -112,15 +119,15 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
     mbar_init(smem_u32(bar), 1);
     fence_mbar_init();
   }
-  // The tile: chunk c = tid % 16 of rows tid / 16 + 8 i, 128-byte swizzle.
+  // The tile: chunk c = tid % 16 of rows tid / 16 + 16 i, 128-byte swizzle.
   {
     const int c = tid & 15;
     const bf16* rb = static_cast<const bf16*>(a.src.base) + bb * a.src.sb + hh * a.src.sh + a.src.off;
     const int32_t* cd = a.cand ? a.cand + (int64_t)u * a.cand_stride : nullptr;
     const uint32_t cbase = smem_u32(tile) + ((c >> 3) * HALF);
 #pragma unroll 4
-    for (int i = 0; i < TM / 8; ++i) {
-      const int r = (tid >> 4) + 8 * i;
+    for (int i = 0; i < TM / (NTH / 16); ++i) {
+      const int r = (tid >> 4) + (NTH / 16) * i;
       const int j = min(t * TM + r, a.m - 1);  // rows past the list repeat its last row (finite, masked)
       const int64_t row = cd ? (int64_t)cd[j] : (int64_t)j;
       cp_async16(cbase + r * 128 + (((c & 7) ^ (r & 7)) << 4), rb + row * a.src.ss + c * 8);
@@ -163,14 +170,18 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
   ok = __syncthreads_and(ok);
   tc_fence_after();
 
-  const int j = t * TM + tid;  // this thread's candidate (TMEM lane tid)
+  // Thread wt of either warpgroup owns candidate j (TMEM lane wt); the two
+  // warpgroups take alternate 32-column chunks.
+  const int j = t * TM + wt;
   const bool valid = j < a.m;
-  const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+  const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
   const int nch = a.nq / 32;
+  float* rw = red + wg * 4 * 32;
+  float* cw = col + wg * 32;
   if (ok && MODE == 0) {
     float2* pt = a.part + (int64_t)u * a.part_unit + (int64_t)t * a.q;
 #pragma unroll 1
-    for (int ch = 0; ch < nch; ++ch) {
+    for (int ch = wg; ch < nch; ch += NWG) {
       float v[32], w[32];
       tmem_ld32(lane_base + 32 * ch, v);
 #pragma unroll
@@ -178,17 +189,17 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
         v[i] = valid ? v[i] * a.sl2 : -INFINITY;
         w[i] = v[i];
       }
-      red[warp * 32 + lane] = xpose_reduce32<true>(w, lane);
-      __syncthreads();
-      if (tid < 32) col[tid] = fmaxf(fmaxf(red[tid], red[32 + tid]), fmaxf(red[64 + tid], red[96 + tid]));
-      __syncthreads();
+      rw[quarter * 32 + lane] = xpose_reduce32<true>(w, lane);
+      wg_sync(wg);
+      if (wt < 32) cw[wt] = fmaxf(fmaxf(rw[wt], rw[32 + wt]), fmaxf(rw[64 + wt], rw[96 + wt]));
+      wg_sync(wg);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) w[i] = valid ? ex2(v[i] - col[i]) : 0.f;
-      red[warp * 32 + lane] = xpose_reduce32<false>(w, lane);
-      __syncthreads();
-      if (tid < 32 && ch * 32 + tid < a.q)
-        pt[ch * 32 + tid] = make_float2(col[tid], (red[tid] + red[32 + tid]) + (red[64 + tid] + red[96 + tid]));
-      __syncthreads();
+      for (int i = 0; i < 32; ++i) w[i] = valid ? ex2(v[i] - cw[i]) : 0.f;
+      rw[quarter * 32 + lane] = xpose_reduce32<false>(w, lane);
+      wg_sync(wg);
+      if (wt < 32 && ch * 32 + wt < a.q)
+        pt[ch * 32 + wt] = make_float2(cw[wt], (rw[wt] + rw[32 + wt]) + (rw[64 + wt] + rw[96 + wt]));
+      wg_sync(wg);
     }
   }
   if (ok && MODE == 1) {
@@ -197,7 +208,7 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
     __syncthreads();
     float mx = -INFINITY;
 #pragma unroll 1
-    for (int ch = 0; ch < nch; ++ch) {
+    for (int ch = wg; ch < nch; ch += NWG) {
       float v[32];
       tmem_ld32(lane_base + 32 * ch, v);
 #pragma unroll
@@ -206,14 +217,22 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
     }
     float z = 0.f;
 #pragma unroll 1
-    for (int ch = 0; ch < nch; ++ch) {
+    for (int ch = wg; ch < nch; ch += NWG) {
       float v[32];
       tmem_ld32(lane_base + 32 * ch, v);
 #pragma unroll
       for (int i = 0; i < 32; ++i)
         if (ch * 32 + i < a.q) z += ex2(fmaf(v[i], a.sl2, -col[ch * 32 + i]) - mx);
     }
-    if (valid) a.W[(int64_t)u * a.w_unit + j] = mx + lg2(z);
+    // Fold the second warpgroup's (max, sum) of the row into the first's.
+    if (wg == 1) xch[wt] = make_float2(mx, z);
+    __syncthreads();
+    if (wg == 0) {
+      const float2 o = xch[wt];
+      const float M = fmaxf(mx, o.x);
+      const float Z = (z > 0.f ? z * ex2(mx - M) : 0.f) + (o.y > 0.f ? o.y * ex2(o.x - M) : 0.f);
+      if (valid) a.W[(int64_t)u * a.w_unit + j] = M + lg2(Z);
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -251,11 +270,11 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
   // Shared memory: the tile, the query block, the reductions, the barrier.
   // At most 512 / cols CTAs may share an SM (TMEM); the request is padded so
   // that shared memory enforces it.
-  size_t smem = 2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (4 * 32 + 256) + 16;
+  size_t smem = 2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 256) + sizeof(float2) * 128 + 16;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;  // CTAs per SM the TMEM allows
   const size_t floor_smem = per_sm / (cap + 1) + 1;
-  if (cap < 16 && smem < floor_smem) smem = floor_smem;
+  if (cap < (size_t)(2048 / NTH) && smem < floor_smem) smem = floor_smem;
   const dim3 grid((unsigned)((m + TM - 1) / TM), (unsigned)p.U);
   cudaError_t e = cudaFuncSetAttribute(tc_score_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e == cudaSuccess)
@@ -315,12 +334,13 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   uint8_t* vt = smem + 2 * HALF;               // V tile, 2 x HALF
   uint8_t* sq = smem + 4 * HALF;               // query block, nq / 8 groups of QGRP
   uint8_t* pb = sq + (a.nq / 8) * QGRP;        // P^T: 16 key groups of nq * 16 bytes
-  float* red = reinterpret_cast<float*>(pb + a.nq * 256);  // [4][32]
-  float* cm = red + 4 * 32;                    // [256] split max per query (log2 units)
+  float* red = reinterpret_cast<float*>(pb + a.nq * 256);  // [NWG][4][32]
+  float* cm = red + NWG * 4 * 32;              // [256] split max per query (log2 units)
   float* cl = cm + 256;                        // [256] split row sums of P
   unsigned long long* bar = reinterpret_cast<unsigned long long*>(cl + 256);  // [2]
   uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 2);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int wg = tid >> 7, wt = tid & 127, quarter = warp & 3;
   const int sp = blockIdx.x, u = blockIdx.y;
   const int64_t bb = u / a.H, hh = u % a.H;
   const int total = a.k + a.ng, t0 = sp * TM;
@@ -334,14 +354,14 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     mbar_init(smem_u32(&bar[1]), 1);
     fence_mbar_init();
   }
-  // K and V rows of the split: chunk c = tid % 16 of rows tid / 16 + 8 i.
+  // K and V rows of the split: chunk c = tid % 16 of rows tid / 16 + 16 i.
   {
     const int c = tid & 15;
     const int32_t* ui = a.idx + (int64_t)u * a.k;
     const uint32_t koff = smem_u32(kt) + ((c >> 3) * HALF), voff = smem_u32(vt) + ((c >> 3) * HALF);
 #pragma unroll 4
-    for (int i = 0; i < TM / 8; ++i) {
-      const int r = (tid >> 4) + 8 * i;
+    for (int i = 0; i < TM / (NTH / 16); ++i) {
+      const int r = (tid >> 4) + (NTH / 16) * i;
       const int tt = min(t0 + r, total - 1);  // keys past the list repeat its last key (P = 0 there)
       const bf16 *kp, *vp;
       if (tt < a.k) {
@@ -397,24 +417,27 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   ok = __syncthreads_and(ok);
   tc_fence_after();
 
-  const bool valid = t0 + tid < total;  // this thread's key (TMEM lane tid)
-  const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+  // Thread wt of either warpgroup owns key t0 + wt (TMEM lane wt); the two
+  // warpgroups take alternate 32-column chunks.
+  const bool valid = t0 + wt < total;
+  const uint32_t qoff = (uint32_t)(quarter * 32) << 16;
   const int nch = a.nq / 32;
+  float* rw = red + wg * 4 * 32;
   if (ok) {
-    uint8_t* prow = pb + (tid >> 3) * (a.nq * 16) + (tid & 7) * 16;
+    uint8_t* prow = pb + (wt >> 3) * (a.nq * 16) + (wt & 7) * 16;
 #pragma unroll 1
-    for (int ch = 0; ch < nch; ++ch) {
+    for (int ch = wg; ch < nch; ch += NWG) {
       float v[32], w[32];
-      tmem_ld32(lane_base + 32 * ch, v);
+      tmem_ld32(tmem + qoff + 32 * ch, v);
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         v[i] = valid ? v[i] * a.sl2 : -INFINITY;
         w[i] = v[i];
       }
-      red[warp * 32 + lane] = xpose_reduce32<true>(w, lane);
-      __syncthreads();
-      if (tid < 32) cm[ch * 32 + tid] = fmaxf(fmaxf(red[tid], red[32 + tid]), fmaxf(red[64 + tid], red[96 + tid]));
-      __syncthreads();
+      rw[quarter * 32 + lane] = xpose_reduce32<true>(w, lane);
+      wg_sync(wg);
+      if (wt < 32) cm[ch * 32 + wt] = fmaxf(fmaxf(rw[wt], rw[32 + wt]), fmaxf(rw[64 + wt], rw[96 + wt]));
+      wg_sync(wg);
       uint32_t pk[16];
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
@@ -429,10 +452,10 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
       for (int c4 = 0; c4 < 4; ++c4)
         *reinterpret_cast<uint4*>(prow + (ch * 4 + c4) * 128) =
             make_uint4(pk[4 * c4], pk[4 * c4 + 1], pk[4 * c4 + 2], pk[4 * c4 + 3]);
-      red[warp * 32 + lane] = xpose_reduce32<false>(w, lane);
-      __syncthreads();
-      if (tid < 32) cl[ch * 32 + tid] = (red[tid] + red[32 + tid]) + (red[64 + tid] + red[96 + tid]);
-      __syncthreads();
+      rw[quarter * 32 + lane] = xpose_reduce32<false>(w, lane);
+      wg_sync(wg);
+      if (wt < 32) cl[ch * 32 + wt] = (rw[wt] + rw[32 + wt]) + (rw[64 + wt] + rw[96 + wt]);
+      wg_sync(wg);
     }
     fence_proxy_async();
     tc_fence_before();
@@ -455,25 +478,25 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     ok2 = __syncthreads_and(ok2);
     tc_fence_after();
     if (ok2) {
-      // Thread tid holds head-dim row tid of O^T: query columns in chunks.
+      // Thread wt holds head-dim row wt of O^T: its warpgroup's query chunks.
       const float ln2 = 0.69314718055994531f;
 #pragma unroll 1
-      for (int ch = 0; ch < nch; ++ch) {
+      for (int ch = wg; ch < nch; ch += NWG) {
         float o[32];
-        tmem_ld32(ocol + ((uint32_t)(warp * 32) << 16) + 32 * ch, o);
+        tmem_ld32(ocol + qoff + 32 * ch, o);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const int col = ch * 32 + i;
-          if (col < a.q) {
-            const int64_t uq = bb * (a.H * a.G) + hh * a.G + col / a.qs;
-            const int iq = col % a.qs;
-            a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + tid] = o[i];
+          const int colq = ch * 32 + i;
+          if (colq < a.q) {
+            const int64_t uq = bb * (a.H * a.G) + hh * a.G + colq / a.qs;
+            const int iq = colq % a.qs;
+            a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + wt] = o[i];
           }
         }
       }
-      for (int col = tid; col < a.q; col += NTH) {
-        const int64_t uq = bb * (a.H * a.G) + hh * a.G + col / a.qs;
-        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + col % a.qs] = make_float2(cm[col] * ln2, cl[col]);
+      for (int colq = tid; colq < a.q; colq += NTH) {
+        const int64_t uq = bb * (a.H * a.G) + hh * a.G + colq / a.qs;
+        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq % a.qs] = make_float2(cm[colq] * ln2, cl[colq]);
       }
     }
   }
@@ -517,11 +540,11 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   a.qstride = kMaxQ;
   a.status = status;
   a.sl2 = 1.4426950408889634f * scale;
-  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + (size_t)a.nq * 256 + sizeof(float) * (4 * 32 + 512) + 32;
+  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + (size_t)a.nq * 256 + sizeof(float) * (NWG * 4 * 32 + 512) + 32;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;
   const size_t floor_smem = per_sm / (cap + 1) + 1;
-  if (cap < 16 && smem < floor_smem) smem = floor_smem;
+  if (cap < (size_t)(2048 / NTH) && smem < floor_smem) smem = floor_smem;
   cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   tc_attn_kernel<<<dim3((unsigned)a.nsplit, (unsigned)(kv.batch * kv.heads)), NTH, smem, s>>>(a);
