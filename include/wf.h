@@ -278,6 +278,9 @@ wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const
  *   calls whose kernels may overlap on the GPU (other streams, other host
  *   threads) race and corrupt each other's results.  Serialise them, e.g.
  *   on one stream.  No part of the array has to start at zero.
+ * - The status word of wf_sparse_attn's workspace lives in the static array
+ *   too, so this call cannot report a tensor-core wait that gave up (it
+ *   never should); use wf_sparse_attn where that report is needed.
  * ------------------------------------------------------------------------- */
 #define WF_NOALLOC_SCRATCH_BYTES (16u << 20)
 wf_status wf_sparse_attn_noalloc(const void* Q, const wf_tensor* q, const void* K, const void* V,
