@@ -317,14 +317,15 @@ def run_gpu(args, cfg, rank, world, device):
                          O=torch.empty_like(lay.Q)))
 
     def one(lay, bf, Q, Kg, Vg, refresh):
+        st = torch.cuda.current_stream()  # the capture stream while a graph is recorded
         if WAVELET:
             if refresh:
-                wf.wf_wavelet_approx(lay.K, w.levels, basis, bf["coeffs"], stream=stream)
-            wf.wf_filter_wavelet(Q, bf["coeffs"], lay.K, w.levels, keep, basis, bf["idx"], bf["ws"], stream=stream)
-            wf.wf_sparse_attn(Q, lay.K, lay.V, bf["idx"], w.k, Kg, Vg, bf["O"], bf["ws"], stream=stream)
+                wf.wf_wavelet_approx(lay.K, w.levels, basis, bf["coeffs"], stream=st)
+            wf.wf_filter_wavelet(Q, bf["coeffs"], lay.K, w.levels, keep, basis, bf["idx"], bf["ws"], stream=st)
+            wf.wf_sparse_attn(Q, lay.K, lay.V, bf["idx"], w.k, Kg, Vg, bf["O"], bf["ws"], stream=st)
         else:
             wf.wf_step(Q, lay.K, lay.V, Kg, Vg, bf["coeffs"], refresh, w.levels, keep, bf["idx"], bf["O"], bf["ws"],
-                       stream)
+                       st)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
     stream = torch.cuda.current_stream()
     refresh_every = w.refresh_every
@@ -337,6 +338,16 @@ def run_gpu(args, cfg, rank, world, device):
     for i in range(args.warmup):
         step(i)
     torch.cuda.synchronize()
+    if args.graph:
+        # One step's launches recorded once and replayed: the same kernels,
+        # without the host launch gaps between them.
+        if refresh_every:
+            raise SystemExit("bench.py: --graph takes workloads without a periodic refresh")
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            step(0)
+        torch.cuda.synchronize()
+        step = lambda i: graph.replay()  # noqa: E731
 
     # Pre-roll of the same steps so that the clock samples see the GPU under load.
     sampler = ClockSampler(device.index if device.index is not None else 0)
@@ -410,6 +421,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=None, help="override the workload's batch (small profiling cases)")
     ap.add_argument("--heads", type=int, default=None, help="override the workload's head count")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay each step from a CUDA graph recorded after the warm-up")
     ap.add_argument("--wavelet", default=None, choices=["haar", "db2"],
                     help="time the literal path for a generic basis (wf_filter_wavelet + wf_sparse_attn): the "
                          "transform of the gathered candidate blocks at every scale")
@@ -458,7 +471,8 @@ def main():
                        "wf_step (per-stage filter and sparse-attention kernels) per layer") + (
                   f"; wf_dwt_build refresh every {w.refresh_every} steps" if w.refresh_every else
                   ("; scale-L rows built once before timing" if WAVELET else "; pyramid built once before timing")),
-              "l2": "flushed before every timed step (256 MiB write)", "parallelism": f"replicas{args.gpus}"}
+              "l2": "flushed before every timed step (256 MiB write)", "parallelism": f"replicas{args.gpus}",
+              "cuda_graph": bool(args.graph)}
     step_bytes = ub["step"] * w.units * w.layers
     if w.refresh_every:
         step_bytes += ub["dwt"] * w.units * w.layers / w.refresh_every
