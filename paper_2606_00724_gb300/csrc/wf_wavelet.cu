@@ -23,7 +23,7 @@ namespace wf {
 namespace {
 
 constexpr int NTH = 256;      // threads per CTA
-constexpr int IN_ROWS = 256;  // gathered rows per CTA before the filter's reach
+constexpr int IN_ROWS = 128;  // gathered rows per CTA before the filter's reach
 
 // Output rows per CTA at scale `level`.
 __host__ __device__ inline int outputs_per_cta(int level) { return (IN_ROWS >> level) > 0 ? (IN_ROWS >> level) : 1; }
