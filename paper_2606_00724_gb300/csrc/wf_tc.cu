@@ -298,9 +298,12 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
 // 128-byte-swizzled tiles, S^T = K Q^T goes to TMEM (keys on the lanes, the
 // unit's query rows on the columns), every thread turns its key's row into
 // P = 2^(s - m) with m the split's per-query max (bf16, stored as P^T in
-// MN-major core matrices), and O^T = V^T P^T goes to TMEM.  The partial
-// (O, m, l) of every query row lands in the flash-decoding layout of the
-// fp32 kernels, per query head, so the same combine kernel finishes it.
+// MN-major core matrices over the dead K tile), and O^T = V^T P^T goes to
+// TMEM.  A key unit's query rows are cut into column blocks of at most 128
+// (grid z), so S^T and O^T fit 256 TMEM columns and two CTAs share an SM.
+// The partial (O, m, l) of every query row lands in the flash-decoding
+// layout of the fp32 kernels, per query head, so the same combine kernel
+// finishes it.
 // ---------------------------------------------------------------------------
 namespace wf {
 namespace {
@@ -318,7 +321,8 @@ struct TcAttnArgs {
   int64_t gsb, gsh, gss;
   const int32_t* idx;
   int n, k, ng, q, G, qs, H;  // q = G qs query rows per key unit; H key heads
-  int nq;                     // MMA columns (q rounded up to 32)
+  int cb;                     // query columns per CTA block (blockIdx.z = block)
+  int nq;                     // MMA columns of a block (its query rows rounded up to 32)
   uint32_t tcols;
   int nsplit;
   float* Opart;               // [query unit][nsplit][qstride][D]
@@ -333,8 +337,10 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   uint8_t* kt = smem;                          // K tile, 2 x HALF
   uint8_t* vt = smem + 2 * HALF;               // V tile, 2 x HALF
   uint8_t* sq = smem + 4 * HALF;               // query block, nq / 8 groups of QGRP
-  uint8_t* pb = sq + (a.nq / 8) * QGRP;        // P^T: 16 key groups of nq * 16 bytes
-  float* red = reinterpret_cast<float*>(pb + a.nq * 256);  // [NWG][4][32]
+  // P^T (16 key groups of nq * 16 bytes, nq <= 128) takes the K tile's place:
+  // the K rows are dead once the S^T products have completed.
+  uint8_t* pb = kt;
+  float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [NWG][4][32]
   float* cm = red + NWG * 4 * 32;              // [256] split max per query (log2 units)
   float* cl = cm + 256;                        // [256] split row sums of P
   unsigned long long* bar = reinterpret_cast<unsigned long long*>(cl + 256);  // [2]
@@ -344,6 +350,8 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   const int sp = blockIdx.x, u = blockIdx.y;
   const int64_t bb = u / a.H, hh = u % a.H;
   const int total = a.k + a.ng, t0 = sp * TM;
+  const int c0 = blockIdx.z * a.cb;           // first query row of this column block
+  const int qb = min(a.cb, a.q - c0);         // its query rows
 
   if (warp == 0) {
     tmem_alloc(smem_u32(tbase), a.tcols);
@@ -384,8 +392,9 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
     const int i = g * 8 + rr;
     const uint32_t dst = smem_u32(sq + g * QGRP + ch * 128 + rr * 16);
-    if (i < a.q) {
-      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + i / a.qs) * a.qsh + (int64_t)(i % a.qs) * a.qss;
+    if (i < qb) {
+      const int qi = c0 + i;
+      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + qi / a.qs) * a.qsh + (int64_t)(qi % a.qs) * a.qss;
       cp_async16(dst, qp + ch * 8);
     } else {
       sts_v4(dst, make_uint4(0, 0, 0, 0));
@@ -486,17 +495,19 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
         tmem_ld32(ocol + qoff + 32 * ch, o);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const int colq = ch * 32 + i;
-          if (colq < a.q) {
+          const int cl_ = ch * 32 + i;  // column within the block
+          if (cl_ < qb) {
+            const int colq = c0 + cl_;
             const int64_t uq = bb * (a.H * a.G) + hh * a.G + colq / a.qs;
             const int iq = colq % a.qs;
             a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + wt] = o[i];
           }
         }
       }
-      for (int colq = tid; colq < a.q; colq += NTH) {
+      for (int cl_ = tid; cl_ < qb; cl_ += NTH) {
+        const int colq = c0 + cl_;
         const int64_t uq = bb * (a.H * a.G) + hh * a.G + colq / a.qs;
-        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq % a.qs] = make_float2(cm[colq] * ln2, cl[colq]);
+        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq % a.qs] = make_float2(cm[cl_] * ln2, cl[cl_]);
       }
     }
   }
@@ -530,7 +541,11 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   a.idx = idx;
   a.n = kv.seq; a.k = p.k; a.ng = p.ng;
   a.G = p.G; a.qs = p.q; a.q = p.G * p.q; a.H = kv.heads;
-  a.nq = (a.q + 31) / 32 * 32;
+  // Column blocks of at most 128 query rows: S^T and O^T then take at most
+  // 256 TMEM columns, so two CTAs share an SM.
+  const int nblk = (a.q + 127) / 128;
+  a.cb = (((a.q + nblk - 1) / nblk) + 31) / 32 * 32;
+  a.nq = a.cb;
   uint32_t cols = 32;
   while ((int)cols < 2 * a.nq) cols *= 2;
   a.tcols = cols;
@@ -540,14 +555,14 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   a.qstride = kMaxQ;
   a.status = status;
   a.sl2 = 1.4426950408889634f * scale;
-  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + (size_t)a.nq * 256 + sizeof(float) * (NWG * 4 * 32 + 512) + 32;
+  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 512) + 32;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;
   const size_t floor_smem = per_sm / (cap + 1) + 1;
   if (cap < (size_t)(2048 / NTH) && smem < floor_smem) smem = floor_smem;
   cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  tc_attn_kernel<<<dim3((unsigned)a.nsplit, (unsigned)(kv.batch * kv.heads)), NTH, smem, s>>>(a);
+  tc_attn_kernel<<<dim3((unsigned)a.nsplit, (unsigned)(kv.batch * kv.heads), (unsigned)nblk), NTH, smem, s>>>(a);
   *nsplit_out = a.nsplit;
   return cudaGetLastError();
 }
