@@ -306,7 +306,7 @@ def run_gpu(args, cfg, rank, world, device):
             # the pyramid), the finer scales' transforms inside every step.
             coeffs = torch.empty(w.batch, w.heads, w.n >> w.levels, w.head_dim, dtype=lay.K.dtype, device=device)
             wf.wf_wavelet_approx(lay.K, w.levels, basis, coeffs)
-            ws = torch.empty(max(wf.wf_filter_wavelet_workspace_bytes(lay.Q, lay.K, w.levels, keep, basis),
+            ws = torch.zeros(max(wf.wf_filter_wavelet_workspace_bytes(lay.Q, lay.K, w.levels, keep, basis),
                                  wf.wf_attn_workspace_bytes(lay.Q, w.k, w.ng)), dtype=torch.uint8, device=device)
         else:
             coeffs = torch.empty(wf.wf_coeffs_bytes(lay.K, w.levels), dtype=torch.uint8, device=device)

@@ -95,7 +95,8 @@ def test_gqa_attention_equals_repeated_key_heads():
     K1, V1, Kg1, Vg1 = rep(batch.K), rep(batch.V), rep(batch.Kg), rep(batch.Vg)
     idx1 = grouped.idx.repeat_interleave(G, dim=0).contiguous()
     O1 = torch.empty_like(batch.Q)
-    ws = torch.empty(wf.wf_attn_workspace_bytes(batch.Q, w.k, w.ng), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(wf.wf_attn_workspace_bytes(batch.Q, w.k, w.ng), dtype=torch.uint8, device="cuda")
     wf.wf_sparse_attn(batch.Q, K1, V1, idx1, w.k, Kg1, Vg1, O1, ws)
+    wf.wf_workspace_status(ws)
     torch.cuda.synchronize()
     assert torch.equal(O1, grouped.O)

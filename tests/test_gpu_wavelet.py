@@ -91,11 +91,12 @@ def _filter_wavelet(batch, w, wv):
     B, H = K.shape[:2]
     top = torch.empty(B, H, w.n >> w.levels, w.head_dim, dtype=K.dtype, device="cuda")
     wf.wf_wavelet_approx(K, w.levels, wv, top)
-    ws = torch.empty(wf.wf_filter_wavelet_workspace_bytes(Q, K, w.levels, w.keep, wv), dtype=torch.uint8,
+    ws = torch.zeros(wf.wf_filter_wavelet_workspace_bytes(Q, K, w.levels, w.keep, wv), dtype=torch.uint8,
                      device="cuda")
     idx = torch.empty(B * H, w.k, dtype=torch.int32, device="cuda")
     sets = torch.empty(B * H, sum(w.keep), dtype=torch.int32, device="cuda")
     wf.wf_filter_wavelet(Q, top, K, w.levels, w.keep, wv, idx, ws, level_sets=sets)
+    wf.wf_workspace_status(ws)
     torch.cuda.synchronize()
     return idx, sets
 

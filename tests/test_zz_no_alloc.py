@@ -26,7 +26,7 @@ def _inputs(cfg, seed):
 @pytest.mark.parametrize("cfg", ["c1", "c2"])
 def test_noalloc_matches_workspace_entry_point(cfg):
     w, batch, idx = _inputs(cfg, 1)
-    ws = torch.empty(wf.wf_attn_workspace_bytes(batch.Q, w.k, w.ng), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(wf.wf_attn_workspace_bytes(batch.Q, w.k, w.ng), dtype=torch.uint8, device="cuda")
     ref = torch.empty_like(batch.Q)
     wf.wf_sparse_attn(batch.Q, batch.K, batch.V, idx, w.k, batch.Kg, batch.Vg, ref, ws)
     for call in range(2):
