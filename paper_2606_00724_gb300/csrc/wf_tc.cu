@@ -5,22 +5,22 @@
 //   stats: per (tile, query row) the max and the sum of 2^(s - max) of the
 //          tile's logits (log2 units) -> part[unit][tile][row];
 //   keys:  the query rows' normalisers c_i = M_i + log2 S_i (folded from all
-//          tiles' partials by a small kernel in between), then each candidate's ranking key
-//          log2 W_j = log2 sum_i 2^(s_ij - c_i) (Eq. 8 as a log-sum-exp)
-//          -> W[unit][j].
+//          tiles' partials by a small kernel in between), then each
+//          candidate's ranking key log2 W_j = log2 sum_i 2^(s_ij - c_i)
+//          (Eq. 8 as a log-sum-exp) -> W[unit][j].
 // The keys pass recomputes the MMA instead of storing the logits: a tile's
 // rows are read twice (the second time mostly from L2) and no logit matrix
 // goes through memory.
 //
-// One CTA of two warpgroups per (tile, unit); each warpgroup covers the 128
-// TMEM lanes (a warp per lane quarter) and takes every other 32-column chunk
-// of the query columns.  All threads gather the tile (16-byte cp.async into the 128-byte-swizzled
-// K-major layout) and the query block (cp.async into K-major core matrices,
-// zero rows up to a multiple of 32), one thread issues the eight MMAs (K = 128) into TMEM
-// and commits them to an mbarrier, and every thread reads back its
-// candidate's row in chunks of 32 query columns.  The wait on the MMAs is
-// bounded (~1 s): on a timeout the CTA sets the status word, waits once more
-// with the same bound, frees its TMEM and leaves.
+// One CTA of two warpgroups per (tile, unit).  All threads gather the tile
+// (16-byte cp.async into the 128-byte-swizzled K-major layout) and the query
+// block (cp.async into K-major core matrices, zero rows up to a multiple of
+// 32); one thread issues the eight MMAs (K = 128) into TMEM and commits them
+// to an mbarrier.  Each warpgroup covers the 128 TMEM lanes (a warp per lane
+// quarter, a thread per candidate) and reads back every other 32-column
+// chunk of the query columns.  The wait on the MMAs is bounded (~1 s): on a
+// timeout the CTA sets the status word, waits once more with the same
+// bound, frees its TMEM and leaves.
 #include <math.h>
 
 #include "wf_internal.cuh"
@@ -270,7 +270,8 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
   // Shared memory: the tile, the query block, the reductions, the barrier.
   // At most 512 / cols CTAs may share an SM (TMEM); the request is padded so
   // that shared memory enforces it.
-  size_t smem = 2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 256) + sizeof(float2) * 128 + 16;
+  size_t smem =
+      2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 256) + sizeof(float2) * 128 + 16;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;  // CTAs per SM the TMEM allows
   const size_t floor_smem = per_sm / (cap + 1) + 1;
