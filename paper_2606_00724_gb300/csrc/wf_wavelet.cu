@@ -11,9 +11,10 @@
 // gathers the TO 2^b input rows plus the (taps - 2)(2^b - 1) rows the filter
 // reaches past them (wrapping around the gathered sequence) into shared
 // memory with 16-byte cp.async copies, and runs the b levels of the cascade
-// there in fp32 (two buffers alternating).  Arithmetic (the storage rule, shared with the Haar pyramid):
-// Haar: fl32(x0 + x1) * fl32(1 / sqrt 2); db2: the products
-// fl32(fl32(h[k]) * x) added left to right in fp32, no fused multiply-add.
+// there in fp32 (two buffers alternating; a thread slides its filter window
+// over a run of outputs for a channel pair).  Arithmetic, the storage rule:
+// Haar: fl32(x0 + x1) * fl32(1 / sqrt 2), as the stored pyramid; db2:
+// fl32(fl32(h[0]) x0), then fused multiply-adds with fl32(h[1..3]) in order.
 // Only the last level is rounded to the key dtype.
 #include <math.h>
 
@@ -45,8 +46,8 @@ __device__ __forceinline__ float rd(const T* p) { return to_f32(*p); }
 template <typename T, int TAPS, int DS>
 __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, int64_t ksb, int64_t ksh, int64_t kss,
                                                      int64_t n, int H, const int32_t* __restrict__ cand,
-                                                     int64_t cand_stride, int m, int level, Taps taps, T* __restrict__ out,
-                                                     int64_t out_unit, int64_t out_row) {
+                                                     int64_t cand_stride, int m, int level, Taps taps,
+                                                     T* __restrict__ out, int64_t out_unit, int64_t out_row) {
   extern __shared__ __align__(16) uint8_t sbuf[];
   const int to = outputs_per_cta(level);
   const int nin = rows_needed(to, level, TAPS);
