@@ -28,7 +28,7 @@ _lib = None
 
 
 def build(force: bool = False) -> str:
-    """Compile the oracle with gcc (no fused multiply-add, no fast-math)."""
+    """Compile the oracle with gcc (no implicit multiply-add contraction, no fast-math)."""
     if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < max(
         os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "wf_oracle.h"))
     ):
