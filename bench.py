@@ -381,29 +381,44 @@ def run_gpu(args, cfg, rank, world, device):
     lay, bf = layers[0], bufs[0]
     # End to end through the public API with host buffers: copy the step's
     # query block and generation rows in from pinned memory, run the step,
-    # copy O and the indices out.
-    hQ = lay.Q.cpu().pin_memory()
-    hKg = lay.Kg.cpu().pin_memory()
-    hVg = lay.Vg.cpu().pin_memory()
-    hO = torch.empty(lay.Q.shape, dtype=lay.Q.dtype, pin_memory=True)
-    hidx = torch.empty(w.units, w.k, dtype=torch.int32, pin_memory=True)
-    dQ, dKg, dVg = torch.empty_like(lay.Q), torch.empty_like(lay.Kg), torch.empty_like(lay.Vg)
+    # copy O and the indices out.  The inputs sit back to back in one pinned
+    # staging buffer and the outputs in another, so each direction is one
+    # copy; the step reads and writes views of the device buffers.
+    def packed(shapes_dtypes, device_or_pin):
+        offs, off = [], 0
+        for shape, dt in shapes_dtypes:
+            offs.append(off)
+            off += (math.prod(shape) * torch.tensor([], dtype=dt).element_size() + 255) // 256 * 256
+        if device_or_pin == "pin":
+            buf = torch.empty(off, dtype=torch.uint8, pin_memory=True)
+        else:
+            buf = torch.empty(off, dtype=torch.uint8, device=device_or_pin)
+        views = [buf[o:o + math.prod(sh) * torch.tensor([], dtype=dt).element_size()].view(dt).view(sh)
+                 for o, (sh, dt) in zip(offs, shapes_dtypes)]
+        return buf, views
+    ins = [(tuple(lay.Q.shape), lay.Q.dtype), (tuple(lay.Kg.shape), lay.Kg.dtype), (tuple(lay.Vg.shape), lay.Vg.dtype)]
+    outs = [(tuple(lay.Q.shape), lay.Q.dtype), ((w.units, w.k), torch.int32)]
+    hin, (hQ, hKg, hVg) = packed(ins, "pin")
+    din, (dQ, dKg, dVg) = packed(ins, device)
+    hout, _ = packed(outs, "pin")
+    dout, (dO, didx) = packed(outs, device)
+    hQ.copy_(lay.Q.cpu())
+    hKg.copy_(lay.Kg.cpu())
+    hVg.copy_(lay.Vg.cpu())
+    bf_e2e = dict(bf, O=dO, idx=didx)
     e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in range(max(args.steps, 20))]
     for a, b in e2e_ev:
         flush.zero_()
         a.record(stream)
-        dQ.copy_(hQ, non_blocking=True)
-        dKg.copy_(hKg, non_blocking=True)
-        dVg.copy_(hVg, non_blocking=True)
-        one(lay, bf, dQ, dKg, dVg, False)
-        hO.copy_(bf["O"], non_blocking=True)
-        hidx.copy_(bf["idx"], non_blocking=True)
+        din.copy_(hin, non_blocking=True)
+        one(lay, bf_e2e, dQ, dKg, dVg, False)
+        hout.copy_(dout, non_blocking=True)
         b.record(stream)
     torch.cuda.synchronize()
     e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
-    h2d = sum(t.numel() * t.element_size() for t in (hQ, hKg, hVg))
-    d2h = hO.numel() * hO.element_size() + hidx.numel() * 4
+    h2d = hin.numel()
+    d2h = hout.numel()
     return dict(w=w, total_ms=total_ms, step_ms=step_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
                 layers=len(layers))
 
