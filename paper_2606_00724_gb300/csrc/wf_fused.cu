@@ -706,7 +706,8 @@ __device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint
 }
 
 // Per-query max (x sl2, log2 units) of the valid rows of TMEM tiles
-// 0..ntl-1 of region tb -> us.mloc.
+// 0..ntl-1 of region tb -> us.mloc.  The column maxima across a warp come
+// from the warp-wide max instruction.
 __device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int ntl, int mc, float sl2) {
   const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
@@ -723,7 +724,14 @@ __device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int 
       for (int i = 0; i < 32; ++i) mx[i] = fmaxf(mx[i], __uint_as_float(ra[i]));
     }
   }
-  us.red[warp][lane] = transpose_reduce32<true>(mx, lane);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) mx[i] = warp_max_f32(mx[i]);
+  if (lane == 0) {
+#pragma unroll
+    for (int i = 0; i < 32; i += 4)
+      sts_v4(smem_u32(&us.red[warp][i]), make_uint4(__float_as_uint(mx[i]), __float_as_uint(mx[i + 1]),
+                                                    __float_as_uint(mx[i + 2]), __float_as_uint(mx[i + 3])));
+  }
   csync();
   if (tid < 32) {
     float m = -INFINITY;
@@ -735,16 +743,18 @@ __device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int 
 }
 
 // Per-query sum of 2^(l - mloc) over the valid rows -> (mloc, sum) into slot
-// `rank` of every cluster CTA's xstat.
+// `rank` of every cluster CTA's xstat.  Query columns go in pairs through the
+// packed fp32 instructions (the same rounding per element as scalar ones).
 __device__ __noinline__ void pass_sum(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
                                       int ntl, int mc, float sl2) {
   const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  float ml[32], acc[32];
+  const f32x2 s2 = pk2(sl2, sl2);
+  f32x2 nml[16], acc[16];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) {
-    ml[i] = us.mloc[i];
-    acc[i] = 0.f;
+  for (int k = 0; k < 16; ++k) {
+    nml[k] = pk2(-us.mloc[2 * k], -us.mloc[2 * k + 1]);
+    acc[k] = pk2(0.f, 0.f);
   }
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
@@ -753,10 +763,20 @@ __device__ __noinline__ void pass_sum(uint32_t rank, uint32_t cs, Misc& ms, Unit
     tmem_wait_ld();
     if (t * TM + tid < mc) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i) acc[i] += ex2(fmaf(__uint_as_float(ra[i]), sl2, -ml[i]));
+      for (int k = 0; k < 16; ++k) {
+        const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
+        acc[k] = add2(acc[k], pk2(ex2(x.x), ex2(x.y)));
+      }
     }
   }
-  us.red[warp][lane] = transpose_reduce32<false>(acc, lane);
+  float a[32];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const float2 v = up2(acc[k]);
+    a[2 * k] = v.x;
+    a[2 * k + 1] = v.y;
+  }
+  us.red[warp][lane] = transpose_reduce32<false>(a, lane);
   csync();
   if (tid < 32) {
     float sum = 0.f;
@@ -772,33 +792,51 @@ __device__ __noinline__ void pass_sum(uint32_t rank, uint32_t cs, Misc& ms, Unit
 
 // Ranking key log2 W_j of each valid row (Eq. 8 as a log-sum-exp over the
 // query rows, against the normaliser c_i in us.cvec), stored at position
-// g0 + j of every cluster CTA's key array of the unit.
+// g0 + j of every cluster CTA's key array of the unit.  Every exponent
+// l sl2 - c_i is at most 0 (c_i is the log of a sum that contains the row's
+// own term), so the sum of 2^(l sl2 - c_i) cannot overflow and is taken
+// unshifted; padded query columns have c_i = +inf and add 0.  Only if the
+// sum is tiny (below 2^-96, where flushed terms could matter) is it taken
+// again shifted by its largest exponent.
 __device__ __noinline__ void pass_keys(uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb, int ntl, int mc,
-                                       int g0, int q, float sl2, uint32_t keys_a) {
+                                       int g0, float sl2, uint32_t keys_a) {
   const int tid = ctid(), warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const uint32_t bar = bar_addr(ms.kbar[pp]);
-  float cv[32];
+  const f32x2 s2 = pk2(sl2, sl2);
+  f32x2 ncv[16];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) cv[i] = us.cvec[i];
+  for (int k = 0; k < 16; ++k) ncv[k] = pk2(-us.cvec[2 * k], -us.cvec[2 * k + 1]);
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
     uint32_t ra[32];
     tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
     const int j = t * TM + tid;
-    float v[32];
-    float mx = -INFINITY;
+    f32x2 z2 = pk2(0.f, 0.f);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      v[i] = fmaf(__uint_as_float(ra[i]), sl2, -cv[i]);
-      if (i < q) mx = fmaxf(mx, v[i]);
+    for (int k = 0; k < 16; ++k) {
+      const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+      z2 = add2(z2, pk2(ex2(v.x), ex2(v.y)));
     }
-    float z = 0.f;
+    float2 zz = up2(z2);
+    float key = lg2(zz.x + zz.y);
+    if (zz.x + zz.y < 0x1p-96f) {
+      float mx = -INFINITY;
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if (i < q) z += ex2(v[i] - mx);
-    const float key = mx + lg2(z);
+      for (int k = 0; k < 16; ++k) {
+        const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+        mx = fmax3(mx, v.x, v.y);
+      }
+      z2 = pk2(0.f, 0.f);
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+        z2 = add2(z2, pk2(ex2(v.x - mx), ex2(v.y - mx)));
+      }
+      zz = up2(z2);
+      key = mx + lg2(zz.x + zz.y);
+    }
     if (j < mc) {
       const uint32_t dst = keys_a + 4u * (uint32_t)(g0 + j);
 #pragma unroll 1
@@ -992,11 +1030,11 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
 #pragma unroll
       for (int r = 0; r < MAXCS; ++r)
         if (r < (int)c.cs && st[r].y > 0.f) S += st[r].y * ex2(st[r].x - M);
-      us.cvec[tid] = M + lg2(S);
+      us.cvec[tid] = tid < p.q ? M + lg2(S) : INFINITY;  // padded query columns weigh 0
     }
     csync();
     if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-    pass_keys(c.cs, ms, us, pp, tb, ntl, mc, g0, p.q, sl2, keys_a);
+    pass_keys(c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a);
     wait_cluster_or_abort(bar_addr(ms.kbar[pp]), ph, ms, p.status);
     // Eq. 9: Top-K (the same result in every CTA of the cluster).
     select_topk(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a);
