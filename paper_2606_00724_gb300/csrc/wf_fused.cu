@@ -852,11 +852,12 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
                                     uint32_t tb, int ntl, int mc) {
   const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  float ml[32], lsum[32];
+  const f32x2 s2 = pk2(sl2, sl2);
+  f32x2 nml[16], lsum2[16];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) {
-    ml[i] = us.mloc[i];
-    lsum[i] = 0.f;
+  for (int k = 0; k < 16; ++k) {
+    nml[k] = pk2(-us.mloc[2 * k], -us.mloc[2 * k + 1]);
+    lsum2[k] = pk2(0.f, 0.f);
   }
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
@@ -868,16 +869,18 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
     uint32_t ra[32];
     tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    const bool ok = t * TM + tid < mc;
     uint32_t w[16];
+    if (t * TM + tid < mc) {
 #pragma unroll
-    for (int i = 0; i < 32; i += 2) {
-      const float p0 = ok ? ex2(fmaf(__uint_as_float(ra[i]), sl2, -ml[i])) : 0.f;
-      const float p1 = ok ? ex2(fmaf(__uint_as_float(ra[i + 1]), sl2, -ml[i + 1])) : 0.f;
-      const __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
-      lsum[i] += __low2float(h2);
-      lsum[i + 1] += __high2float(h2);
-      w[i / 2] = *reinterpret_cast<const uint32_t*>(&h2);
+      for (int k = 0; k < 16; ++k) {
+        const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
+        const __nv_bfloat162 h2 = __floats2bfloat162_rn(ex2(x.x), ex2(x.y));
+        lsum2[k] = add2(lsum2[k], pk2(__low2float(h2), __high2float(h2)));
+        w[k] = *reinterpret_cast<const uint32_t*>(&h2);
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) w[k] = 0u;  // rows past the slice: P = 0
     }
     // P^T, MN-major core matrices: key group r / 8, query chunk ch.
     const int r = tid;
@@ -889,6 +892,13 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_addr(ms.pfull[pp][pb]));
+  }
+  float lsum[32];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const float2 v = up2(lsum2[k]);
+    lsum[2 * k] = v.x;
+    lsum[2 * k + 1] = v.y;
   }
   us.red[warp][lane] = transpose_reduce32<false>(lsum, lane);
   csync();
