@@ -1074,19 +1074,6 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     if (lev >= 1) sets_off += kb;
   }
 
-  // The sparse key list is known: while the producers stream its K rows,
-  // warm L2 with its V rows (bulk prefetch, a separate engine from the copies).
-  {
-    int a0, mc;
-    attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
-    const RowSrc vs = attn_src(c, p, pp, true, a0, mc);
-#pragma unroll 1
-    for (int r = tid; r < mc; r += NCT) {
-      const bf16* row = vs.kind == 3 ? row_ptr<3>(vs, r) : row_ptr<2>(vs, r);
-      prefetch_l2_bulk(row, D * 2);
-    }
-  }
-
   // Attention: S of the key slice, P for the MMA thread, then the combine.
   int a0, mc;
   attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);

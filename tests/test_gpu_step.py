@@ -117,3 +117,34 @@ def test_step_level0_schedule(cfg):
     idx = run.idx.cpu().numpy()
     for u in range(w.units):
         assert np.array_equal(idx[u], batch.targets[u][0].cpu().numpy()), f"unit {u} planted"
+
+
+@pytest.mark.parametrize("n,period,L,keep", [
+    (8192, 64, 3, [512, 256, 300, 400]),            # groups of 128 equal keys: resolved by ranking
+    (8192, 32, 3, [512, 256, 300, 400]),            # groups of 256: re-bucketed until only equal keys remain
+    (32768, 64, 3, [2048, 1024, 1536, 2048]),       # 4096 keys a scale: 32 keys a Top-K thread
+])
+def test_step_exact_ties(n, period, L, keep):
+    # K repeats one block of `period` tokens, so every scale's coefficient
+    # rows, and with them the ranking keys, repeat exactly: the Top-K
+    # boundary falls inside groups of bit-equal keys on both sides, and
+    # Eq. 9's lower-position rule decides.  Indices must match the oracle
+    # at every scale.
+    g = torch.Generator(device="cpu").manual_seed(n + period)
+    B, H, q, ng, d = 1, 2, 32, 8, 128
+
+    def r(rows):
+        return torch.randn(B, H, rows, d, generator=g).to(torch.bfloat16)
+    Q, V, Kg, Vg = r(q).cuda(), r(n).cuda(), r(ng).cuda(), r(ng).cuda()
+    K = r(period).repeat(1, 1, n // period, 1).contiguous().cuda()
+    run = GpuRun(Q, K, V, Kg, Vg, L, keep).step()
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    for u in range(B * H):
+        Qn, Kn, Vn, Kgn, Vgn = (f64(t[0, u]) for t in (Q, K, V, Kg, Vg))
+        pyr, mu0, sets, O = oracle_unit(Qn, Kn, Vn, Kgn, Vgn, L, keep, True)
+        gsets = run.level_sets(u)
+        for lev in range(L, -1, -1):
+            assert np.array_equal(gsets[lev], sets[lev]), f"unit {u} scale {lev}"
+        assert np.array_equal(run.idx[u].cpu().numpy(), mu0), f"unit {u} mu0"
+        assert_close_out(f64(run.O[0, u]), O, torch.bfloat16)
