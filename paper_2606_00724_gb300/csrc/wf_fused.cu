@@ -925,10 +925,9 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
   tmem_ld32_issue(ocol + lane_base, orow);
   tmem_wait_ld();
   const uint32_t ready = bar_addr(ms.cready[pp]);
-  if (tid == 0) {
-#pragma unroll 1
-    for (uint32_t r = 0; r < cs; ++r) mbar_arrive_cluster(map_rank(ready, r));
-  }
+  // One arrival per CTA, each from its own thread (every thread has seen
+  // this unit's PV products complete), so the remote arrivals overlap.
+  if (tid < (int)cs) mbar_arrive_cluster(map_rank(ready, (uint32_t)tid));
   wait_cluster_or_abort(ready, 0u, ms, p.status);
   const uint32_t comb_a = smem_u32(comb);
   const uint32_t cbar = bar_addr(ms.cbar[pp]);
@@ -974,15 +973,33 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
   const float inv = 1.f / den;
   bf16* ob = p.O + (int64_t)(u / p.H) * p.osb + (int64_t)(u % p.H) * p.osh;
   const int d0 = dlo((int)rank, cs), rows = dlo((int)rank + 1, cs) - d0;
-  if (qi < p.q) {
-#pragma unroll 1
-    for (int dl = tid >> 5; dl < rows; dl += NCT / NQ) {
-      float n = 0.f;
+  auto out = [&](int dl) {
+    float n = 0.f;
 #pragma unroll
-      for (int r = 0; r < MAXCS; ++r)
-        if (r < (int)cs) n = fmaf(lds_f32(comb_a + 4u * (uint32_t)((r * rows + dl) * NQ + qi)), f[r], n);
-      ob[(int64_t)qi * p.oss + d0 + dl] = __float2bfloat16_rn(n * inv);
+    for (int r = 0; r < MAXCS; ++r)
+      if (r < (int)cs) n = fmaf(lds_f32(comb_a + 4u * (uint32_t)((r * rows + dl) * NQ + qi)), f[r], n);
+    return n * inv;
+  };
+  // A slice of 32, 64 or 128 rows (clusters of 4, 2, 1): warp w writes rows
+  // [w rows / 4, (w + 1) rows / 4) of its query, 16 bytes a store; otherwise
+  // one element a store.
+  const bool vec = rows % (NCW * 8) == 0 && d0 % 8 == 0 && p.oss % 8 == 0 &&
+                   (reinterpret_cast<uintptr_t>(ob) & 15) == 0;
+  if (qi < p.q && vec) {
+    const int per = rows / NCW, db = warp * per;
+#pragma unroll 1
+    for (int c0 = 0; c0 < per; c0 += 8) {
+      uint32_t w4[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 h = __floats2bfloat162_rn(out(db + c0 + 2 * e), out(db + c0 + 2 * e + 1));
+        w4[e] = *reinterpret_cast<const uint32_t*>(&h);
+      }
+      *reinterpret_cast<uint4*>(ob + (int64_t)qi * p.oss + d0 + db + c0) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
     }
+  } else if (qi < p.q) {
+#pragma unroll 1
+    for (int dl = tid >> 5; dl < rows; dl += NCT / NQ) ob[(int64_t)qi * p.oss + d0 + dl] = __float2bfloat16_rn(out(dl));
   }
 }
 
