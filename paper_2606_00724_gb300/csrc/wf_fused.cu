@@ -271,25 +271,28 @@ __device__ __forceinline__ RowSrc attn_src(const Ctx& c, const FusedParams& p, i
 // ---------------------------------------------------------------------------
 
 // This producer thread's share of one 128-row tile: 16-byte chunk c = pt % 16
-// of rows pt/16 + RSTEP i, written in the 128-byte-swizzled K-major layout
-// (row r, chunk c at half c/8, byte r*128 + ((c%8) ^ (r%8))*16).  The source
-// addresses of a batch of rows are formed before its copies are issued, so
-// the index loads overlap.
+// of rows pt/16 + RSTEP j, written in the 128-byte-swizzled K-major layout
+// (row r, chunk c at half c/8, byte r*128 + ((c%8) ^ (r%8))*16).  The 16
+// lanes of a half-warp copy the same rows, so each lane forms the source
+// address of one row and the half-warp shares them by shuffles: two address
+// computations a thread per tile instead of one per copy.
 constexpr int RSTEP = NPT / 16;
 constexpr int RROWS = (TM + RSTEP - 1) / RSTEP;  // most rows of one thread
 template <int KIND>
 __device__ __forceinline__ void load_share(uint32_t st, int t, const RowSrc& src, int pt) {
-  const int c = pt & 15, r0 = pt >> 4;
+  const int c = pt & 15, r0 = pt >> 4, half = pt & 16;
   const uint32_t cbase = st + ((c >> 3) << 14);
 #pragma unroll 1
-  for (int b = 0; b < RROWS; b += 8) {
-    const bf16* g[8];
+  for (int q = 0; q < RROWS; q += 16) {
+    // This lane's row: j = q + c (clamped; rows past the tile are not copied).
+    const int rj = min(r0 + RSTEP * min(q + c, RROWS - 1), TM - 1);
+    const unsigned long long a = reinterpret_cast<unsigned long long>(row_ptr<KIND>(src, t * TM + rj));
 #pragma unroll
-    for (int k = 0; k < 8; ++k) g[k] = row_ptr<KIND>(src, t * TM + min(r0 + RSTEP * (b + k), TM - 1)) + c * 8;
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const int r = r0 + RSTEP * (b + k);
-      if (b + k < RROWS && r < TM) cp_async16(cbase + r * 128 + (((c & 7) ^ (r & 7)) << 4), g[k]);
+    for (int k = 0; k < 16; ++k) {
+      const unsigned long long ak = __shfl_sync(0xffffffffu, a, half | k);
+      const int r = r0 + RSTEP * (q + k);
+      if (q + k < RROWS && r < TM)
+        cp_async16(cbase + r * 128 + (((c ^ r) & 7) << 4), reinterpret_cast<const bf16*>(ak) + c * 8);
     }
   }
 }
