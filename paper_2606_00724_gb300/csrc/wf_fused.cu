@@ -201,18 +201,28 @@ struct RowSrc {
   int64_t gstride;
   uint32_t J;  // shared address of the selection the rows derive from
   int kind, g0, mc, kk;
+  int rows;  // rows of the source: indices from a selection are clamped below it
 };
 
-// Branch-free, so a batch of row addresses is formed without divergence.
+// Row r of a slice.  Kinds 0 and 1: the row index in the source; kinds 2
+// and 3: the row's address (a key row or a generation row).  Indices read
+// from a selection are valid rows; the clamp keeps every address inside the
+// source even when a wait gave up and the selection was made from stale data
+// (the status word then reports the failure).
+template <int KIND>
+__device__ __forceinline__ uint32_t row_index(const RowSrc& s, int r) {
+  const int pos = s.g0 + (r < s.mc ? r : 0);  // rows past the slice repeat its first row
+  const uint32_t row = KIND == 0 ? (uint32_t)pos
+                                 : 2u * lds_u32(s.J + 4u * (uint32_t)(pos >> 1)) + (uint32_t)(pos & 1);
+  return min(row, (uint32_t)s.rows - 1u);
+}
 template <int KIND>
 __device__ __forceinline__ const bf16* row_ptr(const RowSrc& s, int r) {
-  const int pos = s.g0 + (r < s.mc ? r : 0);  // rows past the slice repeat its first row
-  if (KIND == 0) return s.base + (int64_t)pos * s.stride;
-  if (KIND == 1) return s.base + (int64_t)(2 * (int)lds_u32(s.J + 4u * (uint32_t)(pos >> 1)) + (pos & 1)) * s.stride;
+  const int pos = s.g0 + (r < s.mc ? r : 0);
   const int pk = min(pos, s.kk - 1);
-  const int tok = KIND == 3 ? (int)lds_u32(s.J + 4u * (uint32_t)pk)
-                            : 2 * (int)lds_u32(s.J + 4u * (uint32_t)(pk >> 1)) + (pk & 1);
-  const bf16* key = s.base + (int64_t)tok * s.stride;
+  const uint32_t tok0 = KIND == 3 ? lds_u32(s.J + 4u * (uint32_t)pk)
+                                  : 2u * lds_u32(s.J + 4u * (uint32_t)(pk >> 1)) + (uint32_t)(pk & 1);
+  const bf16* key = s.base + (int64_t)min(tok0, (uint32_t)s.rows - 1u) * s.stride;
   const bf16* gen = s.gbase + (int64_t)(pos - s.kk) * s.gstride;
   return pos < s.kk ? key : gen;
 }
@@ -245,6 +255,7 @@ __device__ __forceinline__ RowSrc scale_src(const Ctx& c, const FusedParams& p, 
   s.g0 = g0;
   s.mc = mc;
   s.kk = 0;
+  s.rows = lev >= 1 ? (int)(p.n >> lev) : (int)p.n;
   return s;
 }
 
@@ -263,6 +274,7 @@ __device__ __forceinline__ RowSrc attn_src(const Ctx& c, const FusedParams& p, i
   s.g0 = a0;
   s.mc = mc;
   s.kk = p.keep[0];
+  s.rows = (int)p.n;
   return s;
 }
 
@@ -271,28 +283,44 @@ __device__ __forceinline__ RowSrc attn_src(const Ctx& c, const FusedParams& p, i
 // ---------------------------------------------------------------------------
 
 // This producer thread's share of one 128-row tile: 16-byte chunk c = pt % 16
-// of rows pt/16 + RSTEP j, written in the 128-byte-swizzled K-major layout
-// (row r, chunk c at half c/8, byte r*128 + ((c%8) ^ (r%8))*16).  The 16
-// lanes of a half-warp copy the same rows, so each lane forms the source
-// address of one row and the half-warp shares them by shuffles: two address
-// computations a thread per tile instead of one per copy.
+// of rows r0 + RSTEP j (r0 = pt / 16, j < RROWS), written in the
+// 128-byte-swizzled K-major layout (row r, chunk c at half c/8, byte
+// r*128 + ((c%8) ^ (r%8))*16).  The 16 lanes of a half-warp copy the same
+// rows, so each lane forms one row's index or address per 16 rows and the
+// half-warp shares them by shuffles.  The swizzle term of a thread's rows
+// repeats every 4 rows (RSTEP j mod 8 takes 4 values), so each destination
+// is one add.
 constexpr int RSTEP = NPT / 16;
 constexpr int RROWS = (TM + RSTEP - 1) / RSTEP;  // most rows of one thread
+static_assert(RSTEP == 6 && RROWS == 22, "the row schedule below assumes 6 rows a step");
 template <int KIND>
 __device__ __forceinline__ void load_share(uint32_t st, int t, const RowSrc& src, int pt) {
   const int c = pt & 15, r0 = pt >> 4, half = pt & 16;
-  const uint32_t cbase = st + ((c >> 3) << 14);
-#pragma unroll 1
-  for (int q = 0; q < RROWS; q += 16) {
-    // This lane's row: j = q + c (clamped; rows past the tile are not copied).
-    const int rj = min(r0 + RSTEP * min(q + c, RROWS - 1), TM - 1);
-    const unsigned long long a = reinterpret_cast<unsigned long long>(row_ptr<KIND>(src, t * TM + rj));
+  const uint32_t dbase = st + ((c >> 3) << 14) + (uint32_t)r0 * 128u;
+  uint32_t xr[4];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const unsigned long long ak = __shfl_sync(0xffffffffu, a, half | k);
-      const int r = r0 + RSTEP * (q + k);
-      if (q + k < RROWS && r < TM)
-        cp_async16(cbase + r * 128 + (((c ^ r) & 7) << 4), reinterpret_cast<const bf16*>(ak) + c * 8);
+  for (int m = 0; m < 4; ++m) xr[m] = (uint32_t)((c ^ (r0 + RSTEP * m)) & 7) << 4;
+  // Rows j = c and j = 16 + c of this half-warp (clamped into the tile).
+  const int ra = t * TM + r0 + RSTEP * c;
+  const int rb = t * TM + min(r0 + RSTEP * min(16 + c, RROWS - 1), TM - 1);
+  if (KIND <= 1) {
+    const char* cb = reinterpret_cast<const char*>(src.base) + c * 16;
+    const uint32_t sb = (uint32_t)src.stride * 2u;  // row stride in bytes
+    const uint32_t ia = row_index<KIND>(src, ra), ib = row_index<KIND>(src, rb);
+#pragma unroll
+    for (int j = 0; j < RROWS; ++j) {
+      const uint32_t idx = __shfl_sync(0xffffffffu, j < 16 ? ia : ib, half | (j & 15));
+      if (RSTEP * j + RSTEP - 1 < TM || r0 + RSTEP * j < TM)
+        cp_async16(dbase + 128u * RSTEP * j + xr[j & 3], cb + (size_t)idx * sb);
+    }
+  } else {
+    const unsigned long long pa = reinterpret_cast<unsigned long long>(row_ptr<KIND>(src, ra));
+    const unsigned long long pb = reinterpret_cast<unsigned long long>(row_ptr<KIND>(src, rb));
+#pragma unroll
+    for (int j = 0; j < RROWS; ++j) {
+      const unsigned long long ak = __shfl_sync(0xffffffffu, j < 16 ? pa : pb, half | (j & 15));
+      if (RSTEP * j + RSTEP - 1 < TM || r0 + RSTEP * j < TM)
+        cp_async16(dbase + 128u * RSTEP * j + xr[j & 3], reinterpret_cast<const bf16*>(ak) + c * 8);
     }
   }
 }
