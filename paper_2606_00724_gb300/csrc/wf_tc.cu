@@ -39,10 +39,16 @@ constexpr int HALF = TM * 128;         // one 64-column half of the tile
 constexpr int QGRP = (D / 8) * 128;    // bytes per 8-row group of the query block
 constexpr long long kWait = 1ll << 31;
 
+// floor(i / qs) for 0 <= i, qs <= 256 from the reciprocal: (i + 1/2) / qs
+// lies at least 1/(2 qs) from an integer, far beyond the rounding of the
+// product, so truncation is exact.
+__device__ __forceinline__ int head_of(int i, float rqs) { return __float2int_rz(((float)i + 0.5f) * rqs); }
+
 struct TcArgs {
   const bf16* Q;
   int64_t qsb, qsh, qss;
   int q, G, qs, H;              // query rows per unit (G heads of qs rows), key heads
+  float rqs;                    // 1 / qs (head of a query row without a division)
   RowSrc src;                   // candidate rows (row index = cand[j] or j)
   const int32_t* cand;
   int64_t cand_stride;
@@ -139,7 +145,8 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
     const int i = g * 8 + rr;
     const uint32_t dst = smem_u32(sq + g * QGRP + ch * 128 + rr * 16);
     if (i < a.q) {
-      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + i / a.qs) * a.qsh + (int64_t)(i % a.qs) * a.qss;
+      const int hi = head_of(i, a.rqs);
+      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + hi) * a.qsh + (int64_t)(i - hi * a.qs) * a.qss;
       cp_async16(dst, qp + ch * 8);
     } else {
       sts_v4(dst, make_uint4(0, 0, 0, 0));
@@ -252,6 +259,7 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
   a.Q = static_cast<const bf16*>(Q);
   a.qsb = qd.stride_b; a.qsh = qd.stride_h; a.qss = qd.stride_s;
   a.q = p.q; a.G = p.G; a.qs = p.qs; a.H = p.H;
+  a.rqs = 1.0f / (float)a.qs;
   a.src = src;
   a.cand = cand;
   a.cand_stride = p.cmax;
@@ -322,6 +330,7 @@ struct TcAttnArgs {
   int64_t gsb, gsh, gss;
   const int32_t* idx;
   int n, k, ng, q, G, qs, H;  // q = G qs query rows per key unit; H key heads
+  float rqs;                  // 1 / qs
   int cb;                     // query columns per CTA block (blockIdx.z = block)
   int nq;                     // MMA columns of a block (its query rows rounded up to 32)
   uint32_t tcols;
@@ -395,7 +404,8 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     const uint32_t dst = smem_u32(sq + g * QGRP + ch * 128 + rr * 16);
     if (i < qb) {
       const int qi = c0 + i;
-      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + qi / a.qs) * a.qsh + (int64_t)(qi % a.qs) * a.qss;
+      const int hi = head_of(qi, a.rqs);
+      const bf16* qp = a.Q + bb * a.qsb + (hh * a.G + hi) * a.qsh + (int64_t)(qi - hi * a.qs) * a.qss;
       cp_async16(dst, qp + ch * 8);
     } else {
       sts_v4(dst, make_uint4(0, 0, 0, 0));
@@ -499,16 +509,18 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
           const int cl_ = ch * 32 + i;  // column within the block
           if (cl_ < qb) {
             const int colq = c0 + cl_;
-            const int64_t uq = bb * (a.H * a.G) + hh * a.G + colq / a.qs;
-            const int iq = colq % a.qs;
+            const int hq = head_of(colq, a.rqs);
+            const int64_t uq = bb * (a.H * a.G) + hh * a.G + hq;
+            const int iq = colq - hq * a.qs;
             a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + wt] = o[i];
           }
         }
       }
       for (int cl_ = tid; cl_ < qb; cl_ += NTH) {
         const int colq = c0 + cl_;
-        const int64_t uq = bb * (a.H * a.G) + hh * a.G + colq / a.qs;
-        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq % a.qs] = make_float2(cm[cl_] * ln2, cl[cl_]);
+        const int hq = head_of(colq, a.rqs);
+        const int64_t uq = bb * (a.H * a.G) + hh * a.G + hq;
+        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq - hq * a.qs] = make_float2(cm[cl_] * ln2, cl[cl_]);
       }
     }
   }
@@ -542,6 +554,7 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   a.idx = idx;
   a.n = kv.seq; a.k = p.k; a.ng = p.ng;
   a.G = p.G; a.qs = p.q; a.q = p.G * p.q; a.H = kv.heads;
+  a.rqs = 1.0f / (float)a.qs;
   // Column blocks of at most 128 query rows: S^T and O^T then take at most
   // 256 TMEM columns, so two CTAs share an SM.
   const int nblk = (a.q + 127) / 128;
