@@ -125,18 +125,25 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
     mbar_init(smem_u32(bar), 1);
     fence_mbar_init();
   }
-  // The tile: chunk c = tid % 16 of rows tid / 16 + 16 i, 128-byte swizzle.
+  // The tile: chunk c = tid % 16 of rows r0 + 16 i (r0 = tid / 16),
+  // 128-byte swizzle.  The 16 lanes of a half-warp copy the same 8 rows: lane
+  // c loads the index of row r0 + 16 (c % 8) and the half-warp shares them
+  // by shuffles; the swizzle term of a thread's rows is constant.
   {
-    const int c = tid & 15;
-    const bf16* rb = static_cast<const bf16*>(a.src.base) + bb * a.src.sb + hh * a.src.sh + a.src.off;
+    constexpr int RPT = TM / (NTH / 16);  // rows a thread copies
+    static_assert(RPT == 8 && (NTH / 16) % 8 == 0, "rows of a thread share r % 8");
+    const int c = tid & 15, r0 = tid >> 4, half = tid & 16;
+    const char* rb = reinterpret_cast<const char*>(static_cast<const bf16*>(a.src.base) + bb * a.src.sb +
+                                                   hh * a.src.sh + a.src.off) + c * 16;
     const int32_t* cd = a.cand ? a.cand + (int64_t)u * a.cand_stride : nullptr;
-    const uint32_t cbase = smem_u32(tile) + ((c >> 3) * HALF);
-#pragma unroll 4
-    for (int i = 0; i < TM / (NTH / 16); ++i) {
-      const int r = (tid >> 4) + (NTH / 16) * i;
-      const int j = min(t * TM + r, a.m - 1);  // rows past the list repeat its last row (finite, masked)
-      const int64_t row = cd ? (int64_t)cd[j] : (int64_t)j;
-      cp_async16(cbase + r * 128 + (((c & 7) ^ (r & 7)) << 4), rb + row * a.src.ss + c * 8);
+    const int jl = min(t * TM + r0 + (NTH / 16) * (c & (RPT - 1)), a.m - 1);  // rows past the list repeat its last row
+    const uint32_t rowl = cd ? (uint32_t)cd[jl] : (uint32_t)jl;
+    const uint32_t sb = (uint32_t)a.src.ss * 2u;
+    const uint32_t dbase = smem_u32(tile) + ((c >> 3) * HALF) + (uint32_t)r0 * 128u + (uint32_t)(((c ^ r0) & 7) << 4);
+#pragma unroll
+    for (int i = 0; i < RPT; ++i) {
+      const uint32_t row = __shfl_sync(0xffffffffu, rowl, half | i);
+      cp_async16(dbase + (uint32_t)(NTH / 16) * 128u * i, rb + (size_t)row * sb);
     }
   }
   // The query block, K-major core matrices; rows q .. nq - 1 zero.
@@ -372,30 +379,37 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     mbar_init(smem_u32(&bar[1]), 1);
     fence_mbar_init();
   }
-  // K and V rows of the split: chunk c = tid % 16 of rows tid / 16 + 16 i.
+  // K and V rows of the split: chunk c = tid % 16 of rows r0 + 16 i
+  // (r0 = tid / 16).  Lane c resolves the K and V rows of row r0 + 16 (c % 8)
+  // (a sparse key or a generation row) and the half-warp shares the two row
+  // addresses by shuffles; the swizzle term of a thread's rows is constant.
   {
-    const int c = tid & 15;
+    constexpr int RPT = TM / (NTH / 16);
+    static_assert(RPT == 8 && (NTH / 16) % 8 == 0, "rows of a thread share r % 8");
+    const int c = tid & 15, r0 = tid >> 4, half = tid & 16;
     const int32_t* ui = a.idx + (int64_t)u * a.k;
-    const uint32_t koff = smem_u32(kt) + ((c >> 3) * HALF), voff = smem_u32(vt) + ((c >> 3) * HALF);
-#pragma unroll 4
-    for (int i = 0; i < TM / (NTH / 16); ++i) {
-      const int r = (tid >> 4) + (NTH / 16) * i;
-      const int tt = min(t0 + r, total - 1);  // keys past the list repeat its last key (P = 0 there)
-      const bf16 *kp, *vp;
-      if (tt < a.k) {
-        int row = ui[tt];
-        row = row < 0 ? 0 : (row >= a.n ? a.n - 1 : row);
-        const int64_t o = bb * a.ksb + hh * a.ksh + (int64_t)row * a.kss + c * 8;
-        kp = a.K + o;
-        vp = a.V + o;
-      } else {
-        const int64_t o = bb * a.gsb + hh * a.gsh + (int64_t)(tt - a.k) * a.gss + c * 8;
-        kp = a.Kg + o;
-        vp = a.Vg + o;
-      }
-      const uint32_t so = r * 128 + (((c & 7) ^ (r & 7)) << 4);
-      cp_async16(koff + so, kp);
-      cp_async16(voff + so, vp);
+    const uint32_t xs = (uint32_t)r0 * 128u + (uint32_t)(((c ^ r0) & 7) << 4);
+    const uint32_t koff = smem_u32(kt) + ((c >> 3) * HALF) + xs, voff = smem_u32(vt) + ((c >> 3) * HALF) + xs;
+    const int tl = min(t0 + r0 + (NTH / 16) * (c & (RPT - 1)), total - 1);  // keys past the list repeat its last key (P = 0 there)
+    const bf16 *kl, *vl;
+    if (tl < a.k) {
+      int row = ui[tl];
+      row = row < 0 ? 0 : (row >= a.n ? a.n - 1 : row);
+      const int64_t o = bb * a.ksb + hh * a.ksh + (int64_t)row * a.kss;
+      kl = a.K + o;
+      vl = a.V + o;
+    } else {
+      const int64_t o = bb * a.gsb + hh * a.gsh + (int64_t)(tl - a.k) * a.gss;
+      kl = a.Kg + o;
+      vl = a.Vg + o;
+    }
+    const unsigned long long ka = reinterpret_cast<unsigned long long>(kl), va = reinterpret_cast<unsigned long long>(vl);
+#pragma unroll
+    for (int i = 0; i < RPT; ++i) {
+      const unsigned long long kp = __shfl_sync(0xffffffffu, ka, half | i), vp = __shfl_sync(0xffffffffu, va, half | i);
+      const uint32_t so = (uint32_t)(NTH / 16) * 128u * i;
+      cp_async16(koff + so, reinterpret_cast<const bf16*>(kp) + c * 8);
+      cp_async16(voff + so, reinterpret_cast<const bf16*>(vp) + c * 8);
     }
   }
   for (int e = tid; e < a.nq * (D / 8); e += NTH) {
