@@ -15,13 +15,18 @@
 // over a run of outputs for a channel pair).  Arithmetic, the storage rule:
 // Haar: fl32(x0 + x1) * fl32(1 / sqrt 2), as the stored pyramid; db2:
 // fl32(fl32(h[0]) x0), then fused multiply-adds with fl32(h[1..3]) in order.
-// Only the last level is rounded to the key dtype.
+// A channel pair goes through the packed fp32 instructions, which round each
+// lane as the scalar ones do.  Only the last level is rounded to the key
+// dtype.
 #include <math.h>
 
 #include "wf_internal.cuh"
+#include "wf_sm100.cuh"
 
 namespace wf {
 namespace {
+
+using namespace sm100;
 
 constexpr int NTH = 256;      // threads per CTA
 constexpr int IN_ROWS = 128;  // gathered rows per CTA before the filter's reach
@@ -88,6 +93,10 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   // outputs, sliding its filter window two rows per output (each output is
   // the same fp32 sequence of products and sums).
   const float c32 = 0.70710678118654752440f;  // fl32(1 / sqrt 2)
+  const f32x2 c2 = pk2(c32, c32);
+  f32x2 h2[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) h2[k] = pk2(taps.h[k], taps.h[k]);
   constexpr int PAIRS = DS / 2;
   constexpr int GROUPS = NTH / PAIRS;
   const int cp = tid % PAIRS, grp = tid / PAIRS;
@@ -98,15 +107,15 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
     const float* src = (l & 1) ? X : Y;  // fp32 input of levels >= 2
     const int per = (nout + GROUPS - 1) / GROUPS;
     const int jb = grp * per, je = min(nout, jb + per);
-    auto in = [&](int row) -> float2 {
+    auto in = [&](int row) -> f32x2 {
       if (l == 1) {
         const T* p = X0 + row * DS + 2 * cp;
-        return make_float2(rd(p), rd(p + 1));
+        return pk2(rd(p), rd(p + 1));
       }
-      return *reinterpret_cast<const float2*>(src + row * DS + 2 * cp);
+      return *reinterpret_cast<const f32x2*>(src + row * DS + 2 * cp);
     };
     if (jb < je) {
-      float2 x[TAPS];
+      f32x2 x[TAPS];
 #pragma unroll
       for (int k = 0; k < TAPS - 2; ++k) x[k + 2] = in(2 * jb + k);
 #pragma unroll 1
@@ -115,20 +124,15 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
         for (int k = 0; k < TAPS - 2; ++k) x[k] = x[k + 2];
         x[TAPS - 2] = in(2 * j + TAPS - 2);
         x[TAPS - 1] = in(2 * j + TAPS - 1);
-        float2 v;
+        f32x2 v;
         if (TAPS == 2) {
-          v.x = __fmul_rn(__fadd_rn(x[0].x, x[1].x), c32);
-          v.y = __fmul_rn(__fadd_rn(x[0].y, x[1].y), c32);
+          v = mul2(add2(x[0], x[1]), c2);
         } else {
-          v.x = __fmul_rn(taps.h[0], x[0].x);
-          v.y = __fmul_rn(taps.h[0], x[0].y);
+          v = mul2(h2[0], x[0]);
 #pragma unroll
-          for (int k = 1; k < TAPS; ++k) {
-            v.x = __fmaf_rn(taps.h[k], x[k].x, v.x);
-            v.y = __fmaf_rn(taps.h[k], x[k].y, v.y);
-          }
+          for (int k = 1; k < TAPS; ++k) v = fma2(h2[k], x[k], v);
         }
-        *reinterpret_cast<float2*>(dst + j * DS + 2 * cp) = v;
+        *reinterpret_cast<f32x2*>(dst + j * DS + 2 * cp) = v;
       }
     }
     __syncthreads();
