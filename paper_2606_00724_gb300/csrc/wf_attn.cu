@@ -137,36 +137,49 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
 // One CTA per (unit, query row): the weight exp(m_s - M) of every split s
 // and the denominator are formed once in shared memory, then each output
 // element is one pass over the splits' partial outputs.
-template <typename T>
-__global__ void __launch_bounds__(128) attn_combine_kernel(const float* __restrict__ Opart,
-                                                           const float2* __restrict__ ML, int nsplit, int q, int D,
-                                                           int H, int qstride, T* __restrict__ O, int64_t osb,
-                                                           int64_t osh, int64_t oss) {
-  extern __shared__ float fw[];  // [nsplit] weights, then the denominator
-  const int u = blockIdx.x, i = blockIdx.y;
+// The combine of nsplit partials (O, m, l) per query row: one warp per row,
+// each lane CPL consecutive channels (CPL = D / 32).  Every lane forms the
+// split weights 2^... = exp(m_s - M) itself, so no shared memory or block
+// barrier is needed; the per-element order (weights, then fused multiply-adds
+// in split order, then one division) is the one of a plain loop.
+template <typename T, int D>
+__global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restrict__ Opart,
+                                                           const float2* __restrict__ ML, int nsplit, int q, int H,
+                                                           int qstride, T* __restrict__ O, int64_t osb, int64_t osh,
+                                                           int64_t oss) {
+  constexpr int CPL = D / 32;
+  const int u = blockIdx.x;
+  const int i = blockIdx.y * 8 + (threadIdx.x >> 5);  // query row of this warp
+  if (i >= q) return;
+  const int lane = threadIdx.x & 31;
   const int64_t bb = u / H, hh = u % H;
   const float2* ml = ML + (int64_t)u * nsplit * qstride + i;
-  if (threadIdx.x < 32) {
-    float mx = -INFINITY;
-    for (int s = threadIdx.x; s < nsplit; s += 32) mx = fmaxf(mx, ml[(int64_t)s * qstride].x);
+  float mx = -INFINITY;
+  for (int s = 0; s < nsplit; ++s) mx = fmaxf(mx, ml[(int64_t)s * qstride].x);
+  const float* op = Opart + ((int64_t)u * nsplit * qstride + i) * D + lane * CPL;
+  float num[CPL], den = 0.f;
 #pragma unroll
-    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    for (int s = threadIdx.x; s < nsplit; s += 32) fw[s] = expf(ml[(int64_t)s * qstride].x - mx);
-    __syncwarp();
-    if (threadIdx.x == 0) {
-      float den = 0.f;
-      for (int s = 0; s < nsplit; ++s) den = fmaf(ml[(int64_t)s * qstride].y, fw[s], den);
-      fw[nsplit] = den;
+  for (int e = 0; e < CPL; ++e) num[e] = 0.f;
+#pragma unroll 4
+  for (int s = 0; s < nsplit; ++s) {
+    const float2 st = ml[(int64_t)s * qstride];
+    const float w = expf(st.x - mx);
+    den = fmaf(st.y, w, den);
+    const float* os = op + (int64_t)s * qstride * D;
+    if (CPL == 4) {
+      const float4 v = *reinterpret_cast<const float4*>(os);
+      num[0] = fmaf(v.x, w, num[0]);
+      num[1] = fmaf(v.y, w, num[1]);
+      num[2] = fmaf(v.z, w, num[2]);
+      num[3] = fmaf(v.w, w, num[3]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < CPL; ++e) num[e] = fmaf(os[e], w, num[e]);
     }
   }
-  __syncthreads();
-  const float* op = Opart + ((int64_t)u * nsplit * qstride + i) * D;
-  const float den = fw[nsplit];
-  for (int c = threadIdx.x; c < D; c += blockDim.x) {
-    float num = 0.f;
-    for (int s = 0; s < nsplit; ++s) num = fmaf(op[(int64_t)s * qstride * D + c], fw[s], num);
-    from_f32(O[bb * osb + hh * osh + (int64_t)i * oss + c], num / den);
-  }
+  T* ob = O + bb * osb + hh * osh + (int64_t)i * oss + lane * CPL;
+#pragma unroll
+  for (int e = 0; e < CPL; ++e) from_f32(ob[e], num[e] / den);
 }
 
 // The combine of nsplit partials per query-head unit into O.
@@ -174,11 +187,13 @@ template <typename T>
 cudaError_t combine(const AttnPlan& p, int nsplit, void* O, const wf_tensor& od, void* ws, cudaStream_t s) {
   float* Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
   float2* ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
-  const size_t csmem = sizeof(float) * (size_t)(nsplit + 1);
-  cudaError_t e = cudaFuncSetAttribute(attn_combine_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem);
-  if (e != cudaSuccess) return e;
-  attn_combine_kernel<T><<<dim3((unsigned)p.U, (unsigned)p.q), 128, csmem, s>>>(
-      Opart, ML, nsplit, p.q, p.d, p.H, QMAX, static_cast<T*>(O), od.stride_b, od.stride_h, od.stride_s);
+  const dim3 grid((unsigned)p.U, (unsigned)((p.q + 7) / 8));
+  if (p.d == 128)
+    attn_combine_kernel<T, 128><<<grid, 256, 0, s>>>(Opart, ML, nsplit, p.q, p.H, QMAX, static_cast<T*>(O),
+                                                     od.stride_b, od.stride_h, od.stride_s);
+  else
+    attn_combine_kernel<T, 64><<<grid, 256, 0, s>>>(Opart, ML, nsplit, p.q, p.H, QMAX, static_cast<T*>(O),
+                                                    od.stride_b, od.stride_h, od.stride_s);
   return cudaGetLastError();
 }
 
