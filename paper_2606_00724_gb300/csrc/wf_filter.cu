@@ -181,6 +181,9 @@ __device__ __forceinline__ int block_scan_flag(bool flag, int* warp_tot, int* to
   return r;
 }
 
+// R > 0: the unit's keys stay in registers, R a thread (m <= 1024 R), read
+// once for the four passes and the output; R == 0: read again every pass.
+template <int R>
 __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ W, int64_t w_unit,
                                                       const int32_t* __restrict__ cand, int64_t cand_stride,
                                                       int m, int kk, int expand, int32_t* __restrict__ out,
@@ -196,15 +199,24 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   uint32_t prefix = 0, mask = 0;
   uint32_t need = (uint32_t)kk;
   const int lane = tid & 31;
+  const int nch = R > 0 ? R : (m + 1023) / 1024;  // 1024-key chunks
+  uint32_t kr[R > 0 ? R : 1];
+#pragma unroll
+  for (int r = 0; r < (R > 0 ? R : 1); ++r) {
+    const int j = r * 1024 + tid;
+    kr[r] = (R > 0 && j < m) ? order_key(w[j]) : 0u;
+  }
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
     if (tid < 256) hist[tid] = 0;
     __syncthreads();
     // Keys crowd into few bins (sign and exponent bits first): the lanes of a
     // warp that share a bin add their count with one atomic.
-    for (int base = 0; base < m; base += blockDim.x) {
-      const int j = base + tid;
-      const uint32_t key = j < m ? order_key(w[j]) : 0u;
+#pragma unroll
+    for (int r = 0; r < (R > 0 ? R : 64); ++r) {
+      if (R == 0 && r >= nch) break;
+      const int j = r * 1024 + tid;
+      const uint32_t key = R > 0 ? kr[r] : (j < m ? order_key(w[j]) : 0u);
       const bool in = j < m && (key & mask) == prefix;
       const unsigned act = __ballot_sync(0xffffffffu, in);
       if (in) {
@@ -254,9 +266,11 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
   int32_t* o = out + (int64_t)u * out_stride;
   int32_t* st = sets ? sets + (int64_t)u * sets_stride + sets_off : nullptr;
   int running = 0, eq_seen = 0;
-  for (int base = 0; base < m; base += blockDim.x) {
-    const int j = base + tid;
-    const uint32_t key = j < m ? order_key(w[j]) : 0u;
+#pragma unroll
+  for (int r = 0; r < (R > 0 ? R : 64); ++r) {
+    if (R == 0 && r >= nch) break;
+    const int j = r * 1024 + tid;
+    const uint32_t key = R > 0 ? kr[r] : (j < m ? order_key(w[j]) : 0u);
     const bool gt = j < m && key > prefix;
     const bool eq = j < m && key == prefix;
     const int eq_rank = block_scan_flag(eq, warp_tot, &s_total);
@@ -275,6 +289,21 @@ __global__ void __launch_bounds__(1024) select_kernel(const float* __restrict__ 
     eq_seen += eq_tot;
     __syncthreads();
   }
+}
+
+// The Top-K launch: keys in registers up to 8192 candidates.
+static void launch_select(int U, const float* W, int64_t w_unit, const int32_t* cand, int64_t cand_stride, int m,
+                          int kk, int expand, int32_t* out, int64_t out_stride, int32_t* sets, int64_t sets_stride,
+                          int64_t sets_off, cudaStream_t s) {
+  const int nch = (m + 1023) / 1024;
+#define WF_SELECT(R) select_kernel<R><<<U, 1024, 0, s>>>(W, w_unit, cand, cand_stride, m, kk, expand, out, out_stride, \
+                                                         sets, sets_stride, sets_off)
+  if (nch <= 1) WF_SELECT(1);
+  else if (nch <= 2) WF_SELECT(2);
+  else if (nch <= 4) WF_SELECT(4);
+  else if (nch <= 8) WF_SELECT(8);
+  else WF_SELECT(0);
+#undef WF_SELECT
 }
 
 template <typename T, int D, int QM>
@@ -385,8 +414,8 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
     const bool last = (l == 1) && !p.trim;
     int32_t* out = last ? idx : cand_nxt;
     const int64_t out_stride = last ? p.keep[0] : p.cmax;
-    select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand, p.cmax, m, p.keep[l], 1, out, out_stride, level_sets,
-                                       sets_stride, sets_off);
+    launch_select(p.U, W, p.cmax, cand, p.cmax, m, p.keep[l], 1, out, out_stride, level_sets,
+                                       sets_stride, sets_off, s);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     sets_off += p.keep[l];
     m = 2 * p.keep[l];
@@ -401,7 +430,7 @@ cudaError_t launch_filter(const FilterPlan& p, const void* Q, const wf_tensor& q
     src.ss = kv.stride_s;
     src.off = 0;
     if ((e = skim(p, Q, qd, src, cand_cur, m, logits, part, W, status, s)) != cudaSuccess) return e;
-    select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0);
+    launch_select(p.U, W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0, s);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (level_sets) {
@@ -456,8 +485,8 @@ cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_t
     int32_t* out = last ? idx : cand_nxt;
     const int64_t out_stride = last ? p.keep[0] : p.cmax;
     const int32_t* cand = l == p.L ? nullptr : cand_cur;  // position -> block index at scale l
-    select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand, p.cmax, m, p.keep[l], 1, out, out_stride, level_sets,
-                                       sets_stride, sets_off);
+    launch_select(p.U, W, p.cmax, cand, p.cmax, m, p.keep[l], 1, out, out_stride, level_sets,
+                                       sets_stride, sets_off, s);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     sets_off += p.keep[l];
     m = 2 * p.keep[l];
@@ -471,7 +500,7 @@ cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_t
     src.ss = kv.stride_s;
     src.off = 0;
     if ((e = skim(p, Q, qd, src, cand_cur, m, logits, part, W, status, s)) != cudaSuccess) return e;
-    select_kernel<<<p.U, 1024, 0, s>>>(W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0);
+    launch_select(p.U, W, p.cmax, cand_cur, p.cmax, m, p.keep[0], 0, idx, p.keep[0], nullptr, 0, 0, s);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (level_sets) {
