@@ -67,7 +67,7 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   const int64_t bb = u / H, hh = u % H;
   const int len = m << level;  // the gathered sequence (< 2^31 tokens)
   const int blk_mask = (1 << level) - 1;
-  const T* kb = K + bb * ksb + hh * ksh + c0;
+  const T* kb_src = K + bb * ksb + hh * ksh + c0;
   const int32_t* cd = cand ? cand + (int64_t)u * cand_stride : nullptr;
   const int tid = threadIdx.x;
 
@@ -76,15 +76,28 @@ __global__ void __launch_bounds__(NTH) approx_kernel(const T* __restrict__ K, in
   constexpr int VPR = DS / VEC;  // 16-byte vectors per row
   const uint32_t xs = (uint32_t)__cvta_generic_to_shared(X0);
   const int base = (int)(((int64_t)j0 << level) % len);
-  for (int e = tid; e < nin * VPR; e += NTH) {
-    const int r = e / VPR, v = e % VPR;
-    int p = base + r;
-    if (p >= len) p = p - len < len ? p - len : p % len;  // the filter's reach wraps around
-    int64_t tok = cd ? (((int64_t)cd[p >> level]) << level) + (p & blk_mask) : p;
-    tok = tok < 0 ? 0 : (tok >= n ? n - 1 : tok);  // out-of-range block indices are clamped
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(xs + (uint32_t)((r * DS + v * VEC) * sizeof(T))),
-                 "l"(kb + tok * kss + v * VEC)
-                 : "memory");
+  // Copy e = tid + NTH k is vector v = tid % VPR of row tid / VPR + (NTH / VPR) k.
+  // The VPR lanes of a row share its token: in each batch of VPR copies,
+  // lane v resolves the row of copy kb + v and its group reads them by shuffle.
+  static_assert(32 % VPR == 0 && NTH % VPR == 0, "a row's lanes sit in one warp");
+  const int v = tid % VPR, r0 = tid / VPR, gbase = (tid & 31) & ~(VPR - 1);
+  const int iters = (nin * VPR - tid + NTH - 1) / NTH;  // this thread's copies
+  const int iters_w = (nin * VPR - (tid & ~31) + NTH - 1) / NTH;  // the most of any lane in the warp
+#pragma unroll 1
+  for (int kb = 0; kb < iters_w; kb += VPR) {
+    int p = base + r0 + (NTH / VPR) * (kb + v);
+    p = p < len ? p : (p - len < len ? p - len : p % len);  // the filter's reach wraps around
+    int64_t tl = cd ? (((int64_t)cd[p >> level]) << level) + (p & blk_mask) : p;
+    tl = tl < 0 ? 0 : (tl >= n ? n - 1 : tl);  // out-of-range block indices are clamped
+#pragma unroll
+    for (int k = 0; k < VPR; ++k) {
+      const int64_t tok = __shfl_sync(0xffffffffu, tl, gbase | k);
+      const int it = kb + k, r = r0 + (NTH / VPR) * it;
+      if (it < iters)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(xs + (uint32_t)((r * DS + v * VEC) * sizeof(T))),
+                     "l"(kb_src + tok * kss + v * VEC)
+                     : "memory");
+    }
   }
   asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
