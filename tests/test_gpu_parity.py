@@ -78,6 +78,8 @@ def _rand_case(seed, B, H, n, d, q, ng, dtype, bshd=False, device="cuda"):
     (2048, 128, 64, 32, 4, [256, 128, 128, 128, 128], False),  # 64 query rows
     (128, 64, 7, 2, 3, [128, 64, 32, 16], False),      # keep everything (k = n)
     (64, 128, 3, 0, 6, [1, 1, 1, 1, 1, 1, 1], False),  # deepest pyramid, k = 1
+    (65536, 128, 32, 32, 3, [3000, 4000, 5000, 6000], False),  # lists of 8192 / 12000 / 10000 / 8000: the
+                                                               # Top-K's register and memory paths
 ])
 def test_random_shapes(dtype, n, d, q, ng, L, keep, bshd):
     B, H = 2, 3
