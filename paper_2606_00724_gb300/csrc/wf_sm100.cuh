@@ -1,7 +1,7 @@
 // sm_100-family (sm_103a) device primitives written as inline PTX: tcgen05
 // tensor-core MMA with TMEM accumulators, shared-memory matrix descriptors,
-// mbarriers with bounded waits, cp.async, and thread-block-cluster (DSMEM)
-// access.
+// mbarriers with bounded waits, cp.async, thread-block-cluster (DSMEM)
+// access, packed fp32 pairs and warp-wide float maxima.
 #pragma once
 
 #include <stdint.h>
@@ -184,12 +184,6 @@ __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Asynchronous prefetch of `bytes` (a multiple of 16) from global memory
-// into L2 by the bulk-copy engine (no destination, no completion).
-__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
-
 // ---------------------------------------------------------------------------
 // mbarrier.
 // ---------------------------------------------------------------------------
@@ -318,24 +312,6 @@ __device__ __forceinline__ float warp_max_f32(float x) {
   float r;
   asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(x));
   return r;
-}
-
-// ---------------------------------------------------------------------------
-// TMA (tensor memory accelerator) loads.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ void tma_prefetch_desc(const void* tmap) {
-  asm volatile("prefetch.tensormap [%0];" ::"l"(tmap) : "memory");
-}
-// Four rows y0..y3 of a 2-D tensor map (box of one row, boxDim[0] columns
-// from column x), written to shared memory one after another with the map's
-// swizzle; completion is counted in bytes on the mbarrier.
-__device__ __forceinline__ void tma_gather4(uint32_t dst, const void* tmap, int x, int y0, int y1, int y2, int y3,
-                                            uint32_t mbar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cta.global.tile::gather4.mbarrier::complete_tx::bytes "
-      "[%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
-      "l"(tmap), "r"(x), "r"(y0), "r"(y1), "r"(y2), "r"(y3), "r"(mbar)
-      : "memory");
 }
 
 // ---------------------------------------------------------------------------
