@@ -139,9 +139,9 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
 // element is one pass over the splits' partial outputs.
 // The combine of nsplit partials (O, m, l) per query row: one warp per row,
 // each lane CPL consecutive channels (CPL = D / 32).  Every lane forms the
-// split weights 2^... = exp(m_s - M) itself, so no shared memory or block
-// barrier is needed; the per-element order (weights, then fused multiply-adds
-// in split order, then one division) is the one of a plain loop.
+// split weights exp(m_s - M) (M the largest m_s) itself, so no shared memory
+// or block barrier is needed; the per-element order (weights, then fused
+// multiply-adds in split order, then one division) is the one of a plain loop.
 template <typename T, int D>
 __global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restrict__ Opart,
                                                            const float2* __restrict__ ML, int nsplit, int q, int H,
