@@ -74,16 +74,22 @@ constexpr uint32_t kCsyncId = 1;           // named barriers 1, 2: the compute w
 constexpr uint32_t kIdescScore = idesc_bf16(TM, NQ, 0, 0);  // A = rows (K-major), B = Q (K-major)
 constexpr uint32_t kIdescPV = idesc_bf16(D, NQ, 1, 1);      // A = V^T (MN-major), B = P^T (MN-major)
 
+constexpr int MAXT = 16;  // TMEM tiles of one unit's region (512 columns / 32)
+
 struct UnitState {
-  float2 xstat[MAXCS][NQ];  // (max, sum of exp) of every cluster CTA's slice
+  float2 xstat[MAXCS][NQ];  // (stabiliser, sum of exp) of every cluster CTA's slice
   float2 cstat[MAXCS][NQ];  // attention (max, row sum) of every CTA (d-slice owner side)
-  float mloc[NQ], cvec[NQ], lacc[NQ];
+  float2 kmm[MAXCS][NCW];   // (min, max) of the ranking keys of every cluster warp
+  float2 wstat[NCW][NQ];    // (stabiliser, sum of exp) of each compute warp's rows
+  float cw[NCW][NQ];        // softmax normaliser c_i, one copy per compute warp
+  float mloc[NQ], lacc[NQ];
   float red[NCW][32];
 };
 
 struct Misc {
   unsigned long long full[4], empty[4];
   unsigned long long mdone[MAXP], jready[MAXP], xbar[MAXP], kbar[MAXP];
+  unsigned long long tdone[MAXP][MAXT];  // scale tile t of a unit scored (one phase per scale)
   unsigned long long pfull[MAXP][2], pempty[MAXP][2], cbar[MAXP], cready[MAXP];
   UnitState us[MAXP];
   int abort;
@@ -378,9 +384,11 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
 // ---------------------------------------------------------------------------
 
 // S^T tile t = rows . Q^T into TMEM columns tb + 32 t, for ntl landed tiles.
+// With tdone != 0 (a scale), tile t's completion is also signalled on the
+// barrier at tdone + 8 t, so the compute warps start on it at once.
 template <int S>
 __device__ __forceinline__ void mma_scores(const Ctx& c, const FusedParams& p, int it0, int ntl, uint32_t tb,
-                                           uint32_t sq) {
+                                           uint32_t sq, uint32_t tdone) {
   Misc& ms = *c.ms;
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
@@ -398,6 +406,7 @@ __device__ __forceinline__ void mma_scores(const Ctx& c, const FusedParams& p, i
                    smem_desc(sq + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
     }
     mma_commit(bar_addr(ms.empty[s]));
+    if (tdone) mma_commit(tdone + 8u * (uint32_t)t);
   }
 }
 
@@ -435,9 +444,9 @@ __device__ void mma_role(const Ctx& c, const FusedParams& p) {
       int g0, mc;
       scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
       const int ntl = tiles_of(mc);
-      mma_scores<S>(c, p, it, ntl, c.tmem + pp * p.ucols, smem_u32(c.smem + c.ly.q + pp * Q_BYTES));
+      mma_scores<S>(c, p, it, ntl, c.tmem + pp * p.ucols, smem_u32(c.smem + c.ly.q + pp * Q_BYTES),
+                    bar_addr(ms.tdone[pp][0]));
       it += ntl;
-      if (ntl > 0) mma_commit(bar_addr(ms.mdone[pp]));  // an empty slice has no phase
     }
   }
   for (int pp = 0; pp < c.np; ++pp) {
@@ -446,7 +455,7 @@ __device__ void mma_role(const Ctx& c, const FusedParams& p) {
     const int ntl = tiles_of(mc);
     const uint32_t tb = c.tmem + pp * p.ucols;
     if (ntl == 0) continue;
-    mma_scores<S>(c, p, it, ntl, tb, smem_u32(c.smem + c.ly.q + pp * Q_BYTES));
+    mma_scores<S>(c, p, it, ntl, tb, smem_u32(c.smem + c.ly.q + pp * Q_BYTES), 0u);
     it += ntl;
     mma_commit(bar_addr(ms.mdone[pp]));
     mma_pv<S>(c, p, pp, it, ntl, tb + p.ucols - 32);
@@ -478,19 +487,19 @@ __device__ __forceinline__ float transpose_reduce32(float (&v)[32], int lane) {
 }
 
 // Top-K scratch.  It lives in the unit's P buffers, which nothing uses before
-// the attention.
+// the attention.  The histogram and the list counter are zero between calls
+// (zeroed at kernel start, cleared again at the end of every call).
 constexpr int NB = 2048;  // histogram buckets
 constexpr int BPT = NB / NCT;
 struct SelScratch {
   uint32_t hist[NB];
   float2 blist[NCT];    // boundary-bucket keys (key, position)
   float2 sred[2][NCW];  // (min, max) per warp, alternating rounds
-  uint32_t ssel[2][4];  // boundary bucket, missing count, bucket count (alternating rounds)
   int wsum[4][NCW];     // per-warp sums of the scans (slot per scan)
   uint32_t bcnt;
 };
-static_assert(sizeof(SelScratch) <= UNIT_P_BYTES, "Top-K scratch must fit the P buffers");
-static_assert(BPT % 4 == 0, "buckets are read four at a time");
+static_assert((sizeof(SelScratch) + 15) / 16 * 16 <= UNIT_P_BYTES, "Top-K scratch must fit the P buffers");
+static_assert(BPT % 4 == 0, "buckets are cleared four at a time");
 
 #define SC_ADDR(sc_a, field) ((sc_a) + (uint32_t)offsetof(SelScratch, field))
 
@@ -521,22 +530,19 @@ __device__ __forceinline__ int bucket_of(float v, float lo, float scale) {
   return min(NB - 1, __float_as_int(__fadd_rd(x, 8388608.f)) - 0x4B000000);
 }
 
-// (min, max) of the undecided keys over the compute threads, via slot `par`.
-template <int R>
-__device__ __forceinline__ float2 cta_minmax(const float (&kv)[R], uint32_t act, uint32_t sc_a, int par) {
+// (min, max) of the undecided keys (bit i of act: position j0 + i of the key
+// array) over the compute threads, via slot `par`.
+__device__ __forceinline__ float2 cta_minmax(uint32_t keys_a, int j0, uint32_t act, uint32_t sc_a, int par) {
   const int lane = threadIdx.x & 31, warp = ctid() >> 5;
   float lo = INFINITY, hi = -INFINITY;
-#pragma unroll
-  for (int x = 0; x < R; ++x) {
-    const bool a = (act >> x) & 1u;
-    lo = fminf(lo, a ? kv[x] : INFINITY);
-    hi = fmaxf(hi, a ? kv[x] : -INFINITY);
+#pragma unroll 1
+  for (uint32_t a = act; a; a &= a - 1) {
+    const float v = lds_f32(keys_a + 4u * (uint32_t)(j0 + __ffs(a) - 1));
+    lo = fminf(lo, v);
+    hi = fmaxf(hi, v);
   }
-#pragma unroll
-  for (int o = 16; o; o >>= 1) {
-    lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-    hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-  }
+  lo = warp_min_f32(lo);
+  hi = warp_max_f32(hi);
   if (lane == 0) sts_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + warp), __float_as_uint(lo), __float_as_uint(hi));
   csync();
 #pragma unroll
@@ -548,92 +554,96 @@ __device__ __forceinline__ float2 cta_minmax(const float (&kv)[R], uint32_t act,
   return make_float2(lo, hi);
 }
 
+// Every warp locates the boundary bucket in the histogram by itself, with no
+// barrier or broadcast: the bucket holding the need-th largest undecided key
+// (buckets ranked high to low), how many of its keys are still needed, and
+// how many it holds.  Lane l sums the 64 buckets [NB - 64 (l + 1), NB - 64 l)
+// (reading them in a lane-rotated order, free of bank conflicts); a scan over
+// the lanes finds the chunk, and a second scan over that chunk's buckets, two
+// a lane, the bucket.
+__device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, int lane) {
+  const uint32_t cbase = hist_a + 4u * (uint32_t)(NB - 64 * (lane + 1));
+  uint32_t tot = 0;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const uint4 v = lds_v4(cbase + 16u * (uint32_t)((i + lane) & 15));
+    tot += v.x + v.y + v.z + v.w;
+  }
+  uint32_t incl = tot;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const int lc = __ffs(__ballot_sync(0xffffffffu, incl >= need)) - 1;
+  const uint32_t above = __shfl_sync(0xffffffffu, incl - tot, lc);
+  const int bb = NB - 1 - 64 * lc - 2 * lane;                 // this lane's buckets bb and bb - 1
+  const uint2 pr = lds_v2(hist_a + 4u * (uint32_t)(bb - 1));  // .x = bucket bb - 1, .y = bucket bb
+  const uint32_t pair = pr.x + pr.y;
+  uint32_t inc2 = pair;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, inc2, o);
+    if (lane >= o) inc2 += t;
+  }
+  const int l2 = __ffs(__ballot_sync(0xffffffffu, above + inc2 >= need)) - 1;
+  const uint32_t before = above + inc2 - pair;
+  const bool upper = before + pr.y >= need;
+  const uint32_t b = upper ? (uint32_t)bb : (uint32_t)(bb - 1);
+  const uint32_t nd = upper ? need - before : need - before - pr.y;
+  const uint32_t ct = upper ? pr.y : pr.x;
+  return make_uint3(__shfl_sync(0xffffffffu, b, l2), __shfl_sync(0xffffffffu, nd, l2),
+                    __shfl_sync(0xffffffffu, ct, l2));
+}
+
 // Top-K of the m keys at keys_a (largest first, lower position wins ties):
 // the kk chosen candidate indices, in ascending position order, overwrite the
 // key array.  A candidate's index is its position at the top scale, else
 // 2 J[j/2] + j%2 with J the previous selection at jprev_a (Eq. 10).
-// Each thread holds a run of R keys in registers (slot x holds position
-// j0 + (x + rot) % R; the rotation spreads a warp's reads over the banks) and
-// one bit per slot for "undecided" and "taken".  Each round spreads the
-// undecided keys over NB buckets linear in [min, max] of those keys (fp32
-// arithmetic is monotone, so a key in a higher bucket is strictly larger) and
-// locates the bucket holding the boundary from the bucket counts: keys above
-// it are taken, keys below it dropped.  A boundary bucket of at most NCT keys
-// is resolved exactly, each owner ranking its keys on (key, -position)
-// against the bucket's list; a larger one is bucketed again over its own
-// range.  If only equal keys remain, the lowest positions are taken.
-template <int R>
-__device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a) {
+// [lo, hi] is the range of the keys (sent along with them).
+// Each thread owns the run of R positions j0 = tid R .. j0 + R - 1 (R a power
+// of two, at most 32), with one bit per position for "undecided" and
+// "taken"; the keys stay in shared memory and every pass re-reads them,
+// visiting a run in a lane-rotated order so that a warp's reads hit distinct
+// banks.  Each round spreads the undecided keys over NB buckets linear in
+// [lo, hi] (fp32 arithmetic is monotone, so a key in a higher bucket is
+// strictly larger); every warp then finds the bucket holding the boundary from
+// the counts: keys above it are taken, keys below it dropped.  A boundary
+// bucket of at most NCT keys is resolved exactly, each owner ranking its keys
+// on (key, -position) against the bucket's list; a larger one is bucketed
+// again over its own range.  If only equal keys remain, the lowest positions
+// are taken.
+__device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
+                                         float lo, float hi, int R) {
   const int tid = ctid(), lane = tid & 31;
   const int j0 = tid * R;
   const int rot = (lane * R) >> 5;
-  float kv[R];
-  uint32_t act = 0, took = 0;  // bit x = slot x
-#pragma unroll
-  for (int x = 0; x < R; ++x) {
-    const int j = j0 + ((x + rot) & (R - 1));
-    kv[x] = lds_f32(keys_a + 4u * (uint32_t)min(j, m - 1));
-    act |= (uint32_t)(j < m) << x;
-  }
+  const int nv = max(0, min(R, m - j0));  // valid positions of the run
+  uint32_t act = nv >= 32 ? 0xffffffffu : (1u << nv) - 1u, took = 0;
+  auto key = [&](int i) { return lds_f32(keys_a + 4u * (uint32_t)min(j0 + i, m - 1)); };
   const uint32_t hist_a = SC_ADDR(sc_a, hist);
-  const uint32_t own_a = hist_a + 4u * (uint32_t)(NB - BPT * (tid + 1));  // buckets bhi - BPT + 1 .. bhi
-  const int bhi = NB - 1 - BPT * tid;  // thread order = buckets from high to low
-#pragma unroll
-  for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
-  float2 lh = cta_minmax<R>(kv, act, sc_a, 0);  // its barrier also publishes the cleared buckets
+  const uint32_t own_a = hist_a + 4u * (uint32_t)(BPT * tid);  // the buckets this thread clears
   uint32_t need = (uint32_t)kk;
   bool resolved = false;
 #pragma unroll 1
   for (int iter = 0; iter < 6; ++iter) {
-    const int par = iter & 1;
-    const float lo = lh.x, hi = lh.y;
     if (!(hi > lo)) break;  // every undecided key is equal (or none is left)
     const float scale = (float)NB / (hi - lo);
-#pragma unroll
-    for (int x = 0; x < R; ++x) reds_add_if((act >> x) & 1u, hist_a + 4u * bucket_of(kv[x], lo, scale), 1u);
-    csync();
-    uint32_t cw[BPT];
-#pragma unroll
-    for (int i = 0; i < BPT / 4; ++i) {
-      const uint4 v = lds_v4(own_a + 16u * i);
-      cw[4 * i] = v.x;
-      cw[4 * i + 1] = v.y;
-      cw[4 * i + 2] = v.z;
-      cw[4 * i + 3] = v.w;
-    }
-    uint32_t tot = 0;
-#pragma unroll
-    for (int i = 0; i < BPT; ++i) tot += cw[i];
-    const uint32_t above = (uint32_t)cta_excl_scan((int)tot, SC_ADDR(sc_a, wsum) + 16u * par);
-    // Every thread has read its buckets: clear them for the next round.
-#pragma unroll
-    for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
-    if (above < need && above + tot >= need) {
-      // This thread's buckets hold the boundary: walk them from high to low
-      // (branch-free; the first bucket that reaches `need` wins).
-      uint32_t acc = above, sb = 0, sneed = 0, scnt = 0;
-      bool found = false;
-#pragma unroll
-      for (int k = BPT - 1; k >= 0; --k) {  // cw[k] is bucket bhi - (BPT - 1 - k)
-        const bool hit = !found && acc + cw[k] >= need;
-        sb = hit ? (uint32_t)(bhi - (BPT - 1 - k)) : sb;
-        sneed = hit ? need - acc : sneed;
-        scnt = hit ? cw[k] : scnt;
-        found = found || hit;
-        acc += cw[k];
-      }
-      sts_v4(SC_ADDR(sc_a, ssel) + 16u * par, make_uint4(sb, sneed, scnt, 0));
-      sts_u32(SC_ADDR(sc_a, bcnt), 0u);
-    }
-    csync();
-    const uint4 sel = lds_v4(SC_ADDR(sc_a, ssel) + 16u * par);
-    const int sb = (int)sel.x;
-    need = sel.y;
-    const uint32_t cnt = sel.z;
-#pragma unroll
+#pragma unroll 4
     for (int x = 0; x < R; ++x) {
-      const uint32_t bit = ((act >> x) & 1u) << x;  // 0 for a decided slot
-      const int bk = bucket_of(kv[x], lo, scale);
+      const int i = (x + rot) & (R - 1);
+      reds_add_if((act >> i) & 1u, hist_a + 4u * bucket_of(key(i), lo, scale), 1u);
+    }
+    csync();
+    const uint3 bd = warp_boundary(hist_a, need, lane);
+    const int sb = (int)bd.x;
+    need = bd.y;
+    const uint32_t cnt = bd.z;
+#pragma unroll 4
+    for (int x = 0; x < R; ++x) {
+      const int i = (x + rot) & (R - 1);
+      const uint32_t bit = act & (1u << i);  // 0 for a decided position
+      const int bk = bucket_of(key(i), lo, scale);
       took |= bk > sb ? bit : 0u;
       act &= bk != sb ? ~bit : ~0u;
     }
@@ -657,21 +667,17 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
       if (lane == 31 && incl > 0) wbase = atoms_add(SC_ADDR(sc_a, bcnt), (uint32_t)incl);
       wbase = __shfl_sync(0xffffffffu, wbase, 31);
       uint32_t slot = wbase + (uint32_t)(incl - nb);
-#pragma unroll
-      for (int x = 0; x < R; ++x) {
-        const bool a = (act >> x) & 1u;
-        sts_v2_if(a, SC_ADDR(sc_a, blist) + 8u * slot, __float_as_uint(kv[x]), (uint32_t)(j0 + ((x + rot) & (R - 1))));
-        slot += a ? 1u : 0u;
+#pragma unroll 1
+      for (uint32_t a = act; a; a &= a - 1, ++slot) {
+        const int i = __ffs(a) - 1;
+        sts_v2(SC_ADDR(sc_a, blist) + 8u * slot, __float_as_uint(key(i)), (uint32_t)(j0 + i));
       }
       csync();
 #pragma unroll 1
       for (uint32_t a = act; a; a &= a - 1) {
-        const int x = __ffs(a) - 1;
-        float kx = 0.f;
-#pragma unroll
-        for (int y = 0; y < R; ++y)
-          if (y == x) kx = kv[y];
-        const int jx = j0 + ((x + rot) & (R - 1));
+        const int i = __ffs(a) - 1;
+        const float kx = key(i);
+        const int jx = j0 + i;
         uint32_t rank = 0;
 #pragma unroll 1
         for (uint32_t v0 = 0; v0 < cnt; v0 += 4) {
@@ -684,56 +690,53 @@ __device__ __noinline__ void select_reg(uint32_t keys_a, int m, int kk, uint32_t
             rank += (v0 + k < cnt) && ((ko > kx) || (ko == kx && (int)o[k].y < jx));
           }
         }
-        if (rank < need) took |= 1u << x;
+        if (rank < need) took |= 1u << i;
       }
       act = 0;
       resolved = true;
       break;
     }
-    lh = cta_minmax<R>(kv, act, sc_a, par ^ 1);  // the boundary bucket's range for the next round
-  }
-  // Position-order masks (bit i = position j0 + i).
-  uint32_t take = 0, eq = 0;
+    // The boundary bucket again over its own range, with a cleared histogram.
+    csync();  // every warp has read the histogram
 #pragma unroll
-  for (int x = 0; x < R; ++x) {
-    const int i = (x + rot) & (R - 1);
-    take |= ((took >> x) & 1u) << i;
-    eq |= ((act >> x) & 1u) << i;
+    for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
+    const float2 lh = cta_minmax(keys_a, j0, act, sc_a, iter & 1);  // its barrier also publishes the cleared buckets
+    lo = lh.x;
+    hi = lh.y;
   }
+  uint32_t take = took;
   if (!resolved) {
     // Only equal keys are undecided: the first `need` by position are taken.
-    const int eq_base = cta_excl_scan(__popc(eq), SC_ADDR(sc_a, wsum) + 48u);
+    const int eq_base = cta_excl_scan(__popc(act), SC_ADDR(sc_a, wsum) + 48u);
     int remaining = (int)need - eq_base;
-    for (uint32_t e = eq; e && remaining > 0; --remaining) {
+    for (uint32_t e = act; e && remaining > 0; --remaining) {
       const uint32_t low = e & (~e + 1u);
       take |= low;
       e ^= low;
     }
   }
-  // Candidate indices of the slots (read before anything is written), then
-  // each winner at its output rank.  The scan's barrier orders every key read
-  // before the key array is overwritten.
-  int cid[R];
-#pragma unroll
-  for (int x = 0; x < R; ++x) {
-    const int j = j0 + ((x + rot) & (R - 1));
-    cid[x] = (top || j >= m) ? j : (int)lds_u32(jprev_a + 4u * (uint32_t)(j >> 1));
+  // Each winner at its output rank.  The scan's barrier orders every read of
+  // the keys, the histogram and the boundary list before the key array is
+  // overwritten and the scratch cleared.
+  int r = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum) + 32u);
+#pragma unroll 1
+  for (uint32_t a = take; a; a &= a - 1, ++r) {
+    const int j = j0 + __ffs(a) - 1;
+    const int cv = top ? j : 2 * (int)lds_u32(jprev_a + 4u * (uint32_t)(j >> 1)) + (j & 1);
+    sts_u32(keys_a + 4u * (uint32_t)r, (uint32_t)cv);
   }
-  const int base = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum) + 32u);
 #pragma unroll
-  for (int x = 0; x < R; ++x) {
-    const int i = (x + rot) & (R - 1);
-    const int j = j0 + i;
-    const int cv = top ? j : 2 * cid[x] + (j & 1);
-    sts_u32_if((take >> i) & 1u, keys_a + 4u * (uint32_t)(base + __popc(take & ((1u << i) - 1u))), (uint32_t)cv);
-  }
+  for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
+  if (tid == 0) sts_u32(SC_ADDR(sc_a, bcnt), 0u);
   csync();
 }
 
-// Top-K dispatch: 16 keys per compute thread up to 2048 candidates, else 32.
-__device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a) {
-  if (m <= 16 * NCT) select_reg<16>(keys_a, m, kk, jprev_a, top, sc_a);
-  else select_reg<32>(keys_a, m, kk, jprev_a, top, sc_a);
+// Top-K dispatch: R = the smallest power of two with R NCT >= m (m <= 32 NCT).
+__device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
+                                            float lo, float hi) {
+  int R = 1;
+  while (R * NCT < m) R <<= 1;
+  select_keys(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
 }
 
 // Per-query max (x sl2, log2 units) of the valid rows of TMEM tiles
@@ -773,26 +776,77 @@ __device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int 
   csync();
 }
 
-// Per-query sum of 2^(l - mloc) over the valid rows -> (mloc, sum) into slot
-// `rank` of every cluster CTA's xstat.  Query columns go in pairs through the
-// packed fp32 instructions (the same rounding per element as scalar ones).
-__device__ __noinline__ void pass_sum(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
-                                      int ntl, int mc, float sl2) {
+// The warp's (stabiliser, sum of 2^(l sl2 - stabiliser)) per query over its
+// rows of TMEM tiles 0..ntl-1, with the stabiliser the column maximum over
+// all those rows: the overflow path of scale_sums, one query column at a
+// time (compact code for a path that real inputs never take).
+__device__ __noinline__ float2 warp_sums_exact(uint32_t tb, int ntl, int mc, float sl2) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  float2 out = make_float2(-INFINITY, 0.f);
+#pragma unroll 1
+  for (int i = 0; i < 32; ++i) {
+    float mx = -INFINITY;
+#pragma unroll 1
+    for (int t = 0; t < ntl; ++t) {
+      const float v = tmem_ld1(tb + lane_base + 32 * t + i);
+      if (t * TM + tid < mc) mx = fmaxf(mx, v);
+    }
+    const float mi = warp_max_f32(mx) * sl2;
+    float sum = 0.f;
+#pragma unroll 1
+    for (int t = 0; t < ntl; ++t) {
+      const float v = tmem_ld1(tb + lane_base + 32 * t + i);
+      if (t * TM + tid < mc) sum += ex2(fmaf(v, sl2, -mi));
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == i) out = make_float2(mi, sum);
+  }
+  return out;
+}
+
+// Softmax statistics of one scale (Eq. 7-8), tile by tile as the MMA thread
+// completes them, so that the exponentials of early tiles overlap the
+// copies of later ones.  Each compute warp takes as its stabiliser per query
+// the largest logit (x sl2, log2 units) of its rows in the first tile (a
+// warp with no row there has none in later tiles either) and accumulates the
+// sum of 2^(l sl2 - m) over its rows.  A later logit more than ~127 above the
+// stabiliser would overflow the sum; the warp then redoes its sums with the
+// maximum over all its rows.  The four warps' (m, sum) merge into the CTA's
+// (M, S) per query, which goes to slot `rank` of every cluster CTA's xstat.
+// tpar holds the parity of each tile barrier's next phase.
+__device__ __noinline__ void scale_sums(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
+                                        int ntl, int mc, float sl2, uint32_t& tpar, int* status) {
   const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const f32x2 s2 = pk2(sl2, sl2);
   f32x2 nml[16], acc[16];
+  float mcol = -INFINITY;  // lane i: this warp's stabiliser of query i
 #pragma unroll
   for (int k = 0; k < 16; ++k) {
-    nml[k] = pk2(-us.mloc[2 * k], -us.mloc[2 * k + 1]);
     acc[k] = pk2(0.f, 0.f);
+    nml[k] = pk2(0.f, 0.f);
   }
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
+    wait_or_abort(bar_addr(ms.tdone[pp][t]), (tpar >> t) & 1u, ms, status);
+    tpar ^= 1u << t;
+    tc_fence_after();
     uint32_t ra[32];
     tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    if (t * TM + tid < mc) {
+    const bool valid = t * TM + tid < mc;
+    if (t == 0) {
+      float m2[2];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        m2[i & 1] = warp_max_f32(valid ? __uint_as_float(ra[i]) : -INFINITY) * sl2;
+        mcol = lane == i ? m2[i & 1] : mcol;
+        if (i & 1) nml[i >> 1] = pk2(-m2[0], -m2[1]);
+      }
+    }
+    if (valid) {
 #pragma unroll
       for (int k = 0; k < 16; ++k) {
         const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
@@ -807,37 +861,82 @@ __device__ __noinline__ void pass_sum(uint32_t rank, uint32_t cs, Misc& ms, Unit
     a[2 * k] = v.x;
     a[2 * k + 1] = v.y;
   }
-  us.red[warp][lane] = transpose_reduce32<false>(a, lane);
+  float2 st = make_float2(mcol, transpose_reduce32<false>(a, lane));
+  if (__any_sync(0xffffffffu, !(st.y <= 3.0e38f))) st = warp_sums_exact(tb, ntl, mc, sl2);
+  sts_v2(smem_u32(&us.wstat[warp][lane]), __float_as_uint(st.x), __float_as_uint(st.y));
   csync();
   if (tid < 32) {
-    float sum = 0.f;
+    float2 w[NCW];
 #pragma unroll
-    for (int w = 0; w < NCW; ++w) sum += us.red[w][tid];
+    for (int k = 0; k < NCW; ++k) {
+      const uint2 v = lds_v2(smem_u32(&us.wstat[k][tid]));
+      w[k] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < NCW; ++k)
+      if (w[k].y > 0.f) M = fmaxf(M, w[k].x);
+    float S = 0.f;
+#pragma unroll
+    for (int k = 0; k < NCW; ++k)
+      if (w[k].y > 0.f) S = fmaf(w[k].y, ex2(w[k].x - M), S);
     const uint32_t dst = smem_u32(&us.xstat[rank][tid]);
     const uint32_t bar = bar_addr(ms.xbar[pp]);
 #pragma unroll 1
     for (uint32_t r = 0; r < cs; ++r)
-      st_async_v2(map_rank(dst, r), __float_as_uint(us.mloc[tid]), __float_as_uint(sum), map_rank(bar, r));
+      st_async_v2(map_rank(dst, r), __float_as_uint(M), __float_as_uint(S), map_rank(bar, r));
   }
 }
 
+// Softmax normaliser per query, c_i = M + log2 S over the whole candidate
+// set from the cluster's (M, S) pairs (padded query columns get +inf and
+// weigh 0), into this warp's copy us.cw[warp].  Every warp forms its own copy,
+// so no barrier across the warps is needed.
+__device__ __forceinline__ void warp_normaliser(UnitState& us, uint32_t cs, int q) {
+  const int lane = threadIdx.x & 31, warp = ctid() >> 5;
+  float2 st[MAXCS];
+#pragma unroll
+  for (int r = 0; r < MAXCS; ++r) {
+    const uint2 v = lds_v2(smem_u32(&us.xstat[min(r, (int)cs - 1)][lane]));
+    st[r] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+  }
+  float M = -INFINITY;
+#pragma unroll
+  for (int r = 0; r < MAXCS; ++r)
+    if (r < (int)cs && st[r].y > 0.f) M = fmaxf(M, st[r].x);
+  float S = 0.f;
+#pragma unroll
+  for (int r = 0; r < MAXCS; ++r)
+    if (r < (int)cs && st[r].y > 0.f) S = fmaf(st[r].y, ex2(st[r].x - M), S);
+  us.cw[warp][lane] = lane < q ? M + lg2(S) : INFINITY;
+  __syncwarp();
+}
+
 // Ranking key log2 W_j of each valid row (Eq. 8 as a log-sum-exp over the
-// query rows, against the normaliser c_i in us.cvec), stored at position
-// g0 + j of every cluster CTA's key array of the unit.  Every exponent
+// query rows, against the normaliser c_i in the warp's copy us.cw[warp]),
+// stored at position g0 + j of every cluster CTA's key array of the unit;
+// each warp's (min, max) key goes to slot (rank, warp) of every CTA's kmm on
+// the same barrier.  Every exponent
 // l sl2 - c_i is at most 0 (c_i is the log of a sum that contains the row's
 // own term), so the sum of 2^(l sl2 - c_i) cannot overflow and is taken
 // unshifted; padded query columns have c_i = +inf and add 0.  Only if the
 // sum is tiny (below 2^-96, where flushed terms could matter) is it taken
 // again shifted by its largest exponent.
-__device__ __noinline__ void pass_keys(uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb, int ntl, int mc,
-                                       int g0, float sl2, uint32_t keys_a) {
-  const int tid = ctid(), warp = tid >> 5;
+__device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
+                                       int ntl, int mc, int g0, float sl2, uint32_t keys_a) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const uint32_t bar = bar_addr(ms.kbar[pp]);
   const f32x2 s2 = pk2(sl2, sl2);
   f32x2 ncv[16];
+  const uint32_t cw_a = smem_u32(&us.cw[warp][0]);
 #pragma unroll
-  for (int k = 0; k < 16; ++k) ncv[k] = pk2(-us.cvec[2 * k], -us.cvec[2 * k + 1]);
+  for (int k = 0; k < 8; ++k) {
+    const uint4 v = lds_v4(cw_a + 16u * k);
+    ncv[2 * k] = pk2(-__uint_as_float(v.x), -__uint_as_float(v.y));
+    ncv[2 * k + 1] = pk2(-__uint_as_float(v.z), -__uint_as_float(v.w));
+  }
+  float kmin = INFINITY, kmax = -INFINITY;
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
     uint32_t ra[32];
@@ -869,11 +968,24 @@ __device__ __noinline__ void pass_keys(uint32_t cs, Misc& ms, UnitState& us, int
       key = mx + lg2(zz.x + zz.y);
     }
     if (j < mc) {
+      kmin = fminf(kmin, key);
+      kmax = fmaxf(kmax, key);
       const uint32_t dst = keys_a + 4u * (uint32_t)(g0 + j);
 #pragma unroll 1
       for (uint32_t r = 0; r < cs; ++r) st_async_b32(map_rank(dst, r), __float_as_uint(key), map_rank(bar, r));
     }
   }
+  // The warp's key range goes with the keys (the Top-K's first bucket range).
+  kmin = warp_min_f32(kmin);
+  kmax = warp_max_f32(kmax);
+  if (lane == 0) {
+    const uint32_t dst = smem_u32(&us.kmm[rank][warp]);
+#pragma unroll 1
+    for (uint32_t r = 0; r < cs; ++r)
+      st_async_v2(map_rank(dst, r), __float_as_uint(kmin), __float_as_uint(kmax), map_rank(bar, r));
+  }
+  // Every TMEM read of the scale is done before the Top-K's barriers.
+  tc_fence_before();
 }
 
 // Attention: P = 2^(s - m) (bf16, P^T MN-major core matrices) of every S tile
@@ -1047,16 +1159,16 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   const int u = c.u0 + pp;
   const float sl2 = p.scale_log2;
   int64_t sets_off = 0;
-  // Parity of the unit's next mdone phase.  The MMA thread commits a phase
-  // only for a non-empty stream, and every such stream waits on these warps'
-  // progress (through the producers' copies or the P tiles), so it is never
-  // two phases ahead.
+  // Parity of the unit's next mdone phase (the attention's two: S tiles
+  // scored, then PV products done).  The MMA thread commits a phase only for
+  // a non-empty stream.
   uint32_t mdp = 0;
   auto wait_mdone = [&]() {
     wait_or_abort(bar_addr(ms.mdone[pp]), mdp, ms, p.status);
     mdp ^= 1u;
     tc_fence_after();
   };
+  uint32_t tpar = 0;  // parity of each scale-tile barrier's next phase
 #pragma unroll 1
   for (int lev = p.L; lev >= c.lev_end; --lev) {
     const uint32_t ph = (uint32_t)(p.L - lev) & 1u;  // phase of the per-scale barriers
@@ -1067,36 +1179,32 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     const int kb = p.keep[lev];
     int32_t* J = unit_J(c, p, pp, lev);  // receives this scale's keys, then its selection
     const uint32_t keys_a = smem_u32(J);
-    if (ntl > 0) wait_mdone();
-    pass_max(ms, us, tb, ntl, mc, sl2);
-    pass_sum(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2);
+    scale_sums(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2, tpar, p.status);
     wait_cluster_or_abort(bar_addr(ms.xbar[pp]), ph, ms, p.status);
-    // Softmax normaliser per query: c = M + log2 S over the whole candidate set.
-    if (tid < 32) {
-      const uint32_t xs_a = smem_u32(&us.xstat[0][tid]);
-      float2 st[MAXCS];
-#pragma unroll
-      for (int r = 0; r < MAXCS; ++r) {
-        const uint2 v = lds_v2(xs_a + (uint32_t)(min(r, (int)c.cs - 1) * NQ * 8));
-        st[r] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
-      }
-      float M = -INFINITY;
-#pragma unroll
-      for (int r = 0; r < MAXCS; ++r)
-        if (r < (int)c.cs && st[r].y > 0.f) M = fmaxf(M, st[r].x);
-      float S = 0.f;
-#pragma unroll
-      for (int r = 0; r < MAXCS; ++r)
-        if (r < (int)c.cs && st[r].y > 0.f) S += st[r].y * ex2(st[r].x - M);
-      us.cvec[tid] = tid < p.q ? M + lg2(S) : INFINITY;  // padded query columns weigh 0
-    }
-    csync();
+    // This phase is complete for tid 0, so the arrival arms the next one.
     if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-    pass_keys(c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a);
+    warp_normaliser(us, c.cs, p.q);
+    pass_keys(c.rank, c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a);
     wait_cluster_or_abort(bar_addr(ms.kbar[pp]), ph, ms, p.status);
+    // The keys' range from the cluster warps' (min, max).
+    float lo, hi;
+    {
+      const int lane = tid & 31;
+      float2 mm = make_float2(INFINITY, -INFINITY);
+      if (lane < (int)c.cs * NCW) {
+        const uint2 v = lds_v2(smem_u32(&us.kmm[lane / NCW][lane % NCW]));
+        mm = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+      }
+      lo = warp_min_f32(mm.x);
+      hi = warp_max_f32(mm.y);
+    }
     // Eq. 9: Top-K (the same result in every CTA of the cluster).
-    select_topk(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a);
-    if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, lev - 1));
+    select_topk(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a, lo, hi);
+    if (tid == 0) {
+      if (lev > c.lev_end)
+        mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, lev - 1) + c.cs * NCW * 8u);
+      mbar_arrive(bar_addr(ms.jready[pp]));  // the selection is complete (the Top-K ends on a barrier)
+    }
     if (c.rank == 0) {
       int32_t* ls = p.level_sets ? p.level_sets + (int64_t)u * p.sets_stride + sets_off : nullptr;
       if (lev >= 1 && ls) {
@@ -1116,9 +1224,6 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
         }
       }
     }
-    tc_fence_before();
-    csync();
-    if (tid == 0) mbar_arrive(bar_addr(ms.jready[pp]));
     if (lev >= 1) sets_off += kb;
   }
 
@@ -1159,6 +1264,7 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
       mbar_init(bar_addr(ms.jready[pp]), 1);
       mbar_init(bar_addr(ms.xbar[pp]), 1);
       mbar_init(bar_addr(ms.kbar[pp]), 1);
+      for (int t = 0; t < MAXT; ++t) mbar_init(bar_addr(ms.tdone[pp][t]), 1);
     }
     for (int pp = 0; pp < MAXP; ++pp) {
       for (int i = 0; i < 2; ++i) {
@@ -1173,7 +1279,7 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     // Arm the first phase of every receive barrier (bytes this CTA expects).
     for (int pp = 0; pp < c.np; ++pp) {
       mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)(p.n >> p.L));
+      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)(p.n >> p.L) + c.cs * NCW * 8u);
       const uint32_t rows = (uint32_t)(dlo((int)c.rank + 1, c.cs) - dlo((int)c.rank, c.cs));
       mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), c.cs * rows * NQ * 4u + c.cs * NQ * 8u);
     }
@@ -1181,6 +1287,12 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   if (warp == MMA_WARP) {
     tmem_alloc(smem_u32(&ms.tmem_base), p.tmem_cols);
     tmem_relinquish();
+  }
+  // The Top-K scratch starts zeroed (histogram, list counter).
+  for (int pp = 0; pp < c.np; ++pp) {
+    uint8_t* sc = smem + c.ly.p + pp * UNIT_P_BYTES;
+    for (int e = tid; e < (int)((sizeof(SelScratch) + 15) / 16); e += NT)
+      *reinterpret_cast<uint4*>(sc + 16 * e) = make_uint4(0, 0, 0, 0);
   }
   // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
   for (int pp = 0; pp < c.np; ++pp) {
