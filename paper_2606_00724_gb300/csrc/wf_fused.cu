@@ -82,6 +82,7 @@ struct UnitState {
   float2 kmm[MAXCS][NCW];   // (min, max) of the ranking keys of every cluster warp
   float2 wstat[NCW][NQ];    // (stabiliser, sum of exp) of each compute warp's rows
   float cw[NCW][NQ];        // softmax normaliser c_i, one copy per compute warp
+  float fw[NCW][NQ];        // 2^(stabiliser - c_i) of each warp (keys from stored exponentials)
   float mloc[NQ], lacc[NQ];
   float red[NCW][32];
 };
@@ -133,6 +134,7 @@ struct FusedParams {
   int* status;
   int q, n, ng, U, H, L, trim, P, cmax, kmax;
   uint32_t tmem_cols, ucols;  // TMEM allocation; columns per unit region
+  uint32_t ecol;              // column of the stored exponentials in a unit region (0: none)
   int32_t keep[12];
   float scale_log2;           // log2(e) / sqrt(d)
 };
@@ -602,25 +604,33 @@ __device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, i
 // 2 J[j/2] + j%2 with J the previous selection at jprev_a (Eq. 10).
 // [lo, hi] is the range of the keys (sent along with them).
 // Each thread owns the run of R positions j0 = tid R .. j0 + R - 1 (R a power
-// of two, at most 32), with one bit per position for "undecided" and
-// "taken"; the keys stay in shared memory and every pass re-reads them,
-// visiting a run in a lane-rotated order so that a warp's reads hit distinct
-// banks.  Each round spreads the undecided keys over NB buckets linear in
-// [lo, hi] (fp32 arithmetic is monotone, so a key in a higher bucket is
-// strictly larger); every warp then finds the bucket holding the boundary from
-// the counts: keys above it are taken, keys below it dropped.  A boundary
-// bucket of at most NCT keys is resolved exactly, each owner ranking its keys
-// on (key, -position) against the bucket's list; a larger one is bucketed
-// again over its own range.  If only equal keys remain, the lowest positions
-// are taken.
+// of two, 4 to 32), with one bit per position for "undecided" and "taken".
+// The keys stay in shared memory; every pass re-reads them four at a time
+// (16-byte loads, the G = R / 4 groups of a run visited in a lane-rotated
+// order so that the 8 lanes of a quarter warp hit distinct banks).  Each
+// round spreads the undecided keys over NB buckets linear in [lo, hi] (fp32
+// arithmetic is monotone, so a key in a higher bucket is strictly larger);
+// every warp then finds the bucket holding the boundary from the counts: keys
+// above it are taken, keys below it dropped.  A boundary bucket of at most
+// NCT keys is resolved exactly, each owner ranking its keys on
+// (key, -position) against the bucket's list; a larger one is bucketed again
+// over its own range.  If only equal keys remain, the lowest positions are
+// taken.
 __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                          float lo, float hi, int R) {
   const int tid = ctid(), lane = tid & 31;
   const int j0 = tid * R;
-  const int rot = (lane * R) >> 5;
-  const int nv = max(0, min(R, m - j0));  // valid positions of the run
+  const int G = R >> 2;                         // groups of four keys in a run
+  const int rotg = ((lane * G) >> 3) & (G - 1);  // first group this lane visits
+  const int nv = max(0, min(R, m - j0));        // valid positions of the run
+  const uint32_t m4 = (uint32_t)((m + 3) & ~3);  // the key array holds m4 >= 4 words
   uint32_t act = nv >= 32 ? 0xffffffffu : (1u << nv) - 1u, took = 0;
-  auto key = [&](int i) { return lds_f32(keys_a + 4u * (uint32_t)min(j0 + i, m - 1)); };
+  // The four keys of group g (clamped into the array; positions past m are
+  // never undecided).
+  auto group = [&](int g) {
+    const uint4 v = lds_v4(keys_a + 4u * min((uint32_t)(j0 + 4 * g), m4 - 4u));
+    return make_float4(__uint_as_float(v.x), __uint_as_float(v.y), __uint_as_float(v.z), __uint_as_float(v.w));
+  };
   const uint32_t hist_a = SC_ADDR(sc_a, hist);
   const uint32_t own_a = hist_a + 4u * (uint32_t)(BPT * tid);  // the buckets this thread clears
   uint32_t need = (uint32_t)kk;
@@ -629,23 +639,35 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
   for (int iter = 0; iter < 6; ++iter) {
     if (!(hi > lo)) break;  // every undecided key is equal (or none is left)
     const float scale = (float)NB / (hi - lo);
-#pragma unroll 4
-    for (int x = 0; x < R; ++x) {
-      const int i = (x + rot) & (R - 1);
-      reds_add_if((act >> i) & 1u, hist_a + 4u * bucket_of(key(i), lo, scale), 1u);
+#pragma unroll 2
+    for (int gg = 0; gg < G; ++gg) {
+      const int g = (gg + rotg) & (G - 1);
+      const float4 v = group(g);
+      const uint32_t a4 = act >> (4 * g);
+      const int b0 = bucket_of(v.x, lo, scale), b1 = bucket_of(v.y, lo, scale);
+      const int b2 = bucket_of(v.z, lo, scale), b3 = bucket_of(v.w, lo, scale);
+      reds_add_if(a4 & 1u, hist_a + 4u * b0, 1u);
+      reds_add_if(a4 & 2u, hist_a + 4u * b1, 1u);
+      reds_add_if(a4 & 4u, hist_a + 4u * b2, 1u);
+      reds_add_if(a4 & 8u, hist_a + 4u * b3, 1u);
     }
     csync();
     const uint3 bd = warp_boundary(hist_a, need, lane);
     const int sb = (int)bd.x;
     need = bd.y;
     const uint32_t cnt = bd.z;
-#pragma unroll 4
-    for (int x = 0; x < R; ++x) {
-      const int i = (x + rot) & (R - 1);
-      const uint32_t bit = act & (1u << i);  // 0 for a decided position
-      const int bk = bucket_of(key(i), lo, scale);
-      took |= bk > sb ? bit : 0u;
-      act &= bk != sb ? ~bit : ~0u;
+#pragma unroll 2
+    for (int gg = 0; gg < G; ++gg) {
+      const int g = (gg + rotg) & (G - 1);
+      const float4 v = group(g);
+      const int bk[4] = {bucket_of(v.x, lo, scale), bucket_of(v.y, lo, scale), bucket_of(v.z, lo, scale),
+                         bucket_of(v.w, lo, scale)};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t bit = act & (1u << (4 * g + e));  // 0 for a decided position
+        took |= bk[e] > sb ? bit : 0u;
+        act &= bk[e] != sb ? ~bit : ~0u;
+      }
     }
     if (cnt == need) {
       took |= act;
@@ -670,13 +692,13 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
 #pragma unroll 1
       for (uint32_t a = act; a; a &= a - 1, ++slot) {
         const int i = __ffs(a) - 1;
-        sts_v2(SC_ADDR(sc_a, blist) + 8u * slot, __float_as_uint(key(i)), (uint32_t)(j0 + i));
+        sts_v2(SC_ADDR(sc_a, blist) + 8u * slot, lds_u32(keys_a + 4u * (uint32_t)(j0 + i)), (uint32_t)(j0 + i));
       }
       csync();
 #pragma unroll 1
       for (uint32_t a = act; a; a &= a - 1) {
         const int i = __ffs(a) - 1;
-        const float kx = key(i);
+        const float kx = lds_f32(keys_a + 4u * (uint32_t)(j0 + i));
         const int jx = j0 + i;
         uint32_t rank = 0;
 #pragma unroll 1
@@ -715,15 +737,30 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
       e ^= low;
     }
   }
-  // Each winner at its output rank.  The scan's barrier orders every read of
-  // the keys, the histogram and the boundary list before the key array is
+  // Each winner at its output rank, four positions at a time (positions
+  // 4g .. 4g + 3 of the run are the children of the previous selection's
+  // entries (j0 + 4g) / 2 and that + 1).  The scan's barrier orders every read
+  // of the keys, the histogram and the boundary list before the key array is
   // overwritten and the scratch cleared.
   int r = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum) + 32u);
 #pragma unroll 1
-  for (uint32_t a = take; a; a &= a - 1, ++r) {
-    const int j = j0 + __ffs(a) - 1;
-    const int cv = top ? j : 2 * (int)lds_u32(jprev_a + 4u * (uint32_t)(j >> 1)) + (j & 1);
-    sts_u32(keys_a + 4u * (uint32_t)r, (uint32_t)cv);
+  for (int g = 0; g < G; ++g) {
+    const uint32_t t4 = (take >> (4 * g)) & 15u;
+    if (!t4) continue;
+    const int j = j0 + 4 * g;
+    int c[4] = {j, j + 1, j + 2, j + 3};
+    if (!top) {
+      const uint2 pj = lds_v2(jprev_a + 4u * (uint32_t)(j >> 1));
+      c[0] = 2 * (int)pj.x;
+      c[1] = 2 * (int)pj.x + 1;
+      c[2] = 2 * (int)pj.y;
+      c[3] = 2 * (int)pj.y + 1;
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      sts_u32_if((t4 >> e) & 1u, keys_a + 4u * (uint32_t)r, (uint32_t)c[e]);
+      r += (t4 >> e) & 1u;
+    }
   }
 #pragma unroll
   for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
@@ -731,10 +768,11 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
   csync();
 }
 
-// Top-K dispatch: R = the smallest power of two with R NCT >= m (m <= 32 NCT).
+// Top-K dispatch: R = the smallest power of two (at least 4) with R NCT >= m
+// (m <= 32 NCT).
 __device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                             float lo, float hi) {
-  int R = 1;
+  int R = 4;
   while (R * NCT < m) R <<= 1;
   select_keys(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
 }
@@ -816,8 +854,8 @@ __device__ __noinline__ float2 warp_sums_exact(uint32_t tb, int ntl, int mc, flo
 // maximum over all its rows.  The four warps' (m, sum) merge into the CTA's
 // (M, S) per query, which goes to slot `rank` of every cluster CTA's xstat.
 // tpar holds the parity of each tile barrier's next phase.
-__device__ __noinline__ void scale_sums(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
-                                        int ntl, int mc, float sl2, uint32_t& tpar, int* status) {
+__device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
+                                        int ntl, int mc, float sl2, uint32_t ecol, uint32_t& tpar, int* status) {
   const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const f32x2 s2 = pk2(sl2, sl2);
@@ -850,10 +888,17 @@ __device__ __noinline__ void scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
 #pragma unroll
       for (int k = 0; k < 16; ++k) {
         const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
-        acc[k] = add2(acc[k], pk2(ex2(x.x), ex2(x.y)));
+        const float e0 = ex2(x.x), e1 = ex2(x.y);
+        acc[k] = add2(acc[k], pk2(e0, e1));
+        ra[2 * k] = __float_as_uint(e0);
+        ra[2 * k + 1] = __float_as_uint(e1);
       }
     }
+    // The exponentials stay in TMEM for the ranking keys (rows past the
+    // slice store whatever they hold; no key is formed for them).
+    if (ecol) tmem_st32(tb + ecol + lane_base + 32 * t, ra);
   }
+  if (ecol) tmem_wait_st();
   float a[32];
 #pragma unroll
   for (int k = 0; k < 16; ++k) {
@@ -862,7 +907,8 @@ __device__ __noinline__ void scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
     a[2 * k + 1] = v.y;
   }
   float2 st = make_float2(mcol, transpose_reduce32<false>(a, lane));
-  if (__any_sync(0xffffffffu, !(st.y <= 3.0e38f))) st = warp_sums_exact(tb, ntl, mc, sl2);
+  const bool overflow = __any_sync(0xffffffffu, !(st.y <= 3.0e38f));
+  if (overflow) st = warp_sums_exact(tb, ntl, mc, sl2);
   sts_v2(smem_u32(&us.wstat[warp][lane]), __float_as_uint(st.x), __float_as_uint(st.y));
   csync();
   if (tid < 32) {
@@ -886,6 +932,7 @@ __device__ __noinline__ void scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
     for (uint32_t r = 0; r < cs; ++r)
       st_async_v2(map_rank(dst, r), __float_as_uint(M), __float_as_uint(S), map_rank(bar, r));
   }
+  return ecol != 0 && !overflow;  // the stored exponentials are relative to this warp's stabilisers
 }
 
 // Softmax normaliser per query, c_i = M + log2 S over the whole candidate
@@ -908,64 +955,87 @@ __device__ __forceinline__ void warp_normaliser(UnitState& us, uint32_t cs, int 
 #pragma unroll
   for (int r = 0; r < MAXCS; ++r)
     if (r < (int)cs && st[r].y > 0.f) S = fmaf(st[r].y, ex2(st[r].x - M), S);
-  us.cw[warp][lane] = lane < q ? M + lg2(S) : INFINITY;
+  const float c = lane < q ? M + lg2(S) : INFINITY;
+  us.cw[warp][lane] = c;
+  us.fw[warp][lane] = ex2(us.wstat[warp][lane].x - c);  // 0 for padded columns and for a warp without rows
   __syncwarp();
 }
 
-// Ranking key log2 W_j of each valid row (Eq. 8 as a log-sum-exp over the
-// query rows, against the normaliser c_i in the warp's copy us.cw[warp]),
-// stored at position g0 + j of every cluster CTA's key array of the unit;
-// each warp's (min, max) key goes to slot (rank, warp) of every CTA's kmm on
-// the same barrier.  Every exponent
-// l sl2 - c_i is at most 0 (c_i is the log of a sum that contains the row's
-// own term), so the sum of 2^(l sl2 - c_i) cannot overflow and is taken
-// unshifted; padded query columns have c_i = +inf and add 0.  Only if the
-// sum is tiny (below 2^-96, where flushed terms could matter) is it taken
-// again shifted by its largest exponent.
+// Ranking key log2 W_j of each valid row (Eq. 8), stored at position g0 + j
+// of every cluster CTA's key array of the unit; each warp's (min, max) key
+// goes to slot (rank, warp) of every CTA's kmm on the same barrier.
+// With the scale's exponentials e = 2^(l sl2 - m) stored in TMEM at column
+// ecol (eok: the warp's sums used those stabilisers m), W_j = sum_i e_ij f_i
+// with f_i = 2^(m_i - c_i) from us.fw: fused multiply-adds, no exponentials.
+// Otherwise, and for a row whose W is tiny (below 2^-96, where flushed terms
+// could matter), the key is a log-sum-exp of the logits over the query rows
+// against the normaliser c_i (us.cw): every exponent l sl2 - c_i is at most 0
+// (c_i is the log of a sum that contains the row's own term), so the sum
+// cannot overflow; padded query columns have c_i = +inf and add 0; a tiny sum
+// is taken again shifted by its largest exponent.
 __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
-                                       int ntl, int mc, int g0, float sl2, uint32_t keys_a) {
+                                       int ntl, int mc, int g0, float sl2, uint32_t keys_a, uint32_t ecol, bool eok) {
   const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const uint32_t bar = bar_addr(ms.kbar[pp]);
   const f32x2 s2 = pk2(sl2, sl2);
-  f32x2 ncv[16];
-  const uint32_t cw_a = smem_u32(&us.cw[warp][0]);
+  f32x2 ncv[16], fv[16];
+  const uint32_t cw_a = smem_u32(&us.cw[warp][0]), fw_a = smem_u32(&us.fw[warp][0]);
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     const uint4 v = lds_v4(cw_a + 16u * k);
     ncv[2 * k] = pk2(-__uint_as_float(v.x), -__uint_as_float(v.y));
     ncv[2 * k + 1] = pk2(-__uint_as_float(v.z), -__uint_as_float(v.w));
+    const uint4 f = lds_v4(fw_a + 16u * k);
+    fv[2 * k] = pk2(__uint_as_float(f.x), __uint_as_float(f.y));
+    fv[2 * k + 1] = pk2(__uint_as_float(f.z), __uint_as_float(f.w));
   }
   float kmin = INFINITY, kmax = -INFINITY;
 #pragma unroll 1
   for (int t = 0; t < ntl; ++t) {
-    uint32_t ra[32];
-    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
-    tmem_wait_ld();
     const int j = t * TM + tid;
-    f32x2 z2 = pk2(0.f, 0.f);
+    uint32_t ra[32];
+    float key = 0.f;
+    bool slow = true;
+    if (eok) {
+      tmem_ld32_issue(tb + ecol + lane_base + 32 * t, ra);
+      tmem_wait_ld();
+      f32x2 z2 = pk2(0.f, 0.f);
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
-      z2 = add2(z2, pk2(ex2(v.x), ex2(v.y)));
+      for (int k = 0; k < 16; ++k) z2 = fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), fv[k], z2);
+      const float2 zz = up2(z2);
+      key = lg2(zz.x + zz.y);
+      slow = zz.x + zz.y < 0x1p-96f;
     }
-    float2 zz = up2(z2);
-    float key = lg2(zz.x + zz.y);
-    if (zz.x + zz.y < 0x1p-96f) {
-      float mx = -INFINITY;
+    if (__any_sync(0xffffffffu, slow && j < mc)) {  // the whole warp reloads the logits (TMEM loads are warp-wide)
+      tmem_ld32_issue(tb + lane_base + 32 * t, ra);
+      tmem_wait_ld();
+      if (slow) {
+        f32x2 z2 = pk2(0.f, 0.f);
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
-        mx = fmax3(mx, v.x, v.y);
-      }
-      z2 = pk2(0.f, 0.f);
+        for (int k = 0; k < 16; ++k) {
+          const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+          z2 = add2(z2, pk2(ex2(v.x), ex2(v.y)));
+        }
+        float2 zz = up2(z2);
+        key = lg2(zz.x + zz.y);
+        if (zz.x + zz.y < 0x1p-96f) {
+          float mx = -INFINITY;
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
-        z2 = add2(z2, pk2(ex2(v.x - mx), ex2(v.y - mx)));
+          for (int k = 0; k < 16; ++k) {
+            const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+            mx = fmax3(mx, v.x, v.y);
+          }
+          z2 = pk2(0.f, 0.f);
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+            z2 = add2(z2, pk2(ex2(v.x - mx), ex2(v.y - mx)));
+          }
+          zz = up2(z2);
+          key = mx + lg2(zz.x + zz.y);
+        }
       }
-      zz = up2(z2);
-      key = mx + lg2(zz.x + zz.y);
     }
     if (j < mc) {
       kmin = fminf(kmin, key);
@@ -1179,12 +1249,12 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     const int kb = p.keep[lev];
     int32_t* J = unit_J(c, p, pp, lev);  // receives this scale's keys, then its selection
     const uint32_t keys_a = smem_u32(J);
-    scale_sums(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2, tpar, p.status);
+    const bool eok = scale_sums(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2, p.ecol, tpar, p.status);
     wait_cluster_or_abort(bar_addr(ms.xbar[pp]), ph, ms, p.status);
     // This phase is complete for tid 0, so the arrival arms the next one.
     if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
     warp_normaliser(us, c.cs, p.q);
-    pass_keys(c.rank, c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a);
+    pass_keys(c.rank, c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a, p.ecol, eok);
     wait_cluster_or_abort(bar_addr(ms.kbar[pp]), ph, ms, p.status);
     // The keys' range from the cluster warps' (min, max).
     float lo, hi;
@@ -1398,13 +1468,18 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
   const int total = keep[0] + n_g;
   // TMEM columns of one unit's region at cluster size cs: the widest scale
   // slice, or the attention slice plus the O^T accumulator.
-  auto unit_cols = [&](int cs) {
+  // TMEM tiles of the widest scale slice at cluster size cs.
+  auto scale_tiles = [&](int cs) {
     auto slice_tiles = [&](int m) { return (2 * (((m + 1) / 2 + cs - 1) / cs) + TM - 1) / TM; };
     int tmax = slice_tiles(n >> levels);
     for (int l = levels; l >= 1; --l) {
       const int t = slice_tiles(2 * keep[l]);
       tmax = tmax > t ? tmax : t;
     }
+    return tmax;
+  };
+  auto unit_cols = [&](int cs) {
+    int tmax = scale_tiles(cs);
     const int ta = ((total + cs - 1) / cs + TM - 1) / TM + 1;
     tmax = tmax > ta ? tmax : ta;
     return 32 * tmax;
@@ -1441,7 +1516,16 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
   const int P = best.P, cs = best.cs, stages = best.stages;
   const size_t smem = best.smem;
   const int clusters = (U + P - 1) / P;
-  const int ucols = unit_cols(cs);
+  int ucols = unit_cols(cs);
+  // Room for the scale's exponentials beside its logits (the ranking keys
+  // then need no exponentials of their own): the widest scale slice twice.
+  const int stiles = scale_tiles(cs);
+  int ecol = 0;
+  const int ecols = ucols > 64 * stiles ? ucols : 64 * stiles;
+  if (P * ecols <= 512) {
+    ecol = 32 * stiles;
+    ucols = ecols;
+  }
   int cols = 32;
   while (cols < P * ucols) cols *= 2;
   fp.ok = true;
@@ -1451,6 +1535,7 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
   fp.smem = smem;
   fp.tmem_cols = cols;
   fp.ucols = ucols;
+  fp.ecol = ecol;
   fp.cmax = cmax;
   fp.kmax = kmax;
   fp.trim = trim;
@@ -1489,6 +1574,7 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   p.cmax = fp.cmax; p.kmax = fp.kmax;
   p.tmem_cols = (uint32_t)fp.tmem_cols;
   p.ucols = (uint32_t)fp.ucols;
+  p.ecol = (uint32_t)fp.ecol;
   for (int l = 0; l <= levels; ++l) p.keep[l] = keep[l];
   p.scale_log2 = kLog2e / sqrtf((float)D);
 

@@ -135,7 +135,7 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
 // per P units.
 struct FusedPlan {
   bool ok;
-  int cs, P, clusters, stages, tmem_cols, ucols, cmax, kmax, U;
+  int cs, P, clusters, stages, tmem_cols, ucols, ecol, cmax, kmax, U;
   size_t smem;
   bool trim;
 };
