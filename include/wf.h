@@ -265,27 +265,35 @@ wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const
  *
  * Same arguments, semantics and results as wf_sparse_attn, minus ws and
  * ws_bytes.  The split-K scratch comes from one static device array of
- * WF_NOALLOC_SCRATCH_BYTES inside libwf, reserved on every device that loads
- * it until the process exits; the call allocates nothing.
+ * WF_NOALLOC_SCRATCH_BYTES inside libwf, reserved in every CUDA context that
+ * loads the library until that context is destroyed (the runtime's primary
+ * context: until the process exits); the call allocates nothing.
  * - Limit: returns WF_ERR_WORKSPACE, and launches nothing, when the call would
  *   need more than WF_NOALLOC_SCRATCH_BYTES (the need is
  *   wf_attn_workspace_bytes(q, k, n_g); e.g. 32 heads with k + n_g <= 960
  *   rows with head_dim 128 fits).
- * - The first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress, with that device current); make that first call
- *   before any stream capture.  It returns WF_ERR_CUDA if the lookup fails.
- * - All calls on a device share the one array and each call overwrites it:
+ * - Contexts: the array has its own device address in each CUDA context.  The
+ *   first call from a context (the runtime's primary context of the current
+ *   device, or any context the caller made current) looks that address up
+ *   with cudaGetSymbolAddress and caches it under the context's unique id;
+ *   later calls from the same context reuse it.  Make that first call before
+ *   any stream capture.  It returns WF_ERR_CUDA if the lookup fails.
+ * - All calls in a context share the one array and each call overwrites it:
  *   calls whose kernels may overlap on the GPU (other streams, other host
  *   threads) race and corrupt each other's results.  Serialise them, e.g.
- *   on one stream.  No part of the array has to start at zero.
- * - The status word of wf_sparse_attn's workspace lives in the static array
- *   too, so this call cannot report a tensor-core wait that gave up (it
- *   never should); use wf_sparse_attn where that report is needed.
+ *   on one stream.  No part of the array has to start at zero, except the
+ *   status word below (zero when the library loads).
+ * - The array's first word is the status word of the tensor-core kernels: if
+ *   one of their bounded waits gives up (it never should), the output is
+ *   undefined and the word is set.  wf_noalloc_status() waits for `stream`,
+ *   returns WF_ERR_TIMEOUT (and clears the word) if it is set, else WF_OK.
+ *   Synchronising; not for the hot loop.
  * ------------------------------------------------------------------------- */
 #define WF_NOALLOC_SCRATCH_BYTES (16u << 20)
 wf_status wf_sparse_attn_noalloc(const void* Q, const wf_tensor* q, const void* K, const void* V,
                                  const wf_tensor* kv, const int32_t* idx, int k, const void* Kg, const void* Vg,
                                  const wf_tensor* g, void* O, const wf_tensor* o, float scale, void* stream);
+wf_status wf_noalloc_status(void* stream);
 
 /* ---------------------------------------------------------------------------
  * One denoising-step layer (Algorithm 1 body): if refresh_coeffs != 0, first

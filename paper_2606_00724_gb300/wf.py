@@ -57,6 +57,7 @@ SIGNATURES = {
     "wf_sparse_attn": (_I, [_P, _T, _P, _P, _T, _P, _I, _P, _P, _T, _P, _T, ctypes.c_float, _P, _SZ, _P]),
     "wf_step_workspace_bytes": (_SZ, [_T, _T, _I, _P, _I]),
     "wf_sparse_attn_noalloc": (_I, [_P, _T, _P, _P, _T, _P, _I, _P, _P, _T, _P, _T, ctypes.c_float, _P]),
+    "wf_noalloc_status": (_I, [_P]),
     "wf_step": (_I, [_P, _T, _P, _P, _T, _P, _P, _T, _P, _SZ, _I, _I, _P, _P, _P, _P, _T, _P, _SZ, _P]),
     "wf_workspace_status": (_I, [_P, _P]),
 }
@@ -215,7 +216,8 @@ def wf_sparse_attn(Q, K, V, idx, k: int, Kg, Vg, O, ws, scale: float = 0.0, stre
 def wf_sparse_attn_noalloc(Q, K, V, idx, k: int, Kg, Vg, O, scale: float = 0.0, stream=None):
     """wf_sparse_attn for callers that cannot allocate device memory: the
     scratch comes from libwf's fixed static device array
-    (WF_NOALLOC_SCRATCH_BYTES = 16 MiB), shared by every call on a device."""
+    (WF_NOALLOC_SCRATCH_BYTES = 16 MiB), shared by every call in a CUDA
+    context."""
     dq, dk, do = desc(Q), desc(K), desc(O)
     dg = desc(Kg) if Kg is not None else None
     if Vg is not None and Kg is not None and (Vg.stride() != Kg.stride() or Vg.shape != Kg.shape):
@@ -226,6 +228,12 @@ def wf_sparse_attn_noalloc(Q, K, V, idx, k: int, Kg, Vg, O, scale: float = 0.0, 
                                         k, _ptr(Kg), _ptr(Vg), ctypes.byref(dg) if dg is not None else None,
                                         _ptr(O), ctypes.byref(do), float(scale), _stream(stream)),
            "wf_sparse_attn_noalloc")
+
+
+def wf_noalloc_status(stream=None):
+    """Raise WfError(WF_ERR_TIMEOUT) if a bounded device wait of the
+    allocation-free attention gave up since the last check (synchronising)."""
+    _check(lib().wf_noalloc_status(_stream(stream)), "wf_noalloc_status")
 
 
 def wf_step_workspace_bytes(Q: torch.Tensor, K: torch.Tensor, levels: int, keep, n_g: int) -> int:

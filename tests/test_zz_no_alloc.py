@@ -2,6 +2,8 @@
 cannot allocate device memory (its scratch is a fixed static device array
 inside libwf).  Checked through the C ABI against wf_sparse_attn, which uses
 a caller workspace, on two calls in a row.  This file is collected last."""
+import threading
+
 import numpy as np
 import pytest
 import torch
@@ -45,6 +47,35 @@ def test_noalloc_matches_workspace_entry_point(cfg):
                               out2)
     torch.cuda.synchronize()
     assert_close_out(f64(out2), f64(ref2), batch.Q.dtype)
+    # No bounded device wait gave up (the status word in the static array).
+    wf.wf_noalloc_status()
+
+
+def test_noalloc_from_another_host_thread():
+    # Another host thread with the same device current uses the same context
+    # (the runtime's primary context), so it finds the cached scratch address.
+    w, batch, idx = _inputs("c2", 3)
+    ws = torch.zeros(wf.wf_attn_workspace_bytes(batch.Q, w.k, w.ng), dtype=torch.uint8, device="cuda")
+    ref = torch.empty_like(batch.Q)
+    wf.wf_sparse_attn(batch.Q, batch.K, batch.V, idx, w.k, batch.Kg, batch.Vg, ref, ws)
+    out = torch.full_like(batch.Q, float("nan"))
+    torch.cuda.synchronize()
+    errors = []
+
+    def worker():
+        try:
+            torch.cuda.set_device(batch.Q.device)
+            wf.wf_sparse_attn_noalloc(batch.Q, batch.K, batch.V, idx, w.k, batch.Kg, batch.Vg, out)
+            torch.cuda.synchronize()
+        except Exception as e:  # reported in the main thread
+            errors.append(e)
+
+    t = threading.Thread(target=worker)
+    t.start()
+    t.join()
+    assert not errors, errors
+    assert_close_out(f64(out), f64(ref), batch.Q.dtype)
+    wf.wf_noalloc_status()
 
 
 def test_noalloc_rejects_oversized_requests():
