@@ -13,6 +13,10 @@ that must move are the query block, the candidate coefficient rows of every
 scale, the level-0 trim rows, K[mu0] and V[mu0], the generation rows, the
 output block and the index list.  L2 is flushed (256 MiB write) before every
 timed step; each step is timed with CUDA events on the launching stream.
+value and ms_per_step use the mean step time over the K timed steps (the
+whole-job rate); step_us_median is the median of the same steps.  On one
+GPU the default run also measures the 128K-token workload (c4) in the same
+process (10 warm-up steps, median of 50) under the key "c4".
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c3]
                        [--impl reference]
@@ -423,6 +427,30 @@ def run_gpu(args, cfg, rank, world, device):
                 layers=len(layers))
 
 
+def measure_extra(args, cfg, device, hbm_peak, peak_kind):
+    """A second workload measured in the same process: 10 warm-up steps, 50
+    timed steps (L2 flushed before each), median and mean step time, the
+    fused kernel's roofline and the clock record of its own timed region."""
+    import types
+    w = synth.WORKLOADS[cfg]
+    a = types.SimpleNamespace(**vars(args))
+    a.steps, a.warmup = 50, 10
+    r = run_gpu(a, cfg, 0, 1, device)
+    ub = unit_bytes(w)
+    mean_us = r["total_ms"] / a.steps * 1e3
+    med_us = statistics.median(r["step_ms"]) * 1e3
+    bytes_launch = ub["step"] * w.units
+    return {"workload": w.name, "steps": a.steps, "warmup": a.warmup, "step_us_median": med_us,
+            "step_us_mean": mean_us,
+            "roofline": {"bound": "hbm", "achieved": bytes_launch / (med_us * 1e-6) / 1e9, "peak": hbm_peak,
+                         "unit": "GB/s", "frac": bytes_launch / (med_us * 1e-6) / 1e9 / hbm_peak,
+                         "frac_of_mean": bytes_launch / (mean_us * 1e-6) / 1e9 / hbm_peak,
+                         "traffic": recorded_traffic(w) if fused_eligible(w) else None,
+                         "kernel": "wf_fused_kernel" if fused_eligible(w) else "per-stage kernels",
+                         "peak_kind": peak_kind, "bytes_per_launch": bytes_launch},
+            "clocks": r["clocks"]}
+
+
 def main():
     global WAVELET
     ap = argparse.ArgumentParser()
@@ -447,6 +475,8 @@ def main():
                     help="step: the filter + sparse-attention step (the metric); cache-update: wf_cache_update of "
                          "--update-rows rows per unit against a full pyramid rebuild")
     ap.add_argument("--update-rows", type=int, default=32)
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the second workload (c4) that the default single-GPU run also measures")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -530,6 +560,7 @@ def main():
         return
 
     r = run_gpu(args, cfg, rank, world, device)
+    step_us_median = statistics.median(r["step_ms"]) * 1e3
     total_ms = r["total_ms"]
     e2e_ms = r["e2e_ms"]
     total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], device)
@@ -550,10 +581,13 @@ def main():
                 "frac_of_nominal_7900": achieved / 7900.0,
                 "traffic": recorded_traffic(w) if fused_eligible(w) else None, "kernel": kname,
                 "peak_kind": peak_kind,
-                "bytes_per_launch": ub["step"] * w.units, "launch_us": per_layer_ms * 1e3}
+                "bytes_per_launch": ub["step"] * w.units, "launch_us": per_layer_ms * 1e3,
+                "frac_median": (ub["step"] * w.units / (step_us_median / w.layers * 1e-6) / 1e9 / hbm_peak
+                                if not w.refresh_every else None)}
     e2e_bytes_per_step = ub["step"] * w.units
     line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "step_us": ms_per_step * 1e3,
+            "step_us_median": step_us_median,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if (w.dtype == "bf16" and w.head_dim == 128) else "f32",
             "data": "synthetic", "config": config, "roofline": roofline, "clocks": r["clocks"],
@@ -562,6 +596,9 @@ def main():
                     "layers": 1},
             "gpu_launches": launches_per_step(w) * w.layers * args.steps + (
                 w.layers * math.ceil(args.steps / w.refresh_every) if w.refresh_every else 0)}
+    if world == 1 and cfg == DEFAULT_WORKLOAD and not args.no_extra and not (args.batch or args.heads) and \
+            not args.wavelet and args.schedule == "default" and not args.graph:
+        line["c4"] = measure_extra(args, "c4", device, hbm_peak, peak_kind)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         units, secs = oracle_units_seconds(w, cfg, args.cpu_seconds)
         line["cpu_baseline"] = {"value": units * ub["step"] / secs / 1e9, "unit": "GB/s", "cores": 1,

@@ -10,8 +10,13 @@ Every function works on one (batch, head) unit with numpy arrays:
 ``[rows, d]`` row-major matrices, int32 index vectors.  ``keep`` is the kept
 count vector: ``keep[b]`` for scale b = 1..L and ``keep[0]`` = final k.
 
-Parity status of each function (what pins it) is listed in the design notes;
-every function here is pinned by a ``-m "not gpu"`` test.
+Every function here is pinned by ``-m "not gpu"`` tests against facts that do
+not come from the oracle itself: perfect reconstruction, Parseval and the
+closed forms of the Haar and db2 transforms, a hand-worked Haar example and
+Daubechies' published db2 taps (``tests/golden/``), brute-force search over
+all k-subsets for the Top-K, the two-candidate logistic closed form and torch
+softmax for the skim weights, torch's fp64 attention for the sparse
+attention, and Table 3's proportion range for the schedules.
 """
 from __future__ import annotations
 

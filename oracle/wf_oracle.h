@@ -15,8 +15,8 @@
  *   - keep[b] (b = 1..L) is the number of level-b coefficients kept by the
  *     Top-K of Eq. 9 at scale b; keep[0] is the final token count k.
  *
- * Readings of the paper that the oracle fixes are listed in the design notes;
- * the ones visible here: Haar pairs tokens (2j, 2j+1) (forced by the blocks of
+ * Readings of the paper that the oracle fixes, as visible in these
+ * signatures: Haar pairs tokens (2j, 2j+1) (forced by the blocks of
  * Eq. 10); orthonormal Haar taps 1/sqrt(2); the softmax of Eq. 7 runs over the
  * current candidates; W of Eq. 8 sums over the query rows; ties in the Top-K
  * of Eq. 9 go to the lower index; a level-0 trim keeps the top keep[0] tokens
