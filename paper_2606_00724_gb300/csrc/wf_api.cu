@@ -3,7 +3,10 @@
 #include <math.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "wf_internal.cuh"
+#include "wf_testing.h"
 
 #define WF_API extern "C" __attribute__((visibility("default")))
 
@@ -343,5 +346,30 @@ WF_API wf_status wf_workspace_status(void* ws, void* stream) {
       return WF_ERR_CUDA;
     return WF_ERR_TIMEOUT;
   }
+  return WF_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Test-only wait-failure controls (include/wf_testing.h).
+// ---------------------------------------------------------------------------
+namespace {
+std::atomic<int> g_test_stall{0};
+std::atomic<long long> g_test_wait_limit{0};
+}  // namespace
+
+namespace wf {
+WaitControls wait_controls() {
+  WaitControls c;
+  c.stall = g_test_stall.load(std::memory_order_relaxed);
+  const long long lim = g_test_wait_limit.load(std::memory_order_relaxed);
+  c.limit = lim > 0 ? lim : kDefaultWaitLimit;
+  return c;
+}
+}  // namespace wf
+
+WF_API wf_status wf_testing_set_wait_failure(int stall, long long wait_limit_cycles) {
+  if (wait_limit_cycles < 0) return WF_ERR_INVALID_ARG;
+  g_test_wait_limit.store(wait_limit_cycles, std::memory_order_relaxed);
+  g_test_stall.store(stall != 0, std::memory_order_relaxed);
   return WF_OK;
 }

@@ -67,7 +67,6 @@ constexpr int MAXCS_PAD_BYTES = 8 * NQ * 4;  // the ragged head-dim slices of a 
 // at most (D + cs) rows of 32 fp32 when cs does not divide D).
 constexpr int UNIT_P_BYTES = 2 * P_BYTES + MAXCS_PAD_BYTES;
 constexpr int kMaxCand = 32 * NCT;         // largest candidate list the Top-K holds in registers
-constexpr long long kWaitLimit = 1ll << 31;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint32_t kCsyncId = 1;           // named barriers 1, 2: the compute warps of unit 0, 1
 
@@ -93,6 +92,9 @@ struct Misc {
   unsigned long long tdone[MAXP][MAXT];  // scale tile t of a unit scored (one phase per scale)
   unsigned long long pfull[MAXP][2], pempty[MAXP][2], cbar[MAXP], cready[MAXP];
   UnitState us[MAXP];
+  unsigned long long stallbar;  // completed by nothing (the test-only stalled first wait)
+  unsigned long long drainbar;  // the MMA thread's final commit
+  long long wait_limit;         // bound of the waits that can give up (cycles)
   int abort;
   uint32_t tmem_base;
 };
@@ -135,6 +137,8 @@ struct FusedParams {
   int q, n, ng, U, H, L, trim, P, cmax, kmax;
   uint32_t tmem_cols, ucols;  // TMEM allocation; columns per unit region
   uint32_t ecol;              // column of the stored exponentials in a unit region (0: none)
+  long long wait_limit;       // bound of the waits that can give up (cycles)
+  int stall;                  // test-only: the MMA thread's first wait never completes
   int32_t keep[12];
   float scale_log2;           // log2(e) / sqrt(d)
 };
@@ -160,12 +164,13 @@ __device__ __forceinline__ void set_abort(Misc& ms, int* status) {
 }
 
 __device__ __noinline__ void wait_or_abort(uint32_t bar, uint32_t parity, Misc& ms, int* status) {
-  if (!aborted(ms) && !mbar_wait_bounded(bar, parity, kWaitLimit, smem_u32(&ms.abort))) set_abort(ms, status);
+  if (!aborted(ms) && !mbar_wait_bounded(bar, parity, ms.wait_limit, smem_u32(&ms.abort))) set_abort(ms, status);
 }
 
 // Wait for a phase completed by other CTAs of the cluster (acquire, cluster scope).
 __device__ __noinline__ void wait_cluster_or_abort(uint32_t bar, uint32_t parity, Misc& ms, int* status) {
-  if (!aborted(ms) && !mbar_wait_cluster_bounded(bar, parity, kWaitLimit, smem_u32(&ms.abort))) set_abort(ms, status);
+  if (!aborted(ms) && !mbar_wait_cluster_bounded(bar, parity, ms.wait_limit, smem_u32(&ms.abort)))
+    set_abort(ms, status);
 }
 
 __device__ __forceinline__ uint32_t bar_addr(const unsigned long long& b) { return smem_u32(&b); }
@@ -379,6 +384,9 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
     produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, attn_src(c, p, pp, true, a0, mc), pt);
     it += ntl;
   }
+  // Copies still in flight (only after a wait gave up) land before the CTA
+  // can leave.
+  cp_async_wait_all();
 }
 
 // ---------------------------------------------------------------------------
@@ -438,7 +446,7 @@ __device__ __forceinline__ void mma_pv(const Ctx& c, const FusedParams& p, int p
 }
 
 template <int S>
-__device__ void mma_role(const Ctx& c, const FusedParams& p) {
+__device__ void mma_role_body(const Ctx& c, const FusedParams& p) {
   Misc& ms = *c.ms;
   int it = 0;
   for (int lev = p.L; lev >= c.lev_end; --lev) {
@@ -464,6 +472,18 @@ __device__ void mma_role(const Ctx& c, const FusedParams& p) {
     it += ntl;
     mma_commit(bar_addr(ms.mdone[pp]));
   }
+}
+
+// The MMA thread: an optional stalled first wait (test-only), the MMAs, then
+// a commit that it waits for (default bound), so that no MMA is still
+// writing TMEM when it is freed, also after a wait gave up.
+template <int S>
+__device__ void mma_role(const Ctx& c, const FusedParams& p) {
+  Misc& ms = *c.ms;
+  if (p.stall) wait_or_abort(bar_addr(ms.stallbar), 0u, ms, p.status);
+  mma_role_body<S>(c, p);
+  mma_commit(bar_addr(ms.drainbar));
+  (void)mbar_wait_bounded(bar_addr(ms.drainbar), 0u, kDefaultWaitLimit);
 }
 
 // ---------------------------------------------------------------------------
@@ -577,7 +597,9 @@ __device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, i
     const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += t;
   }
-  const int lc = __ffs(__ballot_sync(0xffffffffu, incl >= need)) - 1;
+  // Some lane always qualifies (need never exceeds the keys counted); the
+  // clamp only keeps the reads in the histogram should a wait have given up.
+  const int lc = max(0, __ffs(__ballot_sync(0xffffffffu, incl >= need)) - 1);
   const uint32_t above = __shfl_sync(0xffffffffu, incl - tot, lc);
   const int bb = NB - 1 - 64 * lc - 2 * lane;                 // this lane's buckets bb and bb - 1
   const uint2 pr = lds_v2(hist_a + 4u * (uint32_t)(bb - 1));  // .x = bucket bb - 1, .y = bucket bb
@@ -588,7 +610,7 @@ __device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, i
     const uint32_t t = __shfl_up_sync(0xffffffffu, inc2, o);
     if (lane >= o) inc2 += t;
   }
-  const int l2 = __ffs(__ballot_sync(0xffffffffu, above + inc2 >= need)) - 1;
+  const int l2 = max(0, __ffs(__ballot_sync(0xffffffffu, above + inc2 >= need)) - 1);
   const uint32_t before = above + inc2 - pair;
   const bool upper = before + pr.y >= need;
   const uint32_t b = upper ? (uint32_t)bb : (uint32_t)(bb - 1);
@@ -692,7 +714,10 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
 #pragma unroll 1
       for (uint32_t a = act; a; a &= a - 1, ++slot) {
         const int i = __ffs(a) - 1;
-        sts_v2(SC_ADDR(sc_a, blist) + 8u * slot, lds_u32(keys_a + 4u * (uint32_t)(j0 + i)), (uint32_t)(j0 + i));
+        // slot < NCT always (the list holds cnt <= NCT keys); the predicate
+        // keeps the store in the list should a wait have given up.
+        sts_v2_if(slot < (uint32_t)NCT, SC_ADDR(sc_a, blist) + 8u * slot, lds_u32(keys_a + 4u * (uint32_t)(j0 + i)),
+                  (uint32_t)(j0 + i));
       }
       csync();
 #pragma unroll 1
@@ -758,7 +783,9 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
     }
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      sts_u32_if((t4 >> e) & 1u, keys_a + 4u * (uint32_t)r, (uint32_t)c[e]);
+      // r < kk <= m always; the bound keeps the store in the array should a
+      // wait have given up.
+      sts_u32_if(((t4 >> e) & 1u) && (uint32_t)r < (uint32_t)m, keys_a + 4u * (uint32_t)r, (uint32_t)c[e]);
       r += (t4 >> e) & 1u;
     }
   }
@@ -928,8 +955,10 @@ __device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
       if (w[k].y > 0.f) S = fmaf(w[k].y, ex2(w[k].x - M), S);
     const uint32_t dst = smem_u32(&us.xstat[rank][tid]);
     const uint32_t bar = bar_addr(ms.xbar[pp]);
+    // After a wait gave up, this CTA sends nothing to the cluster.
+    const uint32_t nr = aborted(ms) ? 0u : cs;
 #pragma unroll 1
-    for (uint32_t r = 0; r < cs; ++r)
+    for (uint32_t r = 0; r < nr; ++r)
       st_async_v2(map_rank(dst, r), __float_as_uint(M), __float_as_uint(S), map_rank(bar, r));
   }
   return ecol != 0 && !overflow;  // the stored exponentials are relative to this warp's stabilisers
@@ -973,76 +1002,103 @@ __device__ __forceinline__ void warp_normaliser(UnitState& us, uint32_t cs, int 
 // (c_i is the log of a sum that contains the row's own term), so the sum
 // cannot overflow; padded query columns have c_i = +inf and add 0; a tiny sum
 // is taken again shifted by its largest exponent.
-__device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
-                                       int ntl, int mc, int g0, float sl2, uint32_t keys_a, uint32_t ecol, bool eok) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  const uint32_t bar = bar_addr(ms.kbar[pp]);
+// The exact key of one row from its logits (the slow path of pass_keys):
+// the log-sum-exp over the query rows of l sl2 - c_i, with c_i at cw_a
+// (+inf for padded columns); a tiny sum is taken again shifted by its largest
+// exponent.
+__device__ __forceinline__ float key_from_logits(const uint32_t (&ra)[32], uint32_t cw_a, float sl2) {
   const f32x2 s2 = pk2(sl2, sl2);
-  f32x2 ncv[16], fv[16];
-  const uint32_t cw_a = smem_u32(&us.cw[warp][0]), fw_a = smem_u32(&us.fw[warp][0]);
+  f32x2 ncv[16];
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     const uint4 v = lds_v4(cw_a + 16u * k);
     ncv[2 * k] = pk2(-__uint_as_float(v.x), -__uint_as_float(v.y));
     ncv[2 * k + 1] = pk2(-__uint_as_float(v.z), -__uint_as_float(v.w));
-    const uint4 f = lds_v4(fw_a + 16u * k);
-    fv[2 * k] = pk2(__uint_as_float(f.x), __uint_as_float(f.y));
-    fv[2 * k + 1] = pk2(__uint_as_float(f.z), __uint_as_float(f.w));
   }
+  f32x2 z2 = pk2(0.f, 0.f);
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+    z2 = add2(z2, pk2(ex2(v.x), ex2(v.y)));
+  }
+  float2 zz = up2(z2);
+  float key = lg2(zz.x + zz.y);
+  if (zz.x + zz.y < 0x1p-96f) {
+    float mx = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+      mx = fmax3(mx, v.x, v.y);
+    }
+    z2 = pk2(0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
+      z2 = add2(z2, pk2(ex2(v.x - mx), ex2(v.y - mx)));
+    }
+    zz = up2(z2);
+    key = mx + lg2(zz.x + zz.y);
+  }
+  return key;
+}
+
+__device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
+                                       int ntl, int mc, int g0, float sl2, uint32_t keys_a, uint32_t ecol, bool eok) {
+  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  const uint32_t bar = bar_addr(ms.kbar[pp]);
+  const uint32_t cw_a = smem_u32(&us.cw[warp][0]);
   float kmin = INFINITY, kmax = -INFINITY;
+  // After a wait gave up, this CTA sends nothing to the cluster.
+  const uint32_t nr = aborted(ms) ? 0u : cs;
+  auto emit = [&](int j, float key) {
+    if (j < mc) {
+      kmin = fminf(kmin, key);
+      kmax = fmaxf(kmax, key);
+      const uint32_t dst = keys_a + 4u * (uint32_t)(g0 + j);
 #pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
-    const int j = t * TM + tid;
-    uint32_t ra[32];
-    float key = 0.f;
-    bool slow = true;
-    if (eok) {
+      for (uint32_t r = 0; r < nr; ++r) st_async_b32(map_rank(dst, r), __float_as_uint(key), map_rank(bar, r));
+    }
+  };
+  if (eok) {
+    f32x2 fv[16];
+    const uint32_t fw_a = smem_u32(&us.fw[warp][0]);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const uint4 f = lds_v4(fw_a + 16u * k);
+      fv[2 * k] = pk2(__uint_as_float(f.x), __uint_as_float(f.y));
+      fv[2 * k + 1] = pk2(__uint_as_float(f.z), __uint_as_float(f.w));
+    }
+#pragma unroll 1
+    for (int t = 0; t < ntl; ++t) {
+      uint32_t ra[32];
       tmem_ld32_issue(tb + ecol + lane_base + 32 * t, ra);
       tmem_wait_ld();
       f32x2 z2 = pk2(0.f, 0.f);
 #pragma unroll
       for (int k = 0; k < 16; ++k) z2 = fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), fv[k], z2);
       const float2 zz = up2(z2);
-      key = lg2(zz.x + zz.y);
-      slow = zz.x + zz.y < 0x1p-96f;
+      float key = lg2(zz.x + zz.y);
+      const int j = t * TM + tid;
+      const bool slow = zz.x + zz.y < 0x1p-96f;
+      if (__any_sync(0xffffffffu, slow && j < mc)) {
+        // A tiny W: the exact key from the logits (the whole warp reloads them;
+        // TMEM loads are warp-wide).
+        uint32_t sa[32];
+        tmem_ld32_issue(tb + lane_base + 32 * t, sa);
+        tmem_wait_ld();
+        const float k2 = key_from_logits(sa, cw_a, sl2);
+        key = slow ? k2 : key;
+      }
+      emit(j, key);
     }
-    if (__any_sync(0xffffffffu, slow && j < mc)) {  // the whole warp reloads the logits (TMEM loads are warp-wide)
+  } else {
+#pragma unroll 1
+    for (int t = 0; t < ntl; ++t) {
+      uint32_t ra[32];
       tmem_ld32_issue(tb + lane_base + 32 * t, ra);
       tmem_wait_ld();
-      if (slow) {
-        f32x2 z2 = pk2(0.f, 0.f);
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
-          z2 = add2(z2, pk2(ex2(v.x), ex2(v.y)));
-        }
-        float2 zz = up2(z2);
-        key = lg2(zz.x + zz.y);
-        if (zz.x + zz.y < 0x1p-96f) {
-          float mx = -INFINITY;
-#pragma unroll
-          for (int k = 0; k < 16; ++k) {
-            const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
-            mx = fmax3(mx, v.x, v.y);
-          }
-          z2 = pk2(0.f, 0.f);
-#pragma unroll
-          for (int k = 0; k < 16; ++k) {
-            const float2 v = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, ncv[k]));
-            z2 = add2(z2, pk2(ex2(v.x - mx), ex2(v.y - mx)));
-          }
-          zz = up2(z2);
-          key = mx + lg2(zz.x + zz.y);
-        }
-      }
-    }
-    if (j < mc) {
-      kmin = fminf(kmin, key);
-      kmax = fmaxf(kmax, key);
-      const uint32_t dst = keys_a + 4u * (uint32_t)(g0 + j);
-#pragma unroll 1
-      for (uint32_t r = 0; r < cs; ++r) st_async_b32(map_rank(dst, r), __float_as_uint(key), map_rank(bar, r));
+      emit(t * TM + tid, key_from_logits(ra, cw_a, sl2));
     }
   }
   // The warp's key range goes with the keys (the Top-K's first bucket range).
@@ -1051,7 +1107,7 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, Uni
   if (lane == 0) {
     const uint32_t dst = smem_u32(&us.kmm[rank][warp]);
 #pragma unroll 1
-    for (uint32_t r = 0; r < cs; ++r)
+    for (uint32_t r = 0; r < nr; ++r)
       st_async_v2(map_rank(dst, r), __float_as_uint(kmin), __float_as_uint(kmax), map_rank(bar, r));
   }
   // Every TMEM read of the scale is done before the Top-K's barriers.
@@ -1139,12 +1195,15 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
   tmem_wait_ld();
   const uint32_t ready = bar_addr(ms.cready[pp]);
   // One arrival per CTA, each from its own thread (every thread has seen
-  // this unit's PV products complete), so the remote arrivals overlap.
-  if (tid < (int)cs) mbar_arrive_cluster(map_rank(ready, (uint32_t)tid));
+  // this unit's PV products complete), so the remote arrivals overlap.  A CTA
+  // whose wait gave up announces nothing and sends nothing: its P buffers
+  // may still be in use, and the partials of others must not land there.
+  if (tid < (int)cs && !aborted(ms)) mbar_arrive_cluster(map_rank(ready, (uint32_t)tid));
   wait_cluster_or_abort(ready, 0u, ms, p.status);
   const uint32_t comb_a = smem_u32(comb);
   const uint32_t cbar = bar_addr(ms.cbar[pp]);
-  {
+  const bool send = !aborted(ms);  // every owner has announced its buffers free
+  if (send) {
     // Owner of head-dim row d = tid, and the row's place in its buffer.
     int owner = tid * (int)cs / D;
     while (owner + 1 < (int)cs && dlo(owner + 1, cs) <= tid) ++owner;
@@ -1155,7 +1214,7 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
 #pragma unroll
     for (int i = 0; i < 32; i += 4) st_async_v4(dst + 4u * i, orow[i], orow[i + 1], orow[i + 2], orow[i + 3], rb);
   }
-  if (tid < 32) {
+  if (tid < 32 && send) {
     const uint32_t dst = smem_u32(&us.cstat[rank][tid]);
 #pragma unroll 1
     for (uint32_t r = 0; r < cs; ++r)
@@ -1252,7 +1311,10 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     const bool eok = scale_sums(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2, p.ecol, tpar, p.status);
     wait_cluster_or_abort(bar_addr(ms.xbar[pp]), ph, ms, p.status);
     // This phase is complete for tid 0, so the arrival arms the next one.
-    if (tid == 0 && lev > c.lev_end) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
+    // After a wait gave up the phase may still be pending (its bytes never
+    // came): a second arrival would then underflow the phase's arrival
+    // count, so an aborted CTA arms nothing.
+    if (tid == 0 && lev > c.lev_end && !aborted(ms)) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
     warp_normaliser(us, c.cs, p.q);
     pass_keys(c.rank, c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a, p.ecol, eok);
     wait_cluster_or_abort(bar_addr(ms.kbar[pp]), ph, ms, p.status);
@@ -1271,7 +1333,7 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     // Eq. 9: Top-K (the same result in every CTA of the cluster).
     select_topk(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a, lo, hi);
     if (tid == 0) {
-      if (lev > c.lev_end)
+      if (lev > c.lev_end && !aborted(ms))  // as for xbar above
         mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, lev - 1) + c.cs * NCW * 8u);
       mbar_arrive(bar_addr(ms.jready[pp]));  // the selection is complete (the Top-K ends on a barrier)
     }
@@ -1344,6 +1406,9 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
       mbar_init(bar_addr(ms.cbar[pp]), 1);
       mbar_init(bar_addr(ms.cready[pp]), c.cs);
     }
+    mbar_init(bar_addr(ms.stallbar), 1);
+    mbar_init(bar_addr(ms.drainbar), 1);
+    ms.wait_limit = p.wait_limit;
     ms.abort = 0;
     fence_mbar_init();
     // Arm the first phase of every receive barrier (bytes this CTA expects).
@@ -1399,6 +1464,15 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   cluster_arrive();
   cluster_wait();
   if (warp == MMA_WARP) {
+    if (aborted(ms)) {
+      // After a wait gave up, asynchronous stores from cluster CTAs that were
+      // not waited for may still be landing in this CTA's shared memory:
+      // every CTA has issued its last one (all are past the cluster
+      // barrier), so a short pause lets them complete before the CTA leaves.
+      const unsigned long long t0 = globaltimer_ns();
+      while (globaltimer_ns() - t0 < 20000ull) {
+      }
+    }
     tc_fence_after();
     tmem_dealloc(c.tmem, p.tmem_cols);
   }
@@ -1575,6 +1649,9 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   p.tmem_cols = (uint32_t)fp.tmem_cols;
   p.ucols = (uint32_t)fp.ucols;
   p.ecol = (uint32_t)fp.ecol;
+  const WaitControls wc = wait_controls();
+  p.wait_limit = wc.limit;
+  p.stall = wc.stall;
   for (int l = 0; l <= levels; ++l) p.keep[l] = keep[l];
   p.scale_log2 = kLog2e / sqrtf((float)D);
 

@@ -148,4 +148,14 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Bounds of the tensor-core kernels' waits.  The default, about one second of
+// SM clock cycles, can be lowered (and a stalled first wait requested) only
+// through the test-only wf_testing_set_wait_failure.
+constexpr long long kDefaultWaitLimit = 1ll << 31;
+struct WaitControls {
+  int stall;        // the first wait of each CTA waits on a barrier that nothing completes
+  long long limit;  // bound of the waits that can give up, in cycles
+};
+WaitControls wait_controls();
+
 }  // namespace wf

@@ -227,6 +227,13 @@ __device__ __forceinline__ bool abort_set(uint32_t abort_a) {
   asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(abort_a) : "memory");
   return v != 0;
 }
+// Global nanosecond timer.
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
 // Bounded wait for the phase with the given parity: gives up after about
 // `limit` clock cycles, or as soon as the abort word becomes non-zero, and
 // returns false.

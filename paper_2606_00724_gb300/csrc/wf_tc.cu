@@ -347,6 +347,8 @@ struct TcAttnArgs {
   int qstride;
   int* status;
   float sl2;
+  long long wait_limit;  // bound of the waits that can give up (cycles)
+  int stall;             // test-only: the wait on the score MMAs uses a barrier nothing completes
 };
 
 __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ TcAttnArgs a) {
@@ -360,8 +362,8 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [NWG][4][32]
   float* cm = red + NWG * 4 * 32;              // [256] split max per query (log2 units)
   float* cl = cm + 256;                        // [256] split row sums of P
-  unsigned long long* bar = reinterpret_cast<unsigned long long*>(cl + 256);  // [2]
-  uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 2);
+  unsigned long long* bar = reinterpret_cast<unsigned long long*>(cl + 256);  // [3]: S done, PV done, stall
+  uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 3);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int wg = tid >> 7, wt = tid & 127, quarter = warp & 3;
   const int sp = blockIdx.x, u = blockIdx.y;
@@ -377,6 +379,7 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   if (tid == 0) {
     mbar_init(smem_u32(&bar[0]), 1);
     mbar_init(smem_u32(&bar[1]), 1);
+    mbar_init(smem_u32(&bar[2]), 1);
     fence_mbar_init();
   }
   // K and V rows of the split: chunk c = tid % 16 of rows r0 + 16 i
@@ -443,8 +446,9 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     mma_commit(smem_u32(&bar[0]));
   }
   __syncwarp();
-  bool ok = mbar_wait_bounded(smem_u32(&bar[0]), 0u, kWait);
+  bool ok = mbar_wait_bounded(smem_u32(&bar[a.stall ? 2 : 0]), 0u, a.wait_limit);
   if (!ok) {
+    // Drain the score MMAs (default bound) before the TMEM is freed.
     atomicExch(a.status, 1);
     (void)mbar_wait_bounded(smem_u32(&bar[0]), 0u, kWait);
   }
@@ -504,7 +508,7 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
       mma_commit(smem_u32(&bar[1]));
     }
     __syncwarp();
-    bool ok2 = mbar_wait_bounded(smem_u32(&bar[1]), 0u, kWait);
+    bool ok2 = mbar_wait_bounded(smem_u32(&bar[1]), 0u, a.wait_limit);
     if (!ok2) {
       atomicExch(a.status, 1);
       (void)mbar_wait_bounded(smem_u32(&bar[1]), 0u, kWait);
@@ -583,6 +587,9 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   a.qstride = kMaxQ;
   a.status = status;
   a.sl2 = 1.4426950408889634f * scale;
+  const WaitControls wc = wait_controls();
+  a.wait_limit = wc.limit;
+  a.stall = wc.stall;
   size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 512) + 32;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;

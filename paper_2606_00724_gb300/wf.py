@@ -60,6 +60,8 @@ SIGNATURES = {
     "wf_noalloc_status": (_I, [_P]),
     "wf_step": (_I, [_P, _T, _P, _P, _T, _P, _P, _T, _P, _SZ, _I, _I, _P, _P, _P, _P, _T, _P, _SZ, _P]),
     "wf_workspace_status": (_I, [_P, _P]),
+    # include/wf_testing.h (test-only)
+    "wf_testing_set_wait_failure": (_I, [_I, ctypes.c_longlong]),
 }
 
 
@@ -258,3 +260,11 @@ def wf_workspace_status(ws: torch.Tensor, stream=None):
     """Raise WfError(WF_ERR_TIMEOUT) if a bounded device wait of the fused
     step kernel gave up since the last check (synchronising)."""
     _check(lib().wf_workspace_status(_ptr(ws), _stream(stream)), "wf_workspace_status")
+
+
+def wf_testing_set_wait_failure(stall: bool, wait_limit_cycles: int = 0):
+    """Test-only (include/wf_testing.h): make the tensor-core kernels' first
+    wait stall (a barrier nothing completes) and bound the waits that can give
+    up by wait_limit_cycles (0: the default bound).  Reset with (False, 0)."""
+    _check(lib().wf_testing_set_wait_failure(int(bool(stall)), int(wait_limit_cycles)),
+           "wf_testing_set_wait_failure")

@@ -217,3 +217,10 @@ def test_wavelet_rejects(lib):
     assert lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1) > \
         lib.wf_filter_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep)
     assert lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 5) == 0
+
+
+def test_wait_failure_control(lib):
+    # Test-only control (include/wf_testing.h): host-side only, no launch.
+    assert lib.wf_testing_set_wait_failure(0, -1) == -1  # WF_ERR_INVALID_ARG
+    assert lib.wf_testing_set_wait_failure(1, 1000) == 0
+    assert lib.wf_testing_set_wait_failure(0, 0) == 0

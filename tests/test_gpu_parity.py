@@ -47,8 +47,10 @@ def test_small_configs_all_units(cfg):
 
 @pytest.mark.parametrize("cfg", ["c3", "c4", "c5"])
 def test_full_size_sampled_units(cfg):
-    # Full-size layer in the launch configuration the benchmark times; the
-    # oracle checks a few units (first, last, one in between).
+    # Full-size layer through the per-stage kernels (wf_dwt_build, wf_filter,
+    # wf_sparse_attn; the fused kernel that the benchmark times is checked in
+    # test_gpu_step.py); the oracle checks a few units (first, last, one in
+    # between).
     w = synth.WORKLOADS[cfg]
     units = [0, w.units // 2 + 3, w.units - 1]
     w, batch = make_layer(cfg, units=None)

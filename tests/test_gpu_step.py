@@ -43,6 +43,35 @@ def test_step_full_size(cfg):
     idx = run.idx.cpu().numpy()
     for u in range(w.units):
         assert np.array_equal(idx[u], batch.targets[u][0].cpu().numpy()), f"unit {u} planted"
+    # Every unit's output against the oracle's attention over the kernel's
+    # own indices (the selection itself is checked above).
+    for u in range(w.units):
+        b, h = divmod(u, w.heads)
+        Q, K, V, Kg, Vg = (f64(t[b, h]) for t in (batch.Q, batch.K, batch.V, batch.Kg, batch.Vg))
+        assert_close_out(f64(run.O[b, h]), oracle.sparse_attn(Q, K, V, idx[u], Kg, Vg), torch.bfloat16)
+
+
+@pytest.mark.parametrize("cfg", ["c3", "c4"])
+def test_step_unplanted_timing_inputs(cfg):
+    # The distributions the benchmark times (c3: clustered keys, c4: keys with
+    # a low-frequency drift), without planted margins: every sampled unit's
+    # selection must be a valid Top-K at every scale (near-ties allow several
+    # answers) and its output must match the oracle's attention over the
+    # kernel's own indices.
+    w, batch = make_layer(cfg, planted=False)
+    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).step()
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    for u in [0, 5, w.units // 2 + 1, w.units - 1]:
+        b, h = divmod(u, w.heads)
+        Q, K, V, Kg, Vg = (f64(t[b, h]) for t in (batch.Q, batch.K, batch.V, batch.Kg, batch.Vg))
+        pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, True).astype(np.float64)
+        assert np.array_equal(run.pyramid(u), pyr), f"pyramid unit {u}"
+        gsets = run.level_sets(u)
+        eps_valid(Q, pyr, K, w.n, w.levels, w.keep, gsets)
+        idx = run.idx[u].cpu().numpy()
+        assert np.array_equal(idx, gsets[0])
+        assert_close_out(f64(run.O[b, h]), oracle.sparse_attn(Q, K, V, idx, Kg, Vg), torch.bfloat16)
 
 
 def test_step_matches_per_stage_kernels():
