@@ -66,7 +66,7 @@ constexpr int MAXCS_PAD_BYTES = 8 * NQ * 4;  // the ragged head-dim slices of a 
 // (the partial O rows of this CTA's head-dim slice from every cluster CTA:
 // at most (D + cs) rows of 32 fp32 when cs does not divide D).
 constexpr int UNIT_P_BYTES = 2 * P_BYTES + MAXCS_PAD_BYTES;
-constexpr int kMaxCand = 32 * NCT;         // largest candidate list the Top-K holds in registers
+constexpr int kMaxCand = 64 * NCT;         // largest candidate list of the Top-K (64 keys a thread)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint32_t kCsyncId = 1;           // named barriers 1, 2: the compute warps of unit 0, 1
 
@@ -552,14 +552,21 @@ __device__ __forceinline__ int bucket_of(float v, float lo, float scale) {
   return min(NB - 1, __float_as_int(__fadd_rd(x, 8388608.f)) - 0x4B000000);
 }
 
+// Bit counts of the Top-K's position masks (32 or 64 positions a thread).
+__device__ __forceinline__ int popc_m(uint32_t x) { return __popc(x); }
+__device__ __forceinline__ int popc_m(unsigned long long x) { return __popcll(x); }
+__device__ __forceinline__ int ffs_m(uint32_t x) { return __ffs(x); }
+__device__ __forceinline__ int ffs_m(unsigned long long x) { return __ffsll((long long)x); }
+
 // (min, max) of the undecided keys (bit i of act: position j0 + i of the key
 // array) over the compute threads, via slot `par`.
-__device__ __forceinline__ float2 cta_minmax(uint32_t keys_a, int j0, uint32_t act, uint32_t sc_a, int par) {
+template <typename MT>
+__device__ __forceinline__ float2 cta_minmax(uint32_t keys_a, int j0, MT act, uint32_t sc_a, int par) {
   const int lane = threadIdx.x & 31, warp = ctid() >> 5;
   float lo = INFINITY, hi = -INFINITY;
 #pragma unroll 1
-  for (uint32_t a = act; a; a &= a - 1) {
-    const float v = lds_f32(keys_a + 4u * (uint32_t)(j0 + __ffs(a) - 1));
+  for (MT a = act; a; a &= a - 1) {
+    const float v = lds_f32(keys_a + 4u * (uint32_t)(j0 + ffs_m(a) - 1));
     lo = fminf(lo, v);
     hi = fmaxf(hi, v);
   }
@@ -626,7 +633,8 @@ __device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, i
 // 2 J[j/2] + j%2 with J the previous selection at jprev_a (Eq. 10).
 // [lo, hi] is the range of the keys (sent along with them).
 // Each thread owns the run of R positions j0 = tid R .. j0 + R - 1 (R a power
-// of two, 4 to 32), with one bit per position for "undecided" and "taken".
+// of two, 4 to 64), with one bit per position for "undecided" and "taken" in
+// a mask of type MT (32 bits up to R = 32, else 64).
 // The keys stay in shared memory; every pass re-reads them four at a time
 // (16-byte loads, the G = R / 4 groups of a run visited in a lane-rotated
 // order so that the 8 lanes of a quarter warp hit distinct banks).  Each
@@ -638,15 +646,17 @@ __device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, i
 // (key, -position) against the bucket's list; a larger one is bucketed again
 // over its own range.  If only equal keys remain, the lowest positions are
 // taken.
+template <typename MT>
 __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                          float lo, float hi, int R) {
+  constexpr int MB = 8 * (int)sizeof(MT);       // positions a mask holds
   const int tid = ctid(), lane = tid & 31;
   const int j0 = tid * R;
   const int G = R >> 2;                         // groups of four keys in a run
   const int rotg = ((lane * G) >> 3) & (G - 1);  // first group this lane visits
   const int nv = max(0, min(R, m - j0));        // valid positions of the run
   const uint32_t m4 = (uint32_t)((m + 3) & ~3);  // the key array holds m4 >= 4 words
-  uint32_t act = nv >= 32 ? 0xffffffffu : (1u << nv) - 1u, took = 0;
+  MT act = nv >= MB ? ~(MT)0 : (((MT)1 << nv) - 1), took = 0;
   // The four keys of group g (clamped into the array; positions past m are
   // never undecided).
   auto group = [&](int g) {
@@ -665,7 +675,7 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
     for (int gg = 0; gg < G; ++gg) {
       const int g = (gg + rotg) & (G - 1);
       const float4 v = group(g);
-      const uint32_t a4 = act >> (4 * g);
+      const uint32_t a4 = (uint32_t)(act >> (4 * g));
       const int b0 = bucket_of(v.x, lo, scale), b1 = bucket_of(v.y, lo, scale);
       const int b2 = bucket_of(v.z, lo, scale), b3 = bucket_of(v.w, lo, scale);
       reds_add_if(a4 & 1u, hist_a + 4u * b0, 1u);
@@ -686,9 +696,9 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
                          bucket_of(v.w, lo, scale)};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const uint32_t bit = act & (1u << (4 * g + e));  // 0 for a decided position
-        took |= bk[e] > sb ? bit : 0u;
-        act &= bk[e] != sb ? ~bit : ~0u;
+        const MT bit = act & ((MT)1 << (4 * g + e));  // 0 for a decided position
+        took |= bk[e] > sb ? bit : (MT)0;
+        act &= bk[e] != sb ? ~bit : ~(MT)0;
       }
     }
     if (cnt == need) {
@@ -700,7 +710,7 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
     if (cnt <= (uint32_t)NCT) {
       // Append the boundary keys (one atomic per warp), then every owner
       // ranks its own keys against the list.
-      const int nb = __popc(act);
+      const int nb = popc_m(act);
       int incl = nb;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -712,8 +722,8 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
       wbase = __shfl_sync(0xffffffffu, wbase, 31);
       uint32_t slot = wbase + (uint32_t)(incl - nb);
 #pragma unroll 1
-      for (uint32_t a = act; a; a &= a - 1, ++slot) {
-        const int i = __ffs(a) - 1;
+      for (MT a = act; a; a &= a - 1, ++slot) {
+        const int i = ffs_m(a) - 1;
         // slot < NCT always (the list holds cnt <= NCT keys); the predicate
         // keeps the store in the list should a wait have given up.
         sts_v2_if(slot < (uint32_t)NCT, SC_ADDR(sc_a, blist) + 8u * slot, lds_u32(keys_a + 4u * (uint32_t)(j0 + i)),
@@ -721,8 +731,8 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
       }
       csync();
 #pragma unroll 1
-      for (uint32_t a = act; a; a &= a - 1) {
-        const int i = __ffs(a) - 1;
+      for (MT a = act; a; a &= a - 1) {
+        const int i = ffs_m(a) - 1;
         const float kx = lds_f32(keys_a + 4u * (uint32_t)(j0 + i));
         const int jx = j0 + i;
         uint32_t rank = 0;
@@ -737,7 +747,7 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
             rank += (v0 + k < cnt) && ((ko > kx) || (ko == kx && (int)o[k].y < jx));
           }
         }
-        if (rank < need) took |= 1u << i;
+        if (rank < need) took |= (MT)1 << i;
       }
       act = 0;
       resolved = true;
@@ -751,13 +761,13 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
     lo = lh.x;
     hi = lh.y;
   }
-  uint32_t take = took;
+  MT take = took;
   if (!resolved) {
     // Only equal keys are undecided: the first `need` by position are taken.
-    const int eq_base = cta_excl_scan(__popc(act), SC_ADDR(sc_a, wsum) + 48u);
+    const int eq_base = cta_excl_scan(popc_m(act), SC_ADDR(sc_a, wsum) + 48u);
     int remaining = (int)need - eq_base;
-    for (uint32_t e = act; e && remaining > 0; --remaining) {
-      const uint32_t low = e & (~e + 1u);
+    for (MT e = act; e && remaining > 0; --remaining) {
+      const MT low = e & (~e + 1);
       take |= low;
       e ^= low;
     }
@@ -767,10 +777,10 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
   // entries (j0 + 4g) / 2 and that + 1).  The scan's barrier orders every read
   // of the keys, the histogram and the boundary list before the key array is
   // overwritten and the scratch cleared.
-  int r = cta_excl_scan(__popc(take), SC_ADDR(sc_a, wsum) + 32u);
+  int r = cta_excl_scan(popc_m(take), SC_ADDR(sc_a, wsum) + 32u);
 #pragma unroll 1
   for (int g = 0; g < G; ++g) {
-    const uint32_t t4 = (take >> (4 * g)) & 15u;
+    const uint32_t t4 = (uint32_t)(take >> (4 * g)) & 15u;
     if (!t4) continue;
     const int j = j0 + 4 * g;
     int c[4] = {j, j + 1, j + 2, j + 3};
@@ -796,12 +806,13 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
 }
 
 // Top-K dispatch: R = the smallest power of two (at least 4) with R NCT >= m
-// (m <= 32 NCT).
+// (m <= 64 NCT); 64-bit position masks only for R = 64.
 __device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                             float lo, float hi) {
   int R = 4;
   while (R * NCT < m) R <<= 1;
-  select_keys(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
+  if (R <= 32) select_keys<uint32_t>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
+  else select_keys<unsigned long long>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
 }
 
 // Per-query max (x sl2, log2 units) of the valid rows of TMEM tiles
@@ -1485,6 +1496,23 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
 // ---------------------------------------------------------------------------
 namespace {
 
+// The kernel's dynamic shared-memory limit, raised once per device and stage
+// count to the largest size requested so far instead of on every launch.
+cudaError_t ensure_smem_limit(int stages, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::pair<int, int>, size_t> raised;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  size_t& cur = raised[std::make_pair(dev, stages)];
+  if (cur >= smem) return cudaSuccess;
+  e = stages == 4 ? cudaFuncSetAttribute(wf_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)
+                  : cudaFuncSetAttribute(wf_fused_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) cur = smem;
+  return e;
+}
+
 // How many clusters of cs CTAs (with `smem` bytes each) can be resident at
 // once on the current device; cached per configuration.
 int max_active_clusters(int stages, int cs, size_t smem) {
@@ -1509,13 +1537,10 @@ int max_active_clusters(int stages, int cs, size_t smem) {
   cfg.numAttrs = 1;
   int n = 0;
   cudaError_t e;
-  if (stages == 4) {
-    e = cudaFuncSetAttribute(wf_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<4>, &cfg);
-  } else {
-    e = cudaFuncSetAttribute(wf_fused_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<3>, &cfg);
-  }
+  e = ensure_smem_limit(stages, smem);  // only ever raised, so a launch's earlier limit still holds
+  if (e == cudaSuccess)
+    e = stages == 4 ? cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<4>, &cfg)
+                    : cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<3>, &cfg);
   if (e != cudaSuccess) {
     (void)cudaGetLastError();
     n = 0;
@@ -1667,18 +1692,9 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e;
-  if (fp.stages == 4) {
-    e = cudaFuncSetAttribute(wf_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)cfg.dynamicSmemBytes);
-    if (e != cudaSuccess) return e;
-    e = cudaLaunchKernelEx(&cfg, wf_fused_kernel<4>, p);
-  } else {
-    e = cudaFuncSetAttribute(wf_fused_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)cfg.dynamicSmemBytes);
-    if (e != cudaSuccess) return e;
-    e = cudaLaunchKernelEx(&cfg, wf_fused_kernel<3>, p);
-  }
+  cudaError_t e = ensure_smem_limit(fp.stages, cfg.dynamicSmemBytes);
+  if (e != cudaSuccess) return e;
+  e = fp.stages == 4 ? cudaLaunchKernelEx(&cfg, wf_fused_kernel<4>, p) : cudaLaunchKernelEx(&cfg, wf_fused_kernel<3>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

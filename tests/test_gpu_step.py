@@ -128,11 +128,13 @@ def test_step_random_shapes(B, H, n, q, ng, L, keep, bshd):
         assert_close_out(f64(run.O[b, h]), O, torch.bfloat16)
 
 
-@pytest.mark.parametrize("cfg", ["c2", "c3", "c5"])
+@pytest.mark.parametrize("cfg", ["c2", "c3", "c4", "c5"])
 def test_step_level0_schedule(cfg):
     # The token level as its own selection step (wf_level0_schedule): the
     # level-0 scan over raw keys keeps k of 2 keep[1] candidates.  Planted
-    # ladder built for that schedule; full-size layer in the fused kernel.
+    # ladder built for that schedule; full-size layer in the fused kernel
+    # (at 128K the finest scales hold up to 7304 candidates: 64 keys a Top-K
+    # thread).
     import dataclasses
     w0 = synth.WORKLOADS[cfg]
     keep = tuple(wf.wf_level0_schedule(w0.n, w0.levels, w0.k))
