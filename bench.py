@@ -46,7 +46,7 @@ from paper_2606_00724_gb300 import synth  # noqa: E402
 
 METRIC = "fused filter+sparse-attn step latency (us) & achieved HBM GB/s vs roofline, 1 GB300"
 DEFAULT_WORKLOAD = "c3"
-WAVELET = None  # None: the Haar pyramid path (wf_step); "haar" / "db2": the literal path (wf_filter_wavelet)
+WAVELET = None  # None: the Haar pyramid path (wf_step); "haar" / "db2": the literal path (wf_step_wavelet)
 
 
 def peaks():
@@ -97,7 +97,13 @@ def wavelet_unit_bytes(w: synth.Workload) -> int:
 def fused_eligible(w: synth.Workload) -> bool:
     """wf_step runs its single fused kernel for bf16, head_dim 128, <= 32 query
     rows and one query head per key head (the Haar pyramid path)."""
-    return WAVELET is None and w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group == 1
+    return WAVELET is None and fused_shape(w)
+
+
+def fused_shape(w: synth.Workload) -> bool:
+    """Shapes the fused kernel serves: bf16, head_dim 128, <= 32 query rows,
+    one query head per key head."""
+    return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group == 1
 
 
 def recorded_traffic(w: synth.Workload):
@@ -123,6 +129,8 @@ def launches_per_step(w: synth.Workload) -> int:
     if fused_eligible(w):
         return 1
     trim = int(w.keep[0]) < 2 * int(w.keep[1])
+    if WAVELET and fused_shape(w):  # one fused launch per scale, a transform before each below the top
+        return w.levels + (w.levels - 1)
     if WAVELET:  # one transform kernel per scale below the top
         return 3 * w.levels + (w.levels - 1) + 3 * trim + 2
     return 3 * w.levels + 3 * trim + 2
@@ -310,8 +318,8 @@ def run_gpu(args, cfg, rank, world, device):
             # the pyramid), the finer scales' transforms inside every step.
             coeffs = torch.empty(w.batch, w.heads, w.n >> w.levels, w.head_dim, dtype=lay.K.dtype, device=device)
             wf.wf_wavelet_approx(lay.K, w.levels, basis, coeffs)
-            ws = torch.zeros(max(wf.wf_filter_wavelet_workspace_bytes(lay.Q, lay.K, w.levels, keep, basis),
-                                 wf.wf_attn_workspace_bytes(lay.Q, w.k, w.ng)), dtype=torch.uint8, device=device)
+            ws = torch.zeros(wf.wf_step_wavelet_workspace_bytes(lay.Q, lay.K, w.levels, keep, basis, w.ng),
+                             dtype=torch.uint8, device=device)
         else:
             coeffs = torch.empty(wf.wf_coeffs_bytes(lay.K, w.levels), dtype=torch.uint8, device=device)
             wf.wf_dwt_build(lay.K, w.levels, coeffs)
@@ -325,8 +333,8 @@ def run_gpu(args, cfg, rank, world, device):
         if WAVELET:
             if refresh:
                 wf.wf_wavelet_approx(lay.K, w.levels, basis, bf["coeffs"], stream=st)
-            wf.wf_filter_wavelet(Q, bf["coeffs"], lay.K, w.levels, keep, basis, bf["idx"], bf["ws"], stream=st)
-            wf.wf_sparse_attn(Q, lay.K, lay.V, bf["idx"], w.k, Kg, Vg, bf["O"], bf["ws"], stream=st)
+            wf.wf_step_wavelet(Q, bf["coeffs"], lay.K, lay.V, Kg, Vg, w.levels, keep, basis, bf["idx"], bf["O"],
+                               bf["ws"], stream=st)
         else:
             wf.wf_step(Q, lay.K, lay.V, Kg, Vg, bf["coeffs"], refresh, w.levels, keep, bf["idx"], bf["O"], bf["ws"],
                        st)
@@ -467,8 +475,8 @@ def main():
     ap.add_argument("--graph", action="store_true",
                     help="replay each step from a CUDA graph recorded after the warm-up")
     ap.add_argument("--wavelet", default=None, choices=["haar", "db2"],
-                    help="time the literal path for a generic basis (wf_filter_wavelet + wf_sparse_attn): the "
-                         "transform of the gathered candidate blocks at every scale")
+                    help="time the literal path for a generic basis (wf_step_wavelet): the transform of the "
+                         "gathered candidate blocks at every scale")
     ap.add_argument("--schedule", default="default", choices=["default", "level0"],
                     help="kept counts: the default schedule, or the token level as its own selection step")
     ap.add_argument("--measure", default="step", choices=["step", "cache-update"],
@@ -511,8 +519,9 @@ def main():
               "context": w.n, "query_block": w.q, "generation_rows": w.ng, "levels": w.levels, "k": w.k,
               "keep": list(w.keep), "layers": w.layers, "storage": w.dtype,
               "step": ("wf_step (one fused filter + sparse-attention kernel) per layer" if fused_eligible(w) else
-                       f"wf_filter_wavelet ({WAVELET}, periodized; the gathered candidate blocks transformed at every "
-                       "scale) + wf_sparse_attn per layer" if WAVELET else
+                       f"wf_step_wavelet ({WAVELET}, periodized; the gathered candidate blocks transformed at every "
+                       "scale" + ("; one fused filter launch per scale, the last with the sparse attention)"
+                                  if fused_shape(w) else "; per-stage kernels)") + " per layer" if WAVELET else
                        "wf_step (per-stage filter and sparse-attention kernels) per layer") + (
                   f"; wf_dwt_build refresh every {w.refresh_every} steps" if w.refresh_every else
                   ("; scale-L rows built once before timing" if WAVELET else "; pyramid built once before timing")),
@@ -575,7 +584,8 @@ def main():
     if w.refresh_every:
         achieved = step_bytes / w.layers / (per_layer_ms * 1e-3) / 1e9
     kname = "wf_fused_kernel" if fused_eligible(w) else (
-        "per-stage kernels (approx/score/weights/select/attn)" if WAVELET else
+        ("approx_kernel + wf_fused_kernel (one launch per scale)" if fused_shape(w) else
+         "per-stage kernels (approx/score/weights/select/attn)") if WAVELET else
         "per-stage kernels (score/weights/select/attn)")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                 "frac_of_nominal_7900": achieved / 7900.0,

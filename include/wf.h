@@ -320,6 +320,30 @@ wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const void* 
                   int refresh_coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
                   void* O, const wf_tensor* o, void* ws, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * One layer on the literal path (Eq. 11 with the basis `wavelet`, as
+ * wf_filter_wavelet): the filter, then the sparse attention with scale
+ * 1/sqrt(d), writing idx (and level_sets, if not NULL) and O exactly as
+ * wf_filter_wavelet + wf_sparse_attn define them.  top: the scale-L rows of
+ * the whole prompt (wf_wavelet_approx with cand = NULL, level = levels),
+ * recomputed by the caller whenever K changes.  Other arguments and rules as
+ * for wf_step; ws: at least wf_step_wavelet_workspace_bytes() bytes, 256-byte
+ * aligned, with the status word of wf_step in its first 4 bytes.
+ *
+ * For bf16 with head_dim 128, at most 32 query rows and one query head per
+ * key head, every scale runs on wf_step's fused kernel: one launch per scale,
+ * after the transform of that scale's candidate blocks, with the previous
+ * selection handed over in ws; the last launch also runs the attention.
+ * wf_filter_wavelet takes the same fused launches (without the attention)
+ * for those shapes.  Other shapes run the per-stage kernels.
+ * ------------------------------------------------------------------------- */
+size_t wf_step_wavelet_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep,
+                                       int wavelet, int n_g);
+wf_status wf_step_wavelet(const void* Q, const wf_tensor* q, const void* top, const void* K, const void* V,
+                          const wf_tensor* kv, const void* Kg, const void* Vg, const wf_tensor* g, int levels,
+                          const int32_t* keep, int wavelet, int32_t* idx, int32_t* level_sets, void* O,
+                          const wf_tensor* o, void* ws, size_t ws_bytes, void* stream);
+
 /* Device status of the last wf_step calls that used workspace ws: waits for
  * `stream`, returns WF_ERR_TIMEOUT (and clears the word) if a bounded device
  * wait gave up, else WF_OK.  Synchronising; not for the hot loop. */

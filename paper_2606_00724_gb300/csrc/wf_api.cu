@@ -62,6 +62,13 @@ wf_status check_keep(int64_t n, int levels, const int32_t* keep) {
 
 wf_status cuda_status(cudaError_t e) { return e == cudaSuccess ? WF_OK : WF_ERR_CUDA; }
 
+// Number of SMs of the current device.
+bool device_sms(int* sms) {
+  int dev = 0;
+  return cudaGetDevice(&dev) == cudaSuccess &&
+         cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
+}
+
 int64_t ceil_guarded(double v) { return (int64_t)ceil(v - 1e-9); }
 
 wf_status check_filter_args(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep) {
@@ -250,8 +257,16 @@ WF_API wf_status wf_filter_wavelet(const void* Q, const wf_tensor* q, const void
     return WF_ERR_ALIGN;
   const wf::FilterPlan p = wf::plan_filter(*q, *kv, levels, keep);
   if (ws_bytes < wf::wavelet_filter_bytes(p)) return WF_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!device_sms(&sms)) return WF_ERR_CUDA;
+  const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, 0, nullptr, sms);
+  if (fp.ok && q->heads == kv->heads)
+    return cuda_status(wf::launch_literal_fused(fp, p, Q, *q, top, K, nullptr, *kv, nullptr, nullptr, nullptr,
+                                                wavelet, idx, level_sets, nullptr, nullptr, ws,
+                                                static_cast<int*>(ws), s));
   return cuda_status(wf::launch_filter_wavelet(p, Q, *q, top, K, *kv, wavelet, idx, level_sets, ws,
-                                               static_cast<int*>(ws), static_cast<cudaStream_t>(stream)));
+                                               static_cast<int*>(ws), s));
 }
 
 WF_API size_t wf_attn_workspace_bytes(const wf_tensor* q, int k, int n_g) {
@@ -311,10 +326,8 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   if (coeffs_bytes < wf_coeffs_bytes(kv, levels)) return WF_ERR_WORKSPACE;
   if (ws_bytes < wf_step_workspace_bytes(q, kv, levels, keep, n_g)) return WF_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return WF_ERR_CUDA;
+  int sms = 0;
+  if (!device_sms(&sms)) return WF_ERR_CUDA;
   int* status = static_cast<int*>(ws);  // set by the fused kernel on a timeout; read and cleared by wf_workspace_status
   void* scratch = static_cast<char*>(ws) + kStatusBytes;
   cudaError_t e = cudaSuccess;
@@ -329,6 +342,50 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
   const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
   if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, status, s)) != cudaSuccess)
     return WF_ERR_CUDA;
+  const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g, group_of(q, kv));
+  const float sc = 1.0f / sqrtf((float)q->head_dim);
+  e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, status, s);
+  return cuda_status(e);
+}
+
+WF_API size_t wf_step_wavelet_workspace_bytes(const wf_tensor* q, const wf_tensor* kv, int levels,
+                                              const int32_t* keep, int wavelet, int n_g) {
+  if (check_filter_args(q, kv, levels, keep) != WF_OK || n_g < 0) return 0;
+  if (!wf::wavelet_taps(wavelet) || levels > wf::wavelet_max_level(wavelet)) return 0;
+  const size_t f = wf::wavelet_filter_bytes(wf::plan_filter(*q, *kv, levels, keep));
+  const size_t a = wf::plan_attn(*q, keep[0], n_g, 1).total;
+  return kStatusBytes + (f > a ? f : a);
+}
+
+WF_API wf_status wf_step_wavelet(const void* Q, const wf_tensor* q, const void* top, const void* K, const void* V,
+                                 const wf_tensor* kv, const void* Kg, const void* Vg, const wf_tensor* g, int levels,
+                                 const int32_t* keep, int wavelet, int32_t* idx, int32_t* level_sets, void* O,
+                                 const wf_tensor* o, void* ws, size_t ws_bytes, void* stream) {
+  wf_status st = check_filter_args(q, kv, levels, keep);
+  if (st != WF_OK) return st;
+  if (!wf::wavelet_taps(wavelet) || levels > wf::wavelet_max_level(wavelet)) return WF_ERR_UNSUPPORTED;
+  const int n_g = g ? g->seq : 0;
+  if ((st = check_attn_args(q, kv, keep[0], g, n_g, o)) != WF_OK) return st;
+  if (!Q || !top || !K || !V || !idx || !O || !ws) return WF_ERR_INVALID_ARG;
+  if (n_g > 0 && (!Kg || !Vg)) return WF_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(top) || !aligned16(K) || !aligned16(V) || !aligned16(O)) return WF_ERR_ALIGN;
+  if (n_g > 0 && (!aligned16(Kg) || !aligned16(Vg))) return WF_ERR_ALIGN;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || (reinterpret_cast<uintptr_t>(idx) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(level_sets) & 3u) != 0)
+    return WF_ERR_ALIGN;
+  if (ws_bytes < wf_step_wavelet_workspace_bytes(q, kv, levels, keep, wavelet, n_g)) return WF_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!device_sms(&sms)) return WF_ERR_CUDA;
+  int* status = static_cast<int*>(ws);
+  void* scratch = static_cast<char*>(ws) + kStatusBytes;
+  const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
+  const wf::FusedPlan fp = wf::plan_fused(*q, *kv, levels, keep, n_g, n_g > 0 ? g : nullptr, sms);
+  if (fp.ok && q->heads == kv->heads)
+    return cuda_status(wf::launch_literal_fused(fp, fl, Q, *q, top, K, V, *kv, Kg, Vg, n_g > 0 ? g : nullptr, wavelet,
+                                                idx, level_sets, O, o, scratch, status, s));
+  cudaError_t e = wf::launch_filter_wavelet(fl, Q, *q, top, K, *kv, wavelet, idx, level_sets, scratch, status, s);
+  if (e != cudaSuccess) return WF_ERR_CUDA;
   const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g, group_of(q, kv));
   const float sc = 1.0f / sqrtf((float)q->head_dim);
   e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, status, s);

@@ -141,6 +141,19 @@ struct FusedParams {
   int stall;                  // test-only: the MMA thread's first wait never completes
   int32_t keep[12];
   float scale_log2;           // log2(e) / sqrt(d)
+  // The scales this launch runs, lev_top down to lev_bot (the whole chain, L
+  // down to 1 or 0, for the pyramid step).  A launch that starts below L reads
+  // the previous selection J_{lev_top+1} as the children list jin (candidate
+  // block indices of scale lev_top, 2 J[i] and 2 J[i] + 1); one that ends
+  // above the final scale writes the children of its last selection to jout.
+  int lev_top, lev_bot, final_sel, attn;
+  const int32_t* jin;
+  int32_t* jout;
+  int64_t jstride;  // entries per unit of jin and jout
+  // Literal-basis rows: scale lev_top's candidate rows in candidate order
+  // (row j of unit u at lrows + u lrows_unit + j D); null for the pyramid.
+  const bf16* lrows;
+  int64_t lrows_unit;
 };
 
 // Per-CTA constants and shared-memory addresses.
@@ -149,7 +162,7 @@ struct Ctx {
   Misc* ms;
   SmemLayout ly;
   uint32_t rank, cs, tmem;
-  int np, u0, lev_end, stages;
+  int np, u0, lev_top, lev_end, stages;
 };
 
 // Thread index within its unit's compute warps, and their barrier.
@@ -253,8 +266,12 @@ __device__ __forceinline__ int32_t* unit_J(const Ctx& c, const FusedParams& p, i
 // Rows of unit u at scale lev (pyramid level lev, or the raw keys at level 0).
 __device__ __forceinline__ RowSrc scale_src(const Ctx& c, const FusedParams& p, int pp, int lev, int g0, int mc) {
   const int u = c.u0 + pp;
+  const bool lit = p.lrows && lev >= 1 && lev == c.lev_top;  // literal-basis rows of this launch's scale
   RowSrc s;
-  if (lev >= 1) {
+  if (lit) {
+    s.base = p.lrows + (int64_t)u * p.lrows_unit;  // row j: candidate j's transform (kind 0 below)
+    s.stride = D;
+  } else if (lev >= 1) {
     s.base = p.coeffs + ((int64_t)u * p.rows_total + ((int64_t)p.n - ((int64_t)p.n >> (lev - 1)))) * D;
     s.stride = D;
   } else {
@@ -264,11 +281,11 @@ __device__ __forceinline__ RowSrc scale_src(const Ctx& c, const FusedParams& p, 
   s.gbase = nullptr;
   s.gstride = 0;
   s.J = smem_u32(unit_J(c, p, pp, lev + 1));  // the children of the selection one scale up (unused at the top)
-  s.kind = lev == p.L ? 0 : 1;
+  s.kind = (lev == p.L || lit) ? 0 : 1;
   s.g0 = g0;
   s.mc = mc;
   s.kk = 0;
-  s.rows = lev >= 1 ? (int)(p.n >> lev) : (int)p.n;
+  s.rows = lit ? m_total(p, lev) : (lev >= 1 ? (int)(p.n >> lev) : (int)p.n);
   return s;
 }
 
@@ -362,10 +379,10 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
   Misc& ms = *c.ms;
   const int pt = threadIdx.x - P0;
   int it = 0;
-  for (int lev = p.L; lev >= c.lev_end; --lev) {
+  for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
     for (int pp = 0; pp < c.np; ++pp) {
       // The rows of a lower scale are the children of the unit's last selection.
-      if (lev != p.L) wait_or_abort(bar_addr(ms.jready[pp]), (uint32_t)(p.L - lev - 1) & 1u, ms, p.status);
+      if (lev != c.lev_top) wait_or_abort(bar_addr(ms.jready[pp]), (uint32_t)(c.lev_top - lev - 1) & 1u, ms, p.status);
       int g0, mc;
       scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
       const int ntl = tiles_of(mc);
@@ -373,8 +390,8 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
       it += ntl;
     }
   }
-  const int nsel = p.L - c.lev_end + 1;
-  for (int pp = 0; pp < c.np; ++pp) {
+  const int nsel = c.lev_top - c.lev_end + 1;
+  for (int pp = 0; pp < c.np && p.attn; ++pp) {
     wait_or_abort(bar_addr(ms.jready[pp]), (uint32_t)(nsel - 1) & 1u, ms, p.status);
     int a0, mc;
     attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
@@ -449,7 +466,7 @@ template <int S>
 __device__ void mma_role_body(const Ctx& c, const FusedParams& p) {
   Misc& ms = *c.ms;
   int it = 0;
-  for (int lev = p.L; lev >= c.lev_end; --lev) {
+  for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
     for (int pp = 0; pp < c.np; ++pp) {
       int g0, mc;
       scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
@@ -459,7 +476,7 @@ __device__ void mma_role_body(const Ctx& c, const FusedParams& p) {
       it += ntl;
     }
   }
-  for (int pp = 0; pp < c.np; ++pp) {
+  for (int pp = 0; pp < c.np && p.attn; ++pp) {
     int a0, mc;
     attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
     const int ntl = tiles_of(mc);
@@ -1298,7 +1315,8 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   const uint32_t tb = c.tmem + pp * p.ucols;
   const int u = c.u0 + pp;
   const float sl2 = p.scale_log2;
-  int64_t sets_off = 0;
+  int64_t sets_off = 0;  // the level sets of the scales above this launch's first
+  for (int l = p.L; l > c.lev_top; --l) sets_off += p.keep[l];
   // Parity of the unit's next mdone phase (the attention's two: S tiles
   // scored, then PV products done).  The MMA thread commits a phase only for
   // a non-empty stream.
@@ -1310,8 +1328,8 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   };
   uint32_t tpar = 0;  // parity of each scale-tile barrier's next phase
 #pragma unroll 1
-  for (int lev = p.L; lev >= c.lev_end; --lev) {
-    const uint32_t ph = (uint32_t)(p.L - lev) & 1u;  // phase of the per-scale barriers
+  for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
+    const uint32_t ph = (uint32_t)(c.lev_top - lev) & 1u;  // phase of the per-scale barriers
     const int m = m_total(p, lev);
     int g0, mc;
     scale_slice(m, c.rank, c.cs, g0, mc);
@@ -1354,7 +1372,13 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
 #pragma unroll 1
         for (int i = tid; i < kb; i += NCT) ls[i] = J[i];
       }
-      if (lev == c.lev_end) {
+      if (lev == c.lev_end && !p.final_sel) {
+        // A launch that ends above the final scale hands on the children of
+        // its last selection (the next launch's candidates).
+        int32_t* out = p.jout + (int64_t)u * p.jstride;
+#pragma unroll 1
+        for (int t = tid; t < 2 * kb; t += NCT) out[t] = 2 * J[t >> 1] + (t & 1);
+      } else if (lev == c.lev_end) {
         // mu^0: the children of J^1, or the trimmed level-0 selection.
         const int kk = p.keep[0];
         int32_t* out = p.idx + (int64_t)u * kk;
@@ -1369,6 +1393,7 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     }
     if (lev >= 1) sets_off += kb;
   }
+  if (!p.attn) return;
 
   // Attention: S of the key slice, P for the MMA thread, then the combine.
   int a0, mc;
@@ -1393,7 +1418,8 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   c.cs = cluster_size();
   c.u0 = (int)cluster_id_x() * p.P;
   c.np = min(p.P, p.U - c.u0);
-  c.lev_end = p.trim ? 0 : 1;
+  c.lev_top = p.lev_top;
+  c.lev_end = p.lev_bot;
   c.stages = S;
   const int tid = threadIdx.x, warp = tid >> 5;
 
@@ -1425,7 +1451,7 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     // Arm the first phase of every receive barrier (bytes this CTA expects).
     for (int pp = 0; pp < c.np; ++pp) {
       mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)(p.n >> p.L) + c.cs * NCW * 8u);
+      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, c.lev_top) + c.cs * NCW * 8u);
       const uint32_t rows = (uint32_t)(dlo((int)c.rank + 1, c.cs) - dlo((int)c.rank, c.cs));
       mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), c.cs * rows * NQ * 4u + c.cs * NQ * 8u);
     }
@@ -1439,6 +1465,15 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     uint8_t* sc = smem + c.ly.p + pp * UNIT_P_BYTES;
     for (int e = tid; e < (int)((sizeof(SelScratch) + 15) / 16); e += NT)
       *reinterpret_cast<uint4*>(sc + 16 * e) = make_uint4(0, 0, 0, 0);
+  }
+  // A launch that starts below the top scale: the previous selection
+  // J_{lev_top+1} from the children list it was handed (halved).
+  if (c.lev_top < p.L) {
+    for (int pp = 0; pp < c.np; ++pp) {
+      const int32_t* src = p.jin + (int64_t)(c.u0 + pp) * p.jstride;
+      int32_t* J = unit_J(c, p, pp, c.lev_top + 1);
+      for (int i = tid; i < p.keep[c.lev_top + 1]; i += NT) J[i] = src[2 * i] >> 1;
+    }
   }
   // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
   for (int pp = 0; pp < c.np; ++pp) {
@@ -1646,7 +1681,7 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
 cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                          const wf_tensor& kv, const void* Kg, const void* Vg, const wf_tensor* g,
                          const void* coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
-                         void* O, const wf_tensor& od, int* status, cudaStream_t s) {
+                         void* O, const wf_tensor& od, int* status, cudaStream_t s, const FusedRange* range) {
   FusedParams p;
   memset(&p, 0, sizeof(p));
   p.Q = static_cast<const bf16*>(Q);
@@ -1679,6 +1714,22 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   p.stall = wc.stall;
   for (int l = 0; l <= levels; ++l) p.keep[l] = keep[l];
   p.scale_log2 = kLog2e / sqrtf((float)D);
+  if (range) {
+    p.lev_top = range->lev_top;
+    p.lev_bot = range->lev_bot;
+    p.final_sel = range->final_sel;
+    p.attn = range->attn;
+    p.jin = range->jin;
+    p.jout = range->jout;
+    p.jstride = range->jstride;
+    p.lrows = static_cast<const bf16*>(range->lrows);
+    p.lrows_unit = range->lrows_unit;
+  } else {
+    p.lev_top = levels;
+    p.lev_bot = fp.trim ? 0 : 1;
+    p.final_sel = 1;
+    p.attn = 1;
+  }
 
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)(fp.clusters * fp.cs), 1, 1);
@@ -1697,6 +1748,44 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   e = fp.stages == 4 ? cudaLaunchKernelEx(&cfg, wf_fused_kernel<4>, p) : cudaLaunchKernelEx(&cfg, wf_fused_kernel<3>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+cudaError_t launch_literal_fused(const FusedPlan& fp, const FilterPlan& fl, const void* Q, const wf_tensor& qd,
+                                 const void* top, const void* K, const void* V, const wf_tensor& kv, const void* Kg,
+                                 const void* Vg, const wf_tensor* g, int wavelet, int32_t* idx, int32_t* level_sets,
+                                 void* O, const wf_tensor* od, void* ws, int* status, cudaStream_t s) {
+  char* base = static_cast<char*>(ws);
+  int32_t* cur = reinterpret_cast<int32_t*>(base + fl.off_cand_a);  // candidates of the scale being filtered
+  int32_t* nxt = reinterpret_cast<int32_t*>(base + fl.off_cand_b);
+  void* arows = base + align_up(fl.total, 256);
+  const int L = fl.L;
+  int m = fl.n >> L;
+  cudaError_t e;
+  for (int l = L; l >= 1; --l) {
+    // Scale l's rows: the whole prompt's scale-L rows at the top, else the
+    // transform of the candidates' gathered blocks, in candidate order.
+    if (l < L && (e = launch_wavelet_approx(K, kv, cur, fl.cmax, m, l, wavelet, arows, (int64_t)fl.cmax * D, s)) !=
+                     cudaSuccess)
+      return e;
+    FusedRange r{};
+    r.lev_top = l;
+    r.lev_bot = (l == 1 && fl.trim) ? 0 : l;
+    r.final_sel = l == 1;
+    r.attn = l == 1 && O != nullptr;
+    r.jin = cur;
+    r.jout = nxt;
+    r.jstride = fl.cmax;
+    r.lrows = l == L ? top : arows;
+    r.lrows_unit = l == L ? (int64_t)m * D : (int64_t)fl.cmax * D;
+    if ((e = launch_fused(fp, Q, qd, K, V, kv, Kg, Vg, g, nullptr, L, fl.keep, idx, level_sets, O, od ? *od : qd,
+                          status, s, &r)) != cudaSuccess)
+      return e;
+    m = 2 * fl.keep[l];
+    int32_t* t = cur;
+    cur = nxt;
+    nxt = t;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace wf

@@ -141,10 +141,39 @@ struct FusedPlan {
 };
 FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int n_g,
                      const wf_tensor* g, int num_sms);
+// Part of the chain in one launch (the literal-basis path runs one launch per
+// scale, with the transform of the candidates' blocks between launches):
+// scales lev_top down to lev_bot; the previous selection J_{lev_top+1} as its
+// children list jin (when lev_top < L); the children of the last selection to
+// jout unless final_sel (then mu^0 goes to idx); the attention if attn.
+// Scale lev_top's rows come from lrows ([units][m][d], unit stride lrows_unit
+// elements) when not null, else from the pyramid.
+struct FusedRange {
+  int lev_top, lev_bot, final_sel, attn;
+  const int32_t* jin;
+  int32_t* jout;
+  int64_t jstride;
+  const void* lrows;
+  int64_t lrows_unit;
+};
+// range == nullptr: the whole step (every scale, mu^0, the attention).
 cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd, const void* K, const void* V,
                          const wf_tensor& kv, const void* Kg, const void* Vg, const wf_tensor* g,
                          const void* coeffs, int levels, const int32_t* keep, int32_t* idx, int32_t* level_sets,
-                         void* O, const wf_tensor& od, int* status, cudaStream_t s);
+                         void* O, const wf_tensor& od, int* status, cudaStream_t s,
+                         const FusedRange* range = nullptr);
+
+// The literal-basis filter on the fused kernel (bf16, d 128, one query head
+// per KV head, a fused plan fp for the same shapes): one launch per scale,
+// each after the transform of its candidates' gathered blocks
+// (launch_wavelet_approx, into the block after the filter plan's workspace);
+// the candidate lists pass between launches in the plan's two candidate
+// buffers.  With O not null the last launch also runs the attention (od its
+// descriptor; Kg/Vg/g the generation rows).
+cudaError_t launch_literal_fused(const FusedPlan& fp, const FilterPlan& fl, const void* Q, const wf_tensor& qd,
+                                 const void* top, const void* K, const void* V, const wf_tensor& kv, const void* Kg,
+                                 const void* Vg, const wf_tensor* g, int wavelet, int32_t* idx, int32_t* level_sets,
+                                 void* O, const wf_tensor* od, void* ws, int* status, cudaStream_t s);
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 

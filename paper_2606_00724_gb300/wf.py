@@ -59,6 +59,8 @@ SIGNATURES = {
     "wf_sparse_attn_noalloc": (_I, [_P, _T, _P, _P, _T, _P, _I, _P, _P, _T, _P, _T, ctypes.c_float, _P]),
     "wf_noalloc_status": (_I, [_P]),
     "wf_step": (_I, [_P, _T, _P, _P, _T, _P, _P, _T, _P, _SZ, _I, _I, _P, _P, _P, _P, _T, _P, _SZ, _P]),
+    "wf_step_wavelet_workspace_bytes": (_SZ, [_T, _T, _I, _P, _I, _I]),
+    "wf_step_wavelet": (_I, [_P, _T, _P, _P, _P, _T, _P, _P, _T, _I, _P, _I, _P, _P, _P, _T, _P, _SZ, _P]),
     "wf_workspace_status": (_I, [_P, _P]),
     # include/wf_testing.h (test-only)
     "wf_testing_set_wait_failure": (_I, [_I, ctypes.c_longlong]),
@@ -254,6 +256,25 @@ def wf_step(Q, K, V, Kg, Vg, coeffs, refresh: bool, levels: int, keep, idx, O, w
                          coeffs.numel() * coeffs.element_size(), int(bool(refresh)), levels, _keep_arr(keep),
                          _ptr(idx), _ptr(level_sets), _ptr(O), ctypes.byref(do), _ptr(ws),
                          ws.numel() * ws.element_size(), _stream(stream)), "wf_step")
+
+
+def wf_step_wavelet_workspace_bytes(Q: torch.Tensor, K: torch.Tensor, levels: int, keep, wavelet: int,
+                                    n_g: int) -> int:
+    dq, dk = desc(Q), desc(K)
+    return int(lib().wf_step_wavelet_workspace_bytes(ctypes.byref(dq), ctypes.byref(dk), levels, _keep_arr(keep),
+                                                     wavelet, n_g))
+
+
+def wf_step_wavelet(Q, top, K, V, Kg, Vg, levels: int, keep, wavelet: int, idx, O, ws, stream=None,
+                    level_sets=None):
+    dq, dk, do = desc(Q), desc(K), desc(O)
+    dg = desc(Kg) if Kg is not None else None
+    if V.stride() != K.stride() or V.shape != K.shape:
+        raise ValueError("K and V must share shape and strides")
+    _check(lib().wf_step_wavelet(_ptr(Q), ctypes.byref(dq), _ptr(top), _ptr(K), _ptr(V), ctypes.byref(dk),
+                                 _ptr(Kg), _ptr(Vg), ctypes.byref(dg) if dg is not None else None, levels,
+                                 _keep_arr(keep), wavelet, _ptr(idx), _ptr(level_sets), _ptr(O), ctypes.byref(do),
+                                 _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)), "wf_step_wavelet")
 
 
 def wf_workspace_status(ws: torch.Tensor, stream=None):

@@ -217,6 +217,35 @@ def test_wavelet_rejects(lib):
     assert lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1) > \
         lib.wf_filter_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep)
     assert lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 5) == 0
+    # The literal step: the filter's workspace (or the attention's) after the status block.
+    step_need = lib.wf_step_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1, 4)
+    assert step_need >= 256 + lib.wf_filter_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1)
+    assert step_need >= 256 + lib.wf_attn_workspace_bytes(ctypes.byref(q), 16, 4)
+    assert lib.wf_step_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 5, 4) == 0
+    assert lib.wf_step_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1, -1) == 0
+
+
+@no_gpu
+def test_step_wavelet_rejects(lib):
+    kv = _desc(1, 2, 64, 128)
+    q = _desc(1, 2, 32, 128)
+    g = _desc(1, 2, 4, 128)
+    keep = (ctypes.c_int32 * 3)(16, 8, 8)
+    need = lib.wf_step_wavelet_workspace_bytes(ctypes.byref(q), ctypes.byref(kv), 2, keep, 1, 4)
+    ws = ctypes.c_void_p(0x40000)
+
+    def call(top=FAKE, V=FAKE2, wv=1, Kg=FAKE, ws=ws, ws_bytes=need, idx=ctypes.c_void_p(0x50000), levels=2):
+        return lib.wf_step_wavelet(FAKE, ctypes.byref(q), top, FAKE, V, ctypes.byref(kv), Kg, FAKE2,
+                                   ctypes.byref(g), levels, keep, wv, idx, None, FAKE2, ctypes.byref(q), ws,
+                                   ws_bytes, None)
+    assert call(wv=7) == -8                       # unknown basis
+    assert call(top=None) == -1
+    assert call(V=None) == -1
+    assert call(Kg=None) == -1                    # n_g > 0 needs Kg
+    assert call(top=ctypes.c_void_p(0x10008)) == -4
+    assert call(ws=ctypes.c_void_p(0x40010)) == -4  # ws 256-byte aligned
+    assert call(idx=ctypes.c_void_p(0x50002)) == -4
+    assert call(ws_bytes=need - 1) == -5
 
 
 def test_wait_failure_control(lib):

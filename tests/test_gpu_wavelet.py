@@ -2,13 +2,16 @@
 periodized): wf_wavelet_approx against the oracle's fp32 storage rule bit
 for bit (whole prompt and gathered candidate blocks), the Haar case against
 the stored pyramid and wf_filter, and wf_filter_wavelet's indices against
-the oracle's literal filter on planted inputs (every scale, bit-exact)."""
+the oracle's literal filter on planted inputs (every scale, bit-exact), and
+wf_step_wavelet's indices and output against the oracle.  For bf16 keys with
+head_dim 128 and one query head per key head both calls run the fused
+kernel once per scale."""
 import numpy as np
 import pytest
 import torch
 
 import oracle
-from helpers import GpuRun, f64
+from helpers import GpuRun, assert_close_out, f64
 from paper_2606_00724_gb300 import synth, wf
 
 pytestmark = pytest.mark.gpu
@@ -126,3 +129,42 @@ def test_filter_wavelet_db2_matches_oracle(cfg, units):
         for lev in range(w.levels, -1, -1):
             assert np.array_equal(gsets[lev], osets[lev]), f"unit {u} scale {lev}"
         assert np.array_equal(idx[u].cpu().numpy(), mu0)
+
+
+@pytest.mark.parametrize("cfg,units", [("c2", [0, 31]), ("c3", [0, 63]), ("c4", [31])])
+def test_step_wavelet_db2_matches_oracle(cfg, units):
+    # The literal step: indices and level sets of the planted units against the
+    # oracle's literal filter, every unit's output against the oracle attention
+    # on the GPU's own indices, and the filter-only call agreeing bit for bit.
+    w = synth.WORKLOADS[cfg]
+    batch = synth.make_batch(w, planted=True, device="cuda", cfg=cfg, units=units)
+    Q, K, V = batch.Q, batch.K, batch.V
+    B, H = K.shape[:2]
+    wv = wf.WF_WAVELET_DB2
+    top = torch.empty(B, H, w.n >> w.levels, w.head_dim, dtype=K.dtype, device="cuda")
+    wf.wf_wavelet_approx(K, w.levels, wv, top)
+    ws = torch.zeros(wf.wf_step_wavelet_workspace_bytes(Q, K, w.levels, w.keep, wv, w.ng), dtype=torch.uint8,
+                     device="cuda")
+    idx = torch.empty(B * H, w.k, dtype=torch.int32, device="cuda")
+    sets = torch.empty(B * H, sum(w.keep), dtype=torch.int32, device="cuda")
+    O = torch.empty_like(Q)
+    wf.wf_step_wavelet(Q, top, K, V, batch.Kg, batch.Vg, w.levels, w.keep, wv, idx, O, ws, level_sets=sets)
+    wf.wf_workspace_status(ws)
+    torch.cuda.synchronize()
+    idx_f, sets_f = _filter_wavelet(batch, w, wv)
+    assert torch.equal(idx, idx_f) and torch.equal(sets, sets_f)
+    for u in units:
+        b, h = divmod(u, w.heads)
+        Qu, Ku = f64(Q[b, h]), f64(K[b, h])
+        mu0, osets = oracle.filter_wavelet(Qu, Ku, w.levels, np.array(w.keep), oracle.DB2, spec32=True,
+                                           store_bf16=True, want_sets=True)
+        gsets = oracle.split_level_sets(sets[u].cpu().numpy(), w.levels, w.keep)
+        for lev in range(w.levels, -1, -1):
+            assert np.array_equal(gsets[lev], osets[lev]), f"unit {u} scale {lev}"
+        assert np.array_equal(idx[u].cpu().numpy(), mu0)
+    idx_h = idx.cpu().numpy()
+    for u in range(w.units):
+        b, h = divmod(u, w.heads)
+        ref = oracle.sparse_attn(f64(Q[b, h]), f64(K[b, h]), f64(V[b, h]), idx_h[u], f64(batch.Kg[b, h]),
+                                 f64(batch.Vg[b, h]))
+        assert_close_out(f64(O[b, h]), ref, torch.bfloat16)
