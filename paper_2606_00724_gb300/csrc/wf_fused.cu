@@ -1466,6 +1466,10 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     for (int e = tid; e < (int)((sizeof(SelScratch) + 15) / 16); e += NT)
       *reinterpret_cast<uint4*>(sc + 16 * e) = make_uint4(0, 0, 0, 0);
   }
+  // Global memory only after the grids this launch depends on are done (the
+  // set-up above overlaps their tail when the launch is programmatic).
+  grid_dep_wait();
+  grid_dep_launch();
   // A launch that starts below the top scale: the previous selection
   // J_{lev_top+1} from the children list it was handed (halved).
   if (c.lev_top < p.L) {
@@ -1736,13 +1740,15 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   cfg.blockDim = dim3(NT, 1, 1);
   cfg.dynamicSmemBytes = fp.smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = fp.cs;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = range && range->pdl ? 2 : 1;
   cudaError_t e = ensure_smem_limit(fp.stages, cfg.dynamicSmemBytes);
   if (e != cudaSuccess) return e;
   e = fp.stages == 4 ? cudaLaunchKernelEx(&cfg, wf_fused_kernel<4>, p) : cudaLaunchKernelEx(&cfg, wf_fused_kernel<3>, p);
@@ -1764,10 +1770,11 @@ cudaError_t launch_literal_fused(const FusedPlan& fp, const FilterPlan& fl, cons
   for (int l = L; l >= 1; --l) {
     // Scale l's rows: the whole prompt's scale-L rows at the top, else the
     // transform of the candidates' gathered blocks, in candidate order.
-    if (l < L && (e = launch_wavelet_approx(K, kv, cur, fl.cmax, m, l, wavelet, arows, (int64_t)fl.cmax * D, s)) !=
-                     cudaSuccess)
+    if (l < L && (e = launch_wavelet_approx(K, kv, cur, fl.cmax, m, l, wavelet, arows, (int64_t)fl.cmax * D, s,
+                                            true)) != cudaSuccess)
       return e;
     FusedRange r{};
+    r.pdl = l < L;  // every launch after the first follows one of this pipeline's own
     r.lev_top = l;
     r.lev_bot = (l == 1 && fl.trim) ? 0 : l;
     r.final_sel = l == 1;

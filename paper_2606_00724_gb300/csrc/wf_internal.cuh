@@ -97,8 +97,10 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
 // WF_WAVELET_*) of the keys of blocks [2^level c, 2^level (c + 1)) for the m
 // candidates c of every unit (cand: [units][cand_stride], NULL = all blocks),
 // into out[unit * out_unit + j * head_dim + channel] in the key dtype.
+// pdl: launch as a programmatic dependent of the previous kernel on the stream.
 cudaError_t launch_wavelet_approx(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m,
-                                  int level, int wavelet, void* out, int64_t out_unit, cudaStream_t s);
+                                  int level, int wavelet, void* out, int64_t out_unit, cudaStream_t s,
+                                  bool pdl = false);
 int wavelet_taps(int wavelet);       // 0 for an unknown basis
 int wavelet_max_level(int wavelet);  // deepest scale the approximation kernel supports
 // Filtering with a generic basis (Eq. 11 taken literally): the filter plan's
@@ -148,8 +150,10 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
 // jout unless final_sel (then mu^0 goes to idx); the attention if attn.
 // Scale lev_top's rows come from lrows ([units][m][d], unit stride lrows_unit
 // elements) when not null, else from the pyramid.
+// pdl: launch as a programmatic dependent of the previous kernel on the
+// stream (its set-up overlaps that kernel's tail).
 struct FusedRange {
-  int lev_top, lev_bot, final_sel, attn;
+  int lev_top, lev_bot, final_sel, attn, pdl;
   const int32_t* jin;
   int32_t* jout;
   int64_t jstride;

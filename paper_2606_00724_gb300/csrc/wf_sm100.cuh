@@ -227,6 +227,15 @@ __device__ __forceinline__ bool abort_set(uint32_t abort_a) {
   asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(abort_a) : "memory");
   return v != 0;
 }
+// Programmatic dependent launch.  grid_dep_wait: wait until the grids this
+// one depends on have completed and their memory is visible (a no-op for a
+// launch without the programmatic-serialization attribute).
+// grid_dep_launch: allow the next dependent grid to be scheduled (it starts
+// once every CTA of this grid has called this or exited, and waits in its own
+// grid_dep_wait before touching memory).
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Global nanosecond timer.
 __device__ __forceinline__ unsigned long long globaltimer_ns() {
   unsigned long long t;

@@ -193,6 +193,8 @@ __global__ void __launch_bounds__(NTH, 3) approx_kernel(const T* __restrict__ K,
   const int blk_mask = (1 << level) - 1;
   const int32_t* cd = cand ? cand + (int64_t)u * cand_stride : nullptr;
   const int tid = threadIdx.x;
+  grid_dep_wait();  // the candidates (and the output's previous readers) come from the grids before
+  grid_dep_launch();
 
   // Row r is gathered position (j0 2^b + r) mod len: its token first, then
   // 16-byte copies, VT a row.
@@ -253,7 +255,7 @@ size_t approx_smem(int level, int ds) {
 
 template <typename T, int TAPS, int DS>
 cudaError_t run_ds(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m, int level,
-                   const Taps& taps, void* out, int64_t out_unit, cudaStream_t s) {
+                   const Taps& taps, void* out, int64_t out_unit, cudaStream_t s, bool pdl) {
   const int to = outputs_per_cta(level);
   const size_t smem = approx_smem<T, TAPS>(level, DS);
   // The shared-memory limit, raised per device to the largest size requested
@@ -272,11 +274,20 @@ cudaError_t run_ds(const void* K, const wf_tensor& kv, const int32_t* cand, int6
       cur = smem;
     }
   }
-  const dim3 grid((unsigned)(kv.head_dim / DS), (unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads));
-  approx_kernel<T, TAPS, DS><<<grid, NTH, smem, s>>>(static_cast<const T*>(K), kv.stride_b, kv.stride_h,
-                                                     kv.stride_s, kv.seq, make_fastdiv((uint32_t)kv.heads), cand,
-                                                     cand_stride, m, level, taps, static_cast<T*>(out), out_unit,
-                                                     kv.head_dim);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)(kv.head_dim / DS), (unsigned)((m + to - 1) / to), (unsigned)(kv.batch * kv.heads));
+  cfg.blockDim = dim3(NTH, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  e = cudaLaunchKernelEx(&cfg, approx_kernel<T, TAPS, DS>, static_cast<const T*>(K), kv.stride_b, kv.stride_h,
+                         kv.stride_s, (int64_t)kv.seq, make_fastdiv((uint32_t)kv.heads), cand, cand_stride, m, level,
+                         taps, static_cast<T*>(out), out_unit, (int64_t)kv.head_dim);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -286,12 +297,12 @@ cudaError_t run_ds(const void* K, const wf_tensor& kv, const int32_t* cand, int6
 // whole rows 265 us a step against 301 with 64 channels.
 template <typename T, int TAPS>
 cudaError_t run(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m, int level,
-                const Taps& taps, void* out, int64_t out_unit, cudaStream_t s) {
+                const Taps& taps, void* out, int64_t out_unit, cudaStream_t s, bool pdl) {
   if (kv.head_dim == 128 && approx_smem<T, TAPS>(level, 128) <= 200 * 1024)
-    return run_ds<T, TAPS, 128>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+    return run_ds<T, TAPS, 128>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl);
   if (approx_smem<T, TAPS>(level, 64) <= 200 * 1024)
-    return run_ds<T, TAPS, 64>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
-  return run_ds<T, TAPS, 16>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+    return run_ds<T, TAPS, 64>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl);
+  return run_ds<T, TAPS, 16>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl);
 }
 
 }  // namespace
@@ -301,18 +312,18 @@ int wavelet_taps(int wavelet) { return wavelet == WF_WAVELET_HAAR ? 2 : (wavelet
 int wavelet_max_level(int wavelet) { return wavelet == WF_WAVELET_DB2 ? 8 : 10; }
 
 cudaError_t launch_wavelet_approx(const void* K, const wf_tensor& kv, const int32_t* cand, int64_t cand_stride, int m,
-                                  int level, int wavelet, void* out, int64_t out_unit, cudaStream_t s) {
+                                  int level, int wavelet, void* out, int64_t out_unit, cudaStream_t s, bool pdl) {
   Taps taps{};
   if (wavelet == WF_WAVELET_DB2) {
     // Daubechies' two-vanishing-moment scaling filter, from its closed form.
     const double r = sqrt(3.0), q = 4.0 * sqrt(2.0);
     const double h[4] = {(1.0 + r) / q, (3.0 + r) / q, (3.0 - r) / q, (1.0 - r) / q};
     for (int k = 0; k < 4; ++k) taps.h[k] = (float)h[k];
-    return kv.dtype == WF_BF16 ? run<bf16, 4>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s)
-                               : run<float, 4>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+    return kv.dtype == WF_BF16 ? run<bf16, 4>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl)
+                               : run<float, 4>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl);
   }
-  return kv.dtype == WF_BF16 ? run<bf16, 2>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s)
-                             : run<float, 2>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s);
+  return kv.dtype == WF_BF16 ? run<bf16, 2>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl)
+                             : run<float, 2>(K, kv, cand, cand_stride, m, level, taps, out, out_unit, s, pdl);
 }
 
 }  // namespace wf
