@@ -11,8 +11,10 @@
 //   * one MMA thread issues tcgen05.mma (bf16 in, fp32 out) per landed tile,
 //     writing S^T = rows . Q^T into the unit's TMEM region (32 columns per
 //     tile), and in the attention O^T += V_s^T P^T;
-//   * four compute warps (one per TMEM lane quarter, one candidate row per
-//     thread) read the logits back (tcgen05.ld), form the per-query max and
+//   * four compute warps per unit (one per TMEM lane quarter, one candidate
+//     row per thread; both warpgroups, taking alternate tiles, when a
+//     cluster serves one unit with long candidate lists) read the logits
+//     back (tcgen05.ld), form the per-query max and
 //     sum of exp of the slice, exchange them with the cluster (st.async into
 //     every CTA, completion counted on its mbarrier), compute the ranking key
 //     log2 W_j (Eq. 8) of each candidate, all-gather the keys the same way,
@@ -78,6 +80,8 @@ constexpr int MAXT = 16;  // TMEM tiles of one unit's region (512 columns / 32)
 struct UnitState {
   float2 xstat[MAXCS][NQ];  // (stabiliser, sum of exp) of every cluster CTA's slice
   float2 cstat[MAXCS][NQ];  // attention (max, row sum) of every CTA (d-slice owner side)
+  // Per-warp slots (warp w of the unit at slot w; a WIDE unit's warps 4-7 use
+  // the second unit's slots, which nothing else uses then).
   float2 kmm[MAXCS][NCW];   // (min, max) of the ranking keys of every cluster warp
   float2 wstat[NCW][NQ];    // (stabiliser, sum of exp) of each compute warp's rows
   float cw[NCW][NQ];        // softmax normaliser c_i, one copy per compute warp
@@ -98,6 +102,12 @@ struct Misc {
   int abort;
   uint32_t tmem_base;
 };
+
+// The UnitState holding the per-warp slots of unit warp w (index w % 4).
+template <bool WIDE>
+__device__ __forceinline__ UnitState& wslots(Misc& ms, int pp, int w) {
+  return WIDE ? ms.us[w >> 2] : ms.us[pp];
+}
 
 // Shared-memory layout (byte offsets; the stage ring starts at 0, 1024-byte
 // aligned for the 128-byte swizzle).
@@ -165,9 +175,32 @@ struct Ctx {
   int np, u0, lev_top, lev_end, stages;
 };
 
-// Thread index within its unit's compute warps, and their barrier.
-__device__ __forceinline__ int ctid() { return threadIdx.x & (NCT - 1); }
-__device__ __forceinline__ void csync() { named_sync(kCsyncId + (threadIdx.x >> 7), NCT); }
+// A unit's compute warps: one warpgroup (one per unit of a two-unit cluster),
+// or both warpgroups (WIDE) when the cluster serves one unit; then the
+// warpgroups take alternate tiles and share the Top-K.  Thread index within
+// the unit's compute warps, their count and their barrier.
+template <bool WIDE>
+__host__ __device__ constexpr int unit_warps() {
+  return WIDE ? 2 * NCW : NCW;
+}
+template <bool WIDE>
+__device__ __forceinline__ int ctid() {
+  return threadIdx.x & (32 * unit_warps<WIDE>() - 1);
+}
+template <bool WIDE>
+__device__ __forceinline__ void csync() {
+  named_sync(kCsyncId + (WIDE ? 0u : (threadIdx.x >> 7)), 32 * unit_warps<WIDE>());
+}
+// The warpgroup of a compute thread within its unit (0 unless WIDE), the
+// first tile it takes and its tile stride.
+template <bool WIDE>
+__device__ __forceinline__ int unit_wg() {
+  return WIDE ? (int)((threadIdx.x >> 7) & 1) : 0;
+}
+template <bool WIDE>
+__host__ __device__ constexpr int tile_step() {
+  return WIDE ? 2 : 1;
+}
 
 __device__ __forceinline__ bool aborted(const Misc& ms) { return abort_set(smem_u32(&ms.abort)); }
 
@@ -528,25 +561,27 @@ __device__ __forceinline__ float transpose_reduce32(float (&v)[32], int lane) {
 // Top-K scratch.  It lives in the unit's P buffers, which nothing uses before
 // the attention.  The histogram and the list counter are zero between calls
 // (zeroed at kernel start, cleared again at the end of every call).
-constexpr int NB = 2048;  // histogram buckets
-constexpr int BPT = NB / NCT;
+constexpr int NB = 2048;     // histogram buckets
+constexpr int MAXUW = 2 * NCW;  // most compute warps of a unit
 struct SelScratch {
   uint32_t hist[NB];
-  float2 blist[NCT];    // boundary-bucket keys (key, position)
-  float2 sred[2][NCW];  // (min, max) per warp, alternating rounds
-  int wsum[4][NCW];     // per-warp sums of the scans (slot per scan)
+  float2 blist[32 * MAXUW];  // boundary-bucket keys (key, position)
+  float2 sred[2][MAXUW];     // (min, max) per warp, alternating rounds
+  int wsum[4][MAXUW];        // per-warp sums of the scans (slot per scan, 32 bytes)
   uint32_t bcnt;
 };
 static_assert((sizeof(SelScratch) + 15) / 16 * 16 <= UNIT_P_BYTES, "Top-K scratch must fit the P buffers");
-static_assert(BPT % 4 == 0, "buckets are cleared four at a time");
+static_assert((NB / NCT) % 8 == 0, "buckets are cleared four at a time by up to twice NCT threads");
+static_assert(offsetof(SelScratch, wsum) % 16 == 0, "the scan's warp sums are read 16 bytes at a time");
 
 #define SC_ADDR(sc_a, field) ((sc_a) + (uint32_t)offsetof(SelScratch, field))
 
-// Exclusive prefix sum over the compute threads (thread order), with its
-// per-warp sums in the NCW words at wsum_a.  One barrier: the caller does not
+// Exclusive prefix sum over the unit's compute threads (thread order), with
+// its per-warp sums in the words at wsum_a.  One barrier: the caller does not
 // reuse those words before another barrier has passed.
+template <bool WIDE>
 __device__ __forceinline__ int cta_excl_scan(int v, uint32_t wsum_a) {
-  const int lane = threadIdx.x & 31, warp = ctid() >> 5;
+  const int lane = threadIdx.x & 31, warp = ctid<WIDE>() >> 5;
   int incl = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -554,9 +589,14 @@ __device__ __forceinline__ int cta_excl_scan(int v, uint32_t wsum_a) {
     if (lane >= o) incl += t;
   }
   if (lane == 31) sts_u32(wsum_a + 4u * warp, (uint32_t)incl);
-  csync();
-  const uint4 w = lds_v4(wsum_a);
-  const int before = (warp > 0 ? (int)w.x : 0) + (warp > 1 ? (int)w.y : 0) + (warp > 2 ? (int)w.z : 0);
+  csync<WIDE>();
+  int before = 0;
+#pragma unroll
+  for (int q = 0; q < unit_warps<WIDE>() / 4; ++q) {
+    const uint4 w = lds_v4(wsum_a + 16u * q);
+    before += (warp > 4 * q ? (int)w.x : 0) + (warp > 4 * q + 1 ? (int)w.y : 0) + (warp > 4 * q + 2 ? (int)w.z : 0) +
+              (warp > 4 * q + 3 ? (int)w.w : 0);
+  }
   return before + incl - v;
 }
 
@@ -577,9 +617,9 @@ __device__ __forceinline__ int ffs_m(unsigned long long x) { return __ffsll((lon
 
 // (min, max) of the undecided keys (bit i of act: position j0 + i of the key
 // array) over the compute threads, via slot `par`.
-template <typename MT>
+template <typename MT, bool WIDE>
 __device__ __forceinline__ float2 cta_minmax(uint32_t keys_a, int j0, MT act, uint32_t sc_a, int par) {
-  const int lane = threadIdx.x & 31, warp = ctid() >> 5;
+  const int lane = threadIdx.x & 31, warp = ctid<WIDE>() >> 5;
   float lo = INFINITY, hi = -INFINITY;
 #pragma unroll 1
   for (MT a = act; a; a &= a - 1) {
@@ -589,11 +629,11 @@ __device__ __forceinline__ float2 cta_minmax(uint32_t keys_a, int j0, MT act, ui
   }
   lo = warp_min_f32(lo);
   hi = warp_max_f32(hi);
-  if (lane == 0) sts_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + warp), __float_as_uint(lo), __float_as_uint(hi));
-  csync();
+  if (lane == 0) sts_v2(SC_ADDR(sc_a, sred) + 8u * (par * MAXUW + warp), __float_as_uint(lo), __float_as_uint(hi));
+  csync<WIDE>();
 #pragma unroll
-  for (int w = 0; w < NCW; ++w) {
-    const uint2 r = lds_v2(SC_ADDR(sc_a, sred) + 8u * (par * NCW + w));
+  for (int w = 0; w < unit_warps<WIDE>(); ++w) {
+    const uint2 r = lds_v2(SC_ADDR(sc_a, sred) + 8u * (par * MAXUW + w));
     lo = fminf(lo, __uint_as_float(r.x));
     hi = fmaxf(hi, __uint_as_float(r.y));
   }
@@ -659,15 +699,17 @@ __device__ __forceinline__ uint3 warp_boundary(uint32_t hist_a, uint32_t need, i
 // arithmetic is monotone, so a key in a higher bucket is strictly larger);
 // every warp then finds the bucket holding the boundary from the counts: keys
 // above it are taken, keys below it dropped.  A boundary bucket of at most
-// NCT keys is resolved exactly, each owner ranking its keys on
+// as many keys as the unit has threads is resolved exactly, each owner ranking its keys on
 // (key, -position) against the bucket's list; a larger one is bucketed again
 // over its own range.  If only equal keys remain, the lowest positions are
 // taken.
-template <typename MT>
+template <typename MT, bool WIDE>
 __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                          float lo, float hi, int R) {
   constexpr int MB = 8 * (int)sizeof(MT);       // positions a mask holds
-  const int tid = ctid(), lane = tid & 31;
+  constexpr int TN = 32 * unit_warps<WIDE>();   // the unit's compute threads
+  constexpr int BPT = NB / TN;                  // buckets each thread clears
+  const int tid = ctid<WIDE>(), lane = tid & 31;
   const int j0 = tid * R;
   const int G = R >> 2;                         // groups of four keys in a run
   const int rotg = ((lane * G) >> 3) & (G - 1);  // first group this lane visits
@@ -700,7 +742,7 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
       reds_add_if(a4 & 4u, hist_a + 4u * b2, 1u);
       reds_add_if(a4 & 8u, hist_a + 4u * b3, 1u);
     }
-    csync();
+    csync<WIDE>();
     const uint3 bd = warp_boundary(hist_a, need, lane);
     const int sb = (int)bd.x;
     need = bd.y;
@@ -724,7 +766,7 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
       resolved = true;
       break;
     }
-    if (cnt <= (uint32_t)NCT) {
+    if (cnt <= (uint32_t)TN) {
       // Append the boundary keys (one atomic per warp), then every owner
       // ranks its own keys against the list.
       const int nb = popc_m(act);
@@ -741,12 +783,12 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
 #pragma unroll 1
       for (MT a = act; a; a &= a - 1, ++slot) {
         const int i = ffs_m(a) - 1;
-        // slot < NCT always (the list holds cnt <= NCT keys); the predicate
+        // slot < TN always (the list holds cnt <= TN keys); the predicate
         // keeps the store in the list should a wait have given up.
-        sts_v2_if(slot < (uint32_t)NCT, SC_ADDR(sc_a, blist) + 8u * slot, lds_u32(keys_a + 4u * (uint32_t)(j0 + i)),
+        sts_v2_if(slot < (uint32_t)TN, SC_ADDR(sc_a, blist) + 8u * slot, lds_u32(keys_a + 4u * (uint32_t)(j0 + i)),
                   (uint32_t)(j0 + i));
       }
-      csync();
+      csync<WIDE>();
 #pragma unroll 1
       for (MT a = act; a; a &= a - 1) {
         const int i = ffs_m(a) - 1;
@@ -771,17 +813,17 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
       break;
     }
     // The boundary bucket again over its own range, with a cleared histogram.
-    csync();  // every warp has read the histogram
+    csync<WIDE>();  // every warp has read the histogram
 #pragma unroll
     for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
-    const float2 lh = cta_minmax(keys_a, j0, act, sc_a, iter & 1);  // its barrier also publishes the cleared buckets
+    const float2 lh = cta_minmax<MT, WIDE>(keys_a, j0, act, sc_a, iter & 1);  // its barrier also publishes the cleared buckets
     lo = lh.x;
     hi = lh.y;
   }
   MT take = took;
   if (!resolved) {
     // Only equal keys are undecided: the first `need` by position are taken.
-    const int eq_base = cta_excl_scan(popc_m(act), SC_ADDR(sc_a, wsum) + 48u);
+    const int eq_base = cta_excl_scan<WIDE>(popc_m(act), SC_ADDR(sc_a, wsum) + 96u);
     int remaining = (int)need - eq_base;
     for (MT e = act; e && remaining > 0; --remaining) {
       const MT low = e & (~e + 1);
@@ -794,7 +836,7 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
   // entries (j0 + 4g) / 2 and that + 1).  The scan's barrier orders every read
   // of the keys, the histogram and the boundary list before the key array is
   // overwritten and the scratch cleared.
-  int r = cta_excl_scan(popc_m(take), SC_ADDR(sc_a, wsum) + 32u);
+  int r = cta_excl_scan<WIDE>(popc_m(take), SC_ADDR(sc_a, wsum) + 64u);
 #pragma unroll 1
   for (int g = 0; g < G; ++g) {
     const uint32_t t4 = (uint32_t)(take >> (4 * g)) & 15u;
@@ -819,34 +861,38 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
 #pragma unroll
   for (int i = 0; i < BPT / 4; ++i) sts_v4(own_a + 16u * i, make_uint4(0, 0, 0, 0));
   if (tid == 0) sts_u32(SC_ADDR(sc_a, bcnt), 0u);
-  csync();
+  csync<WIDE>();
 }
 
-// Top-K dispatch: R = the smallest power of two (at least 4) with R NCT >= m
-// (m <= 64 NCT); 64-bit position masks only for R = 64.
+// Top-K dispatch: R = the smallest power of two (at least 4) with R TN >= m
+// (m <= 64 NCT, TN the unit's compute threads); 64-bit position masks only
+// for R = 64.
+template <bool WIDE>
 __device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                             float lo, float hi) {
   int R = 4;
-  while (R * NCT < m) R <<= 1;
-  if (R <= 32) select_keys<uint32_t>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
-  else select_keys<unsigned long long>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
+  while (R * 32 * unit_warps<WIDE>() < m) R <<= 1;
+  if (WIDE || R <= 32) select_keys<uint32_t, WIDE>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
+  else select_keys<unsigned long long, WIDE>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
 }
 
 // Per-query max (x sl2, log2 units) of the valid rows of TMEM tiles
-// 0..ntl-1 of region tb -> us.mloc.  The column maxima across a warp come
-// from the warp-wide max instruction.
-__device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int ntl, int mc, float sl2) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+// 0..ntl-1 of region tb (this warpgroup's share of them) -> mloc of unit pp.
+// The column maxima across a warp come from the warp-wide max instruction.
+template <bool WIDE>
+__device__ __noinline__ void pass_max(Misc& ms, int pp, uint32_t tb, int ntl, int mc, float sl2) {
+  const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
+  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+  UnitState& us = ms.us[pp];
   float mx[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) mx[i] = -INFINITY;
 #pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
+  for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
     uint32_t ra[32];
     tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    if (t * TM + tid < mc) {
+    if (t * TM + row < mc) {
 #pragma unroll
       for (int i = 0; i < 32; ++i) mx[i] = fmaxf(mx[i], __uint_as_float(ra[i]));
     }
@@ -856,41 +902,43 @@ __device__ __noinline__ void pass_max(Misc& ms, UnitState& us, uint32_t tb, int 
   if (lane == 0) {
 #pragma unroll
     for (int i = 0; i < 32; i += 4)
-      sts_v4(smem_u32(&us.red[warp][i]), make_uint4(__float_as_uint(mx[i]), __float_as_uint(mx[i + 1]),
-                                                    __float_as_uint(mx[i + 2]), __float_as_uint(mx[i + 3])));
+      sts_v4(smem_u32(&wslots<WIDE>(ms, pp, warp).red[warp & 3][i]),
+             make_uint4(__float_as_uint(mx[i]), __float_as_uint(mx[i + 1]), __float_as_uint(mx[i + 2]),
+                        __float_as_uint(mx[i + 3])));
   }
-  csync();
+  csync<WIDE>();
   if (tid < 32) {
     float m = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < NCW; ++w) m = fmaxf(m, us.red[w][tid]);
+    for (int w = 0; w < unit_warps<WIDE>(); ++w) m = fmaxf(m, wslots<WIDE>(ms, pp, w).red[w & 3][tid]);
     us.mloc[tid] = m * sl2;
   }
-  csync();
+  csync<WIDE>();
 }
 
 // The warp's (stabiliser, sum of 2^(l sl2 - stabiliser)) per query over its
 // rows of TMEM tiles 0..ntl-1, with the stabiliser the column maximum over
 // all those rows: the overflow path of scale_sums, one query column at a
 // time (compact code for a path that real inputs never take).
+template <bool WIDE>
 __device__ __noinline__ float2 warp_sums_exact(uint32_t tb, int ntl, int mc, float sl2) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
+  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
   float2 out = make_float2(-INFINITY, 0.f);
 #pragma unroll 1
   for (int i = 0; i < 32; ++i) {
     float mx = -INFINITY;
 #pragma unroll 1
-    for (int t = 0; t < ntl; ++t) {
+    for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
       const float v = tmem_ld1(tb + lane_base + 32 * t + i);
-      if (t * TM + tid < mc) mx = fmaxf(mx, v);
+      if (t * TM + row < mc) mx = fmaxf(mx, v);
     }
     const float mi = warp_max_f32(mx) * sl2;
     float sum = 0.f;
 #pragma unroll 1
-    for (int t = 0; t < ntl; ++t) {
+    for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
       const float v = tmem_ld1(tb + lane_base + 32 * t + i);
-      if (t * TM + tid < mc) sum += ex2(fmaf(v, sl2, -mi));
+      if (t * TM + row < mc) sum += ex2(fmaf(v, sl2, -mi));
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
@@ -909,10 +957,12 @@ __device__ __noinline__ float2 warp_sums_exact(uint32_t tb, int ntl, int mc, flo
 // maximum over all its rows.  The four warps' (m, sum) merge into the CTA's
 // (M, S) per query, which goes to slot `rank` of every cluster CTA's xstat.
 // tpar holds the parity of each tile barrier's next phase.
-__device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
-                                        int ntl, int mc, float sl2, uint32_t ecol, uint32_t& tpar, int* status) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+template <bool WIDE>
+__device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, int pp, uint32_t tb, int ntl, int mc,
+                                        float sl2, uint32_t ecol, uint32_t& tpar, int* status) {
+  const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
+  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+  UnitState& us = ms.us[pp];
   const f32x2 s2 = pk2(sl2, sl2);
   f32x2 nml[16], acc[16];
   float mcol = -INFINITY;  // lane i: this warp's stabiliser of query i
@@ -922,15 +972,15 @@ __device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
     nml[k] = pk2(0.f, 0.f);
   }
 #pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
+  for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
     wait_or_abort(bar_addr(ms.tdone[pp][t]), (tpar >> t) & 1u, ms, status);
     tpar ^= 1u << t;
     tc_fence_after();
     uint32_t ra[32];
     tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
-    const bool valid = t * TM + tid < mc;
-    if (t == 0) {
+    const bool valid = t * TM + row < mc;
+    if (t == unit_wg<WIDE>()) {
       float m2[2];
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
@@ -963,23 +1013,24 @@ __device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
   }
   float2 st = make_float2(mcol, transpose_reduce32<false>(a, lane));
   const bool overflow = __any_sync(0xffffffffu, !(st.y <= 3.0e38f));
-  if (overflow) st = warp_sums_exact(tb, ntl, mc, sl2);
-  sts_v2(smem_u32(&us.wstat[warp][lane]), __float_as_uint(st.x), __float_as_uint(st.y));
-  csync();
+  if (overflow) st = warp_sums_exact<WIDE>(tb, ntl, mc, sl2);
+  sts_v2(smem_u32(&wslots<WIDE>(ms, pp, warp).wstat[warp & 3][lane]), __float_as_uint(st.x), __float_as_uint(st.y));
+  csync<WIDE>();
   if (tid < 32) {
-    float2 w[NCW];
+    constexpr int NW = unit_warps<WIDE>();
+    float2 w[NW];
 #pragma unroll
-    for (int k = 0; k < NCW; ++k) {
-      const uint2 v = lds_v2(smem_u32(&us.wstat[k][tid]));
+    for (int k = 0; k < NW; ++k) {
+      const uint2 v = lds_v2(smem_u32(&wslots<WIDE>(ms, pp, k).wstat[k & 3][tid]));
       w[k] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
     }
     float M = -INFINITY;
 #pragma unroll
-    for (int k = 0; k < NCW; ++k)
+    for (int k = 0; k < NW; ++k)
       if (w[k].y > 0.f) M = fmaxf(M, w[k].x);
     float S = 0.f;
 #pragma unroll
-    for (int k = 0; k < NCW; ++k)
+    for (int k = 0; k < NW; ++k)
       if (w[k].y > 0.f) S = fmaf(w[k].y, ex2(w[k].x - M), S);
     const uint32_t dst = smem_u32(&us.xstat[rank][tid]);
     const uint32_t bar = bar_addr(ms.xbar[pp]);
@@ -994,10 +1045,13 @@ __device__ __noinline__ bool scale_sums(uint32_t rank, uint32_t cs, Misc& ms, Un
 
 // Softmax normaliser per query, c_i = M + log2 S over the whole candidate
 // set from the cluster's (M, S) pairs (padded query columns get +inf and
-// weigh 0), into this warp's copy us.cw[warp].  Every warp forms its own copy,
+// weigh 0), into this warp's slot of cw.  Every warp forms its own copy,
 // so no barrier across the warps is needed.
-__device__ __forceinline__ void warp_normaliser(UnitState& us, uint32_t cs, int q) {
-  const int lane = threadIdx.x & 31, warp = ctid() >> 5;
+template <bool WIDE>
+__device__ __forceinline__ void warp_normaliser(Misc& ms, int pp, uint32_t cs, int q) {
+  const int lane = threadIdx.x & 31, warp = ctid<WIDE>() >> 5;
+  UnitState& us = ms.us[pp];
+  UnitState& ws = wslots<WIDE>(ms, pp, warp);
   float2 st[MAXCS];
 #pragma unroll
   for (int r = 0; r < MAXCS; ++r) {
@@ -1013,8 +1067,8 @@ __device__ __forceinline__ void warp_normaliser(UnitState& us, uint32_t cs, int 
   for (int r = 0; r < MAXCS; ++r)
     if (r < (int)cs && st[r].y > 0.f) S = fmaf(st[r].y, ex2(st[r].x - M), S);
   const float c = lane < q ? M + lg2(S) : INFINITY;
-  us.cw[warp][lane] = c;
-  us.fw[warp][lane] = ex2(us.wstat[warp][lane].x - c);  // 0 for padded columns and for a warp without rows
+  ws.cw[warp & 3][lane] = c;
+  ws.fw[warp & 3][lane] = ex2(ws.wstat[warp & 3][lane].x - c);  // 0 for padded columns and for a warp without rows
   __syncwarp();
 }
 
@@ -1070,12 +1124,14 @@ __device__ __forceinline__ float key_from_logits(const uint32_t (&ra)[32], uint3
   return key;
 }
 
-__device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, UnitState& us, int pp, uint32_t tb,
-                                       int ntl, int mc, int g0, float sl2, uint32_t keys_a, uint32_t ecol, bool eok) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+template <bool WIDE>
+__device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, int pp, uint32_t tb, int ntl, int mc,
+                                       int g0, float sl2, uint32_t keys_a, uint32_t ecol, bool eok) {
+  const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
+  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
   const uint32_t bar = bar_addr(ms.kbar[pp]);
-  const uint32_t cw_a = smem_u32(&us.cw[warp][0]);
+  UnitState& ws = wslots<WIDE>(ms, pp, warp);
+  const uint32_t cw_a = smem_u32(&ws.cw[warp & 3][0]);
   float kmin = INFINITY, kmax = -INFINITY;
   // After a wait gave up, this CTA sends nothing to the cluster.
   const uint32_t nr = aborted(ms) ? 0u : cs;
@@ -1090,7 +1146,7 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, Uni
   };
   if (eok) {
     f32x2 fv[16];
-    const uint32_t fw_a = smem_u32(&us.fw[warp][0]);
+    const uint32_t fw_a = smem_u32(&ws.fw[warp & 3][0]);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       const uint4 f = lds_v4(fw_a + 16u * k);
@@ -1098,7 +1154,7 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, Uni
       fv[2 * k + 1] = pk2(__uint_as_float(f.z), __uint_as_float(f.w));
     }
 #pragma unroll 1
-    for (int t = 0; t < ntl; ++t) {
+    for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
       uint32_t ra[32];
       tmem_ld32_issue(tb + ecol + lane_base + 32 * t, ra);
       tmem_wait_ld();
@@ -1107,7 +1163,7 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, Uni
       for (int k = 0; k < 16; ++k) z2 = fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), fv[k], z2);
       const float2 zz = up2(z2);
       float key = lg2(zz.x + zz.y);
-      const int j = t * TM + tid;
+      const int j = t * TM + row;
       const bool slow = zz.x + zz.y < 0x1p-96f;
       if (__any_sync(0xffffffffu, slow && j < mc)) {
         // A tiny W: the exact key from the logits (the whole warp reloads them;
@@ -1122,18 +1178,18 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, Uni
     }
   } else {
 #pragma unroll 1
-    for (int t = 0; t < ntl; ++t) {
+    for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
       uint32_t ra[32];
       tmem_ld32_issue(tb + lane_base + 32 * t, ra);
       tmem_wait_ld();
-      emit(t * TM + tid, key_from_logits(ra, cw_a, sl2));
+      emit(t * TM + row, key_from_logits(ra, cw_a, sl2));
     }
   }
   // The warp's key range goes with the keys (the Top-K's first bucket range).
   kmin = warp_min_f32(kmin);
   kmax = warp_max_f32(kmax);
   if (lane == 0) {
-    const uint32_t dst = smem_u32(&us.kmm[rank][warp]);
+    const uint32_t dst = smem_u32(&ws.kmm[rank][warp & 3]);
 #pragma unroll 1
     for (uint32_t r = 0; r < nr; ++r)
       st_async_v2(map_rank(dst, r), __float_as_uint(kmin), __float_as_uint(kmax), map_rank(bar, r));
@@ -1145,10 +1201,14 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, Uni
 // Attention: P = 2^(s - m) (bf16, P^T MN-major core matrices) of every S tile
 // into the unit's P double buffer for the MMA thread, and the row sums of P
 // -> us.lacc.
-__device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* pbase, UnitState& us, int pp,
-                                    uint32_t tb, int ntl, int mc) {
-  const int tid = ctid(), lane = tid & 31, warp = tid >> 5;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+// WIDE: each warpgroup forms the P tiles of its tiles (t = wg, wg + 2, ...),
+// so each always fills the same one of the two buffers.
+template <bool WIDE>
+__device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* pbase, int pp, uint32_t tb, int ntl,
+                                    int mc) {
+  const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
+  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+  UnitState& us = ms.us[pp];
   const f32x2 s2 = pk2(sl2, sl2);
   f32x2 nml[16], lsum2[16];
 #pragma unroll
@@ -1157,7 +1217,7 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
     lsum2[k] = pk2(0.f, 0.f);
   }
 #pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
+  for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
     const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
     if (t >= 2) {
       if (lane == 0) wait_or_abort(bar_addr(ms.pempty[pp][pb]), (pn - 1) & 1u, ms, status);
@@ -1167,7 +1227,7 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
     tmem_ld32_issue(tb + lane_base + 32 * t, ra);
     tmem_wait_ld();
     uint32_t w[16];
-    if (t * TM + tid < mc) {
+    if (t * TM + row < mc) {
 #pragma unroll
       for (int k = 0; k < 16; ++k) {
         const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
@@ -1180,7 +1240,7 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
       for (int k = 0; k < 16; ++k) w[k] = 0u;  // rows past the slice: P = 0
     }
     // P^T, MN-major core matrices: key group r / 8, query chunk ch.
-    const int r = tid;
+    const int r = row;
     uint8_t* dst = pbase + pb * P_BYTES + (r >> 3) * 512 + (r & 7) * 16;
 #pragma unroll
     for (int ch = 0; ch < 4; ++ch)
@@ -1197,15 +1257,15 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
     lsum[2 * k] = v.x;
     lsum[2 * k + 1] = v.y;
   }
-  us.red[warp][lane] = transpose_reduce32<false>(lsum, lane);
-  csync();
+  wslots<WIDE>(ms, pp, warp).red[warp & 3][lane] = transpose_reduce32<false>(lsum, lane);
+  csync<WIDE>();
   if (tid < 32) {
     float sum = 0.f;
 #pragma unroll
-    for (int w = 0; w < NCW; ++w) sum += us.red[w][tid];
+    for (int w = 0; w < unit_warps<WIDE>(); ++w) sum += wslots<WIDE>(ms, pp, w).red[w & 3][tid];
     us.lacc[tid] = sum;
   }
-  csync();
+  csync<WIDE>();
 }
 
 // Attention combine of unit pp: this CTA's partial O^T rows go to the CTA
@@ -1214,9 +1274,10 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
 // columns of O (bf16).  The partials land in each owner's P buffers of the
 // unit, which are free once the owner's own PV products are done; owners
 // announce that before any partial is sent.
+// (Run by one warpgroup of the unit: four warps, one per TMEM lane quarter.)
 __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32_t rank, uint32_t cs, int u,
                                           uint8_t* comb, UnitState& us, int pp, uint32_t ocol) {
-  const int tid = ctid(), warp = tid >> 5;
+  const int tid = threadIdx.x & (NCT - 1), warp = tid >> 5;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   uint32_t orow[32];
   tmem_ld32_issue(ocol + lane_base, orow);
@@ -1304,10 +1365,13 @@ __device__ __noinline__ void attn_combine(Misc& ms, const FusedParams& p, uint32
 }
 
 // The compute warps of unit pp = threadIdx.x / NCT of the cluster's units.
+// WIDE: both warpgroups serve the cluster's one unit.
+template <bool WIDE>
 __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   Misc& ms = *c.ms;
-  const int tid = ctid();
-  const int pp = threadIdx.x / NCT;
+  constexpr int TN = 32 * unit_warps<WIDE>();  // the unit's compute threads
+  const int tid = ctid<WIDE>();
+  const int pp = WIDE ? 0 : threadIdx.x / NCT;
   if (pp >= c.np) return;
   UnitState& us = ms.us[pp];
   uint8_t* ubuf = c.smem + c.ly.p + pp * UNIT_P_BYTES;  // P buffers, Top-K scratch, combine buffer
@@ -1337,54 +1401,58 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     const int kb = p.keep[lev];
     int32_t* J = unit_J(c, p, pp, lev);  // receives this scale's keys, then its selection
     const uint32_t keys_a = smem_u32(J);
-    const bool eok = scale_sums(c.rank, c.cs, ms, us, pp, tb, ntl, mc, sl2, p.ecol, tpar, p.status);
+    const bool eok = scale_sums<WIDE>(c.rank, c.cs, ms, pp, tb, ntl, mc, sl2, p.ecol, tpar, p.status);
     wait_cluster_or_abort(bar_addr(ms.xbar[pp]), ph, ms, p.status);
     // This phase is complete for tid 0, so the arrival arms the next one.
     // After a wait gave up the phase may still be pending (its bytes never
     // came): a second arrival would then underflow the phase's arrival
     // count, so an aborted CTA arms nothing.
     if (tid == 0 && lev > c.lev_end && !aborted(ms)) mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-    warp_normaliser(us, c.cs, p.q);
-    pass_keys(c.rank, c.cs, ms, us, pp, tb, ntl, mc, g0, sl2, keys_a, p.ecol, eok);
+    warp_normaliser<WIDE>(ms, pp, c.cs, p.q);
+    pass_keys<WIDE>(c.rank, c.cs, ms, pp, tb, ntl, mc, g0, sl2, keys_a, p.ecol, eok);
     wait_cluster_or_abort(bar_addr(ms.kbar[pp]), ph, ms, p.status);
     // The keys' range from the cluster warps' (min, max).
     float lo, hi;
     {
+      constexpr int NW = unit_warps<WIDE>();
       const int lane = tid & 31;
       float2 mm = make_float2(INFINITY, -INFINITY);
-      if (lane < (int)c.cs * NCW) {
-        const uint2 v = lds_v2(smem_u32(&us.kmm[lane / NCW][lane % NCW]));
-        mm = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+#pragma unroll 1
+      for (int e = lane; e < (int)c.cs * NW; e += 32) {  // entry (CTA e / NW, warp e % NW)
+        const int w = e % NW;
+        const uint2 v = lds_v2(smem_u32(&wslots<WIDE>(ms, pp, w).kmm[e / NW][w & 3]));
+        mm = make_float2(fminf(mm.x, __uint_as_float(v.x)), fmaxf(mm.y, __uint_as_float(v.y)));
       }
       lo = warp_min_f32(mm.x);
       hi = warp_max_f32(mm.y);
     }
     // Eq. 9: Top-K (the same result in every CTA of the cluster).
-    select_topk(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a, lo, hi);
+    select_topk<WIDE>(keys_a, m, kb, smem_u32(unit_J(c, p, pp, lev + 1)), lev == p.L, sc_a, lo, hi);
     if (tid == 0) {
       if (lev > c.lev_end && !aborted(ms))  // as for xbar above
-        mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, lev - 1) + c.cs * NCW * 8u);
+        mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]),
+                              4u * (uint32_t)m_total(p, lev - 1) + c.cs * unit_warps<WIDE>() * 8u);
       mbar_arrive(bar_addr(ms.jready[pp]));  // the selection is complete (the Top-K ends on a barrier)
     }
     if (c.rank == 0) {
       int32_t* ls = p.level_sets ? p.level_sets + (int64_t)u * p.sets_stride + sets_off : nullptr;
       if (lev >= 1 && ls) {
 #pragma unroll 1
-        for (int i = tid; i < kb; i += NCT) ls[i] = J[i];
+        for (int i = tid; i < kb; i += TN) ls[i] = J[i];
       }
       if (lev == c.lev_end && !p.final_sel) {
         // A launch that ends above the final scale hands on the children of
         // its last selection (the next launch's candidates).
         int32_t* out = p.jout + (int64_t)u * p.jstride;
 #pragma unroll 1
-        for (int t = tid; t < 2 * kb; t += NCT) out[t] = 2 * J[t >> 1] + (t & 1);
+        for (int t = tid; t < 2 * kb; t += TN) out[t] = 2 * J[t >> 1] + (t & 1);
       } else if (lev == c.lev_end) {
         // mu^0: the children of J^1, or the trimmed level-0 selection.
         const int kk = p.keep[0];
         int32_t* out = p.idx + (int64_t)u * kk;
         int32_t* ls0 = ls ? ls + (lev >= 1 ? kb : 0) : nullptr;
 #pragma unroll 1
-        for (int t = tid; t < kk; t += NCT) {
+        for (int t = tid; t < kk; t += TN) {
           const int tok = p.trim ? J[t] : 2 * J[t >> 1] + (t & 1);
           out[t] = tok;
           if (ls0) ls0[t] = tok;
@@ -1400,13 +1468,14 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
   const int ntl = tiles_of(mc);
   if (ntl > 0) wait_mdone();
-  pass_max(ms, us, tb, ntl, mc, sl2);
-  attn_p(ms, p.status, sl2, ubuf, us, pp, tb, ntl, mc);
+  pass_max<WIDE>(ms, pp, tb, ntl, mc, sl2);
+  attn_p<WIDE>(ms, p.status, sl2, ubuf, pp, tb, ntl, mc);
   if (ntl > 0) wait_mdone();
+  if (unit_wg<WIDE>() != 0) return;  // one warpgroup combines
   attn_combine(ms, p, c.rank, c.cs, u, ubuf, us, pp, tb + p.ucols - 32);
 }
 
-template <int S>
+template <int S, bool WIDE>
 __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__ FusedParams p) {
   extern __shared__ __align__(1024) uint8_t smem[];
   Ctx c;
@@ -1451,7 +1520,7 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     // Arm the first phase of every receive barrier (bytes this CTA expects).
     for (int pp = 0; pp < c.np; ++pp) {
       mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, c.lev_top) + c.cs * NCW * 8u);
+      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, c.lev_top) + c.cs * unit_warps<WIDE>() * 8u);
       const uint32_t rows = (uint32_t)(dlo((int)c.rank + 1, c.cs) - dlo((int)c.rank, c.cs));
       mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), c.cs * rows * NQ * 4u + c.cs * NQ * 8u);
     }
@@ -1500,7 +1569,7 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   cluster_sync();  // every CTA's barriers exist before any remote arrival
 
   if (warp < MMA_WARP) {
-    compute_role(c, p);
+    compute_role<WIDE>(c, p);
   } else if (warp == MMA_WARP) {
     if ((tid & 31) == 0) mma_role<S>(c, p);
     __syncwarp();
@@ -1535,31 +1604,39 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
 // ---------------------------------------------------------------------------
 namespace {
 
-// The kernel's dynamic shared-memory limit, raised once per device and stage
-// count to the largest size requested so far instead of on every launch.
-cudaError_t ensure_smem_limit(int stages, size_t smem) {
+// The kernel instance for a stage count and unit width (one-unit plans with
+// long candidate lists run the WIDE instance, whose two warpgroups both serve
+// the unit).
+typedef void (*FusedKernel)(FusedParams);
+FusedKernel fused_kernel(int stages, bool wide) {
+  if (stages == 4) return wide ? wf_fused_kernel<4, true> : wf_fused_kernel<4, false>;
+  return wide ? wf_fused_kernel<3, true> : wf_fused_kernel<3, false>;
+}
+
+// The kernel's dynamic shared-memory limit, raised once per device and
+// instance to the largest size requested so far instead of on every launch.
+cudaError_t ensure_smem_limit(int stages, bool wide, size_t smem) {
   static std::mutex mu;
-  static std::map<std::pair<int, int>, size_t> raised;
+  static std::map<std::tuple<int, int, bool>, size_t> raised;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   std::lock_guard<std::mutex> lock(mu);
-  size_t& cur = raised[std::make_pair(dev, stages)];
+  size_t& cur = raised[std::make_tuple(dev, stages, wide)];
   if (cur >= smem) return cudaSuccess;
-  e = stages == 4 ? cudaFuncSetAttribute(wf_fused_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)
-                  : cudaFuncSetAttribute(wf_fused_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  e = cudaFuncSetAttribute(fused_kernel(stages, wide), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e == cudaSuccess) cur = smem;
   return e;
 }
 
 // How many clusters of cs CTAs (with `smem` bytes each) can be resident at
 // once on the current device; cached per configuration.
-int max_active_clusters(int stages, int cs, size_t smem) {
+int max_active_clusters(int stages, bool wide, int cs, size_t smem) {
   static std::mutex mu;
-  static std::map<std::tuple<int, int, int, size_t>, int> cache;
+  static std::map<std::tuple<int, int, bool, int, size_t>, int> cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  const auto key = std::make_tuple(dev, stages, cs, smem);
+  const auto key = std::make_tuple(dev, stages, wide, cs, smem);
   std::lock_guard<std::mutex> lock(mu);
   auto it = cache.find(key);
   if (it != cache.end()) return it->second;
@@ -1576,10 +1653,8 @@ int max_active_clusters(int stages, int cs, size_t smem) {
   cfg.numAttrs = 1;
   int n = 0;
   cudaError_t e;
-  e = ensure_smem_limit(stages, smem);  // only ever raised, so a launch's earlier limit still holds
-  if (e == cudaSuccess)
-    e = stages == 4 ? cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<4>, &cfg)
-                    : cudaOccupancyMaxActiveClusters(&n, wf_fused_kernel<3>, &cfg);
+  e = ensure_smem_limit(stages, wide, smem);  // only ever raised, so a launch's earlier limit still holds
+  if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, fused_kernel(stages, wide), &cfg);
   if (e != cudaSuccess) {
     (void)cudaGetLastError();
     n = 0;
@@ -1623,6 +1698,11 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
     return 32 * tmax;
   };
   const size_t kMaxSmem = 227 * 1024;
+  // A one-unit plan runs both warpgroups on its unit when the candidate lists
+  // are long enough for the halved per-thread work to outweigh the wider
+  // barriers (measured: 128K tokens 123.6 -> 116.8 us; 8K tokens, lists of at
+  // most 1024, 49.5 -> 51.6 us).
+  const bool wide1 = cmax >= 2048;
   // For P units per cluster (1, or 2 so that one unit's copies overlap the
   // other's exchanges and Top-K): the largest cluster (any size up to 8)
   // whose grid fits the SMs in one wave, all clusters resident at once, and
@@ -1638,7 +1718,8 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
     ch.smem = smem_layout(ch.stages, P, cmax, kmax).total;
     if (ch.smem > kMaxSmem) return ch;
     for (int c = MAXCS; c >= 1 && ch.cs == 0; --c)
-      if (clusters * c <= num_sms && P * unit_cols(c) <= 512 && clusters <= max_active_clusters(ch.stages, c, ch.smem))
+      if (clusters * c <= num_sms && P * unit_cols(c) <= 512 &&
+          clusters <= max_active_clusters(ch.stages, P == 1 && wide1, c, ch.smem))
         ch.cs = c;
     for (int c = 1; c <= MAXCS && ch.cs == 0; ++c)
       if (P * unit_cols(c) <= 512) ch.cs = c;
@@ -1669,6 +1750,7 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
   fp.ok = true;
   fp.cs = cs;
   fp.P = P;
+  fp.wide = P == 1 && wide1;
   fp.stages = stages;
   fp.smem = smem;
   fp.tmem_cols = cols;
@@ -1749,9 +1831,9 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = range && range->pdl ? 2 : 1;
-  cudaError_t e = ensure_smem_limit(fp.stages, cfg.dynamicSmemBytes);
+  cudaError_t e = ensure_smem_limit(fp.stages, fp.wide, cfg.dynamicSmemBytes);
   if (e != cudaSuccess) return e;
-  e = fp.stages == 4 ? cudaLaunchKernelEx(&cfg, wf_fused_kernel<4>, p) : cudaLaunchKernelEx(&cfg, wf_fused_kernel<3>, p);
+  e = cudaLaunchKernelEx(&cfg, fused_kernel(fp.stages, fp.wide), p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

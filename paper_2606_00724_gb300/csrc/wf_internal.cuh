@@ -140,6 +140,7 @@ struct FusedPlan {
   int cs, P, clusters, stages, tmem_cols, ucols, ecol, cmax, kmax, U;
   size_t smem;
   bool trim;
+  bool wide;  // one unit per cluster served by both compute warpgroups
 };
 FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int n_g,
                      const wf_tensor* g, int num_sms);

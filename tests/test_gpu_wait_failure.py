@@ -3,7 +3,7 @@ the test-only control of include/wf_testing.h: the first wait of every CTA
 waits on a barrier that nothing completes, with a short bound, so it gives
 up.  The call must report WF_ERR_TIMEOUT through the workspace status word,
 write nothing outside its outputs, and leave the context usable: the next
-normal call matches the oracle.  Small shapes only."""
+normal call matches the oracle.  Small layers only (four units)."""
 import dataclasses
 
 import numpy as np
@@ -24,9 +24,9 @@ GUARD = 64          # guard rows / words on each side of an output
 SENTINEL = -12288.0  # exact in bf16
 
 
-def _small_layer():
-    w = dataclasses.replace(synth.WORKLOADS["c3"], name="wait_failure_n4096", batch=1, heads=4, n=4096, levels=3,
-                            keep=tuple(int(x) for x in oracle.default_schedule(4096, 3, 512)))
+def _small_layer(n=4096, levels=3, k=512):
+    w = dataclasses.replace(synth.WORKLOADS["c3"], name=f"wait_failure_n{n}", batch=1, heads=4, n=n, levels=levels,
+                            keep=tuple(int(x) for x in oracle.default_schedule(n, levels, k)))
     b = synth.make_batch(w, planted=True, device="cpu", cfg="c3")
     return w, dataclasses.replace(b, Q=b.Q.cuda(), K=b.K.cuda(), V=b.V.cuda(), Kg=b.Kg.cuda(), Vg=b.Vg.cuda())
 
@@ -58,8 +58,11 @@ def _oracle_unit(w, batch, u):
     return mu0, oracle.sparse_attn(Q, K, V, mu0, Kg, Vg)
 
 
-def test_fused_step_wait_gives_up_then_recovers():
-    w, batch = _small_layer()
+# 4K tokens: two units per cluster; 32K tokens (lists of 2048): one unit per
+# cluster served by both compute warpgroups.
+@pytest.mark.parametrize("n,levels,k,check", [(4096, 3, 512, 4), (32768, 4, 2048, 2)])
+def test_fused_step_wait_gives_up_then_recovers(n, levels, k, check):
+    w, batch = _small_layer(n, levels, k)
     keep = list(w.keep)
     coeffs = torch.empty(wf.wf_coeffs_bytes(batch.K, w.levels), dtype=torch.uint8, device="cuda")
     ws = torch.zeros(wf.wf_step_workspace_bytes(batch.Q, batch.K, w.levels, keep, w.ng), dtype=torch.uint8,
@@ -82,7 +85,7 @@ def test_fused_step_wait_gives_up_then_recovers():
     wf.wf_workspace_status(ws)
     torch.cuda.synchronize()
     _guards_intact(O_full, idx_full)
-    for u in range(w.units):
+    for u in range(check):
         mu0, O_ref = _oracle_unit(w, batch, u)
         assert np.array_equal(idx[u].cpu().numpy(), mu0), f"unit {u}"
         assert_close_out(f64(O[0, u]), O_ref, torch.bfloat16)
