@@ -1390,6 +1390,16 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     mdp ^= 1u;
     tc_fence_after();
   };
+  // A launch that starts below the top scale (its rows dense, so the
+  // producers do not need it): the previous selection J_{lev_top+1}, for the
+  // first Top-K's winners, from the children list it was handed (halved).
+  // The Top-K's first barrier orders it.
+  if (c.lev_top < p.L) {
+    const int32_t* src = p.jin + (int64_t)u * p.jstride;
+    int32_t* Jp = unit_J(c, p, pp, c.lev_top + 1);
+#pragma unroll 1
+    for (int i = tid; i < p.keep[c.lev_top + 1]; i += TN) Jp[i] = src[2 * i] >> 1;
+  }
   uint32_t tpar = 0;  // parity of each scale-tile barrier's next phase
 #pragma unroll 1
   for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
@@ -1539,15 +1549,6 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   // set-up above overlaps their tail when the launch is programmatic).
   grid_dep_wait();
   grid_dep_launch();
-  // A launch that starts below the top scale: the previous selection
-  // J_{lev_top+1} from the children list it was handed (halved).
-  if (c.lev_top < p.L) {
-    for (int pp = 0; pp < c.np; ++pp) {
-      const int32_t* src = p.jin + (int64_t)(c.u0 + pp) * p.jstride;
-      int32_t* J = unit_J(c, p, pp, c.lev_top + 1);
-      for (int i = tid; i < p.keep[c.lev_top + 1]; i += NT) J[i] = src[2 * i] >> 1;
-    }
-  }
   // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
   for (int pp = 0; pp < c.np; ++pp) {
     const int u = c.u0 + pp;
@@ -1801,6 +1802,9 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   for (int l = 0; l <= levels; ++l) p.keep[l] = keep[l];
   p.scale_log2 = kLog2e / sqrtf((float)D);
   if (range) {
+    // A launch below the top scale reads its first scale's rows densely: the
+    // producers never wait for the handed-in selection.
+    if (range->lev_top < levels && !range->lrows) return cudaErrorInvalidValue;
     p.lev_top = range->lev_top;
     p.lev_bot = range->lev_bot;
     p.final_sel = range->final_sel;

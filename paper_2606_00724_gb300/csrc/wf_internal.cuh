@@ -150,7 +150,7 @@ FusedPlan plan_fused(const wf_tensor& q, const wf_tensor& kv, int levels, const 
 // children list jin (when lev_top < L); the children of the last selection to
 // jout unless final_sel (then mu^0 goes to idx); the attention if attn.
 // Scale lev_top's rows come from lrows ([units][m][d], unit stride lrows_unit
-// elements) when not null, else from the pyramid.
+// elements) when not null, else from the pyramid (only when lev_top = L).
 // pdl: launch as a programmatic dependent of the previous kernel on the
 // stream (its set-up overlaps that kernel's tail).
 struct FusedRange {
