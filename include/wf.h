@@ -270,8 +270,9 @@ wf_status wf_sparse_attn(const void* Q, const wf_tensor* q, const void* K, const
  * context: until the process exits); the call allocates nothing.
  * - Limit: returns WF_ERR_WORKSPACE, and launches nothing, when the call would
  *   need more than WF_NOALLOC_SCRATCH_BYTES (the need is
- *   wf_attn_workspace_bytes(q, k, n_g); e.g. 32 heads with k + n_g <= 960
- *   rows with head_dim 128 fits).
+ *   wf_attn_workspace_bytes(q, k, n_g); e.g. 32 heads with head_dim 128 fit
+ *   k + n_g <= 1984 rows with query blocks of at most 32 rows, 960 rows with
+ *   33 to 64).
  * - Contexts: the array has its own device address in each CUDA context.  The
  *   first call from a context (the runtime's primary context of the current
  *   device, or any context the caller made current) looks that address up

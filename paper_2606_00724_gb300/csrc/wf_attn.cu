@@ -22,7 +22,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
     const T* __restrict__ Q, int64_t qsb, int64_t qsh, int64_t qss, const T* __restrict__ K,
     const T* __restrict__ V, int64_t ksb, int64_t ksh, int64_t kss, int n, const int32_t* __restrict__ idx, int k,
     const T* __restrict__ Kg, const T* __restrict__ Vg, int64_t gsb, int64_t gsh, int64_t gss, int ng, int q, int H,
-    int G, float scale, int nsplit, float* __restrict__ Opart, float2* __restrict__ ML) {
+    int G, float scale, int nsplit, int qstride, float* __restrict__ Opart, float2* __restrict__ ML) {
   constexpr int VEC = Vec<T>::N;
   constexpr int KS = D + 4;
   extern __shared__ __align__(16) float smem[];
@@ -93,7 +93,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
       acc1[r] = fmaf(qv.x, k1.x, fmaf(qv.y, k1.y, fmaf(qv.z, k1.z, fmaf(qv.w, k1.w, acc1[r]))));
     }
   }
-  float2* ml = ML + ((int64_t)u * nsplit + sp) * QMAX;  // partials keep the workspace's QMAX-row stride
+  float2* ml = ML + ((int64_t)u * nsplit + sp) * qstride;  // a split's partials: qstride rows
 #pragma unroll
   for (int r = 0; r < QM / 8; ++r) {
     const int i = warp + 8 * r;
@@ -126,7 +126,7 @@ __global__ void __launch_bounds__(256) attn_split_kernel(
 #pragma unroll
     for (int r = 0; r < QPT; ++r) o[r] = fmaf(P[(qg * QPT + r) * (CH + 1) + t], v, o[r]);
   }
-  float* op = Opart + ((int64_t)u * nsplit + sp) * QMAX * D;
+  float* op = Opart + ((int64_t)u * nsplit + sp) * qstride * D;
 #pragma unroll
   for (int r = 0; r < QPT; ++r) {
     const int i = qg * QPT + r;
@@ -189,10 +189,10 @@ cudaError_t combine(const AttnPlan& p, int nsplit, void* O, const wf_tensor& od,
   float2* ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
   const dim3 grid((unsigned)p.U, (unsigned)((p.q + 7) / 8));
   if (p.d == 128)
-    attn_combine_kernel<T, 128><<<grid, 256, 0, s>>>(Opart, ML, nsplit, p.q, p.H, QMAX, static_cast<T*>(O),
+    attn_combine_kernel<T, 128><<<grid, 256, 0, s>>>(Opart, ML, nsplit, p.q, p.H, p.qstride, static_cast<T*>(O),
                                                      od.stride_b, od.stride_h, od.stride_s);
   else
-    attn_combine_kernel<T, 64><<<grid, 256, 0, s>>>(Opart, ML, nsplit, p.q, p.H, QMAX, static_cast<T*>(O),
+    attn_combine_kernel<T, 64><<<grid, 256, 0, s>>>(Opart, ML, nsplit, p.q, p.H, p.qstride, static_cast<T*>(O),
                                                     od.stride_b, od.stride_h, od.stride_s);
   return cudaGetLastError();
 }
@@ -211,7 +211,7 @@ cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const voi
   attn_split_kernel<T, D, QM><<<dim3(p.nsplit, p.U), 256, smem, s>>>(
       static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, static_cast<const T*>(K),
       static_cast<const T*>(V), kv.stride_b, kv.stride_h, kv.stride_s, kv.seq, idx, p.k, static_cast<const T*>(Kg),
-      static_cast<const T*>(Vg), gsb, gsh, gss, p.ng, p.q, p.H, p.G, scale, p.nsplit, Opart, ML);
+      static_cast<const T*>(Vg), gsb, gsh, gss, p.ng, p.q, p.H, p.G, scale, p.nsplit, p.qstride, Opart, ML);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return combine<T>(p, p.nsplit, O, od, ws, s);
 }
@@ -229,9 +229,12 @@ AttnPlan plan_attn(const wf_tensor& q, int k, int ng, int group) {
   p.ng = ng;
   p.dtype = q.dtype;
   p.nsplit = (k + ng + CH - 1) / CH;
+  // Partials of a split take q rows rounded up to 32 (every kernel's query
+  // tile holds at most that many valid rows).
+  p.qstride = (q.seq + 31) / 32 * 32;
   size_t off = 256;  // status block
-  p.off_o = off;  off = align_up(off + (size_t)p.U * p.nsplit * QMAX * p.d * sizeof(float), 256);
-  p.off_ml = off; off = align_up(off + (size_t)p.U * p.nsplit * QMAX * sizeof(float2), 256);
+  p.off_o = off;  off = align_up(off + (size_t)p.U * p.nsplit * p.qstride * p.d * sizeof(float), 256);
+  p.off_ml = off; off = align_up(off + (size_t)p.U * p.nsplit * p.qstride * sizeof(float2), 256);
   p.total = off;
   return p;
 }

@@ -115,6 +115,7 @@ cudaError_t launch_filter_wavelet(const FilterPlan& p, const void* Q, const wf_t
 struct AttnPlan {
   int U, H, q, d, k, ng, nsplit, dtype;
   int G;
+  int qstride;  // query rows a split's partials take: q rounded up to 32
   size_t off_o, off_ml, total;
 };
 constexpr int kAttnChunk = 64;

@@ -584,7 +584,7 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   a.nsplit = (p.k + p.ng + TM - 1) / TM;
   a.Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
   a.ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
-  a.qstride = kMaxQ;
+  a.qstride = p.qstride;
   a.status = status;
   a.sl2 = 1.4426950408889634f * scale;
   const WaitControls wc = wait_controls();

@@ -253,3 +253,14 @@ def test_wait_failure_control(lib):
     assert lib.wf_testing_set_wait_failure(0, -1) == -1  # WF_ERR_INVALID_ARG
     assert lib.wf_testing_set_wait_failure(1, 1000) == 0
     assert lib.wf_testing_set_wait_failure(0, 0) == 0
+
+
+def test_attn_workspace_sized_by_query_rows(lib):
+    # A split's partials take the query rows rounded up to 32, so 32 heads at
+    # d 128 fit the allocation-free array (16 MiB) with k + n_g <= 1984 sparse
+    # rows for query blocks of up to 32 rows, and <= 960 for 33-64 rows.
+    lim = 16 << 20
+    for q, rows in ((32, 1984), (17, 1984), (64, 960), (40, 960)):
+        d = _desc(1, 32, q, 128)
+        assert lib.wf_attn_workspace_bytes(ctypes.byref(d), rows - 32, 32) <= lim, (q, rows)
+        assert lib.wf_attn_workspace_bytes(ctypes.byref(d), rows - 31, 32) > lim, (q, rows)

@@ -79,7 +79,7 @@ def test_noalloc_from_another_host_thread():
 
 
 def test_noalloc_rejects_oversized_requests():
-    # 64 heads x 4096 selected rows needs ~136 MB of split-K scratch, beyond
+    # 64 heads x 4096 selected rows needs ~68 MB of split-K scratch, beyond
     # the fixed 16 MiB: rejected with WF_ERR_WORKSPACE before any launch.
     B, H, n, d, q = 1, 64, 4096, 128, 32
     Q = torch.zeros(B, H, q, d, dtype=torch.bfloat16, device="cuda")
