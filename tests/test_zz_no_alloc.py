@@ -91,3 +91,32 @@ def test_noalloc_rejects_oversized_requests():
         wf.wf_sparse_attn_noalloc(Q, K, K, idx, n, None, None, O)
     assert ei.value.status == -5
     assert torch.count_nonzero(O) == 0
+
+
+def test_noalloc_scratch_looked_up_per_context():
+    # The static array has its own address in every CUDA context.  With a
+    # second (non-primary) driver context current, the status query must look
+    # the array up in that context (a cached primary-context address would
+    # make its 4-byte read fail there), and the primary context must keep
+    # working afterwards.  No kernel runs in the second context.
+    import ctypes
+    try:
+        cu = ctypes.CDLL("libcuda.so.1")
+        create, pop, destroy = cu.cuCtxCreate_v2, cu.cuCtxPopCurrent_v2, cu.cuCtxDestroy_v2
+    except (OSError, AttributeError):
+        pytest.skip("driver entry points unavailable")
+    torch.cuda.synchronize()
+    wf.wf_noalloc_status()  # the primary context's entry
+    dev = ctypes.c_int()
+    assert cu.cuDeviceGet(ctypes.byref(dev), torch.cuda.current_device()) == 0
+    ctx = ctypes.c_void_p()
+    assert create(ctypes.byref(ctx), 0, dev) == 0  # current on this thread from here
+    try:
+        wf.wf_noalloc_status()  # looked up in the second context
+        wf.wf_noalloc_status()  # and served from its cache entry
+    finally:
+        popped = ctypes.c_void_p()
+        assert pop(ctypes.byref(popped)) == 0 and popped.value == ctx.value
+        assert destroy(ctx) == 0
+    wf.wf_noalloc_status()  # the primary context again
+    torch.cuda.synchronize()
