@@ -71,6 +71,7 @@ constexpr int UNIT_P_BYTES = 2 * P_BYTES + MAXCS_PAD_BYTES;
 constexpr int kMaxCand = 64 * NCT;         // largest candidate list of the Top-K (64 keys a thread)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint32_t kCsyncId = 1;           // named barriers 1, 2: the compute warps of unit 0, 1
+constexpr uint32_t kSetupSyncId = 3;       // named barrier 3: the set-up threads (all but the producers)
 
 constexpr uint32_t kIdescScore = idesc_bf16(TM, NQ, 0, 0);  // A = rows (K-major), B = Q (K-major)
 constexpr uint32_t kIdescPV = idesc_bf16(D, NQ, 1, 1);      // A = V^T (MN-major), B = P^T (MN-major)
@@ -1574,55 +1575,68 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     ms.wait_limit = p.wait_limit;
     ms.abort = 0;
     fence_mbar_init();
-    // Arm the first phase of every receive barrier (bytes this CTA expects).
-    for (int pp = 0; pp < c.np; ++pp) {
-      mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
-      mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]), 4u * (uint32_t)m_total(p, c.lev_top) + c.cs * unit_warps<WIDE>() * 8u);
-      const uint32_t rows = (uint32_t)(dlo((int)c.rank + 1, c.cs) - dlo((int)c.rank, c.cs));
-      mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), c.cs * rows * NQ * 4u + c.cs * NQ * 8u);
-    }
   }
-  if (warp == MMA_WARP) {
-    tmem_alloc(smem_u32(&ms.tmem_base), p.tmem_cols);
-    tmem_relinquish();
-  }
-  // The Top-K scratch starts zeroed (histogram, list counter).
-  for (int pp = 0; pp < c.np; ++pp) {
-    uint8_t* sc = smem + c.ly.p + pp * UNIT_P_BYTES;
-    for (int e = tid; e < (int)((sizeof(SelScratch) + 15) / 16); e += NT)
-      *reinterpret_cast<uint4*>(sc + 16 * e) = make_uint4(0, 0, 0, 0);
-  }
-  // Global memory only after the grids this launch depends on are done (the
-  // set-up above overlaps their tail when the launch is programmatic).
-  grid_dep_wait();
-  grid_dep_launch();
-  // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
-  for (int pp = 0; pp < c.np; ++pp) {
-    const int u = c.u0 + pp;
-    const bf16* qb = p.Q + (int64_t)(u / p.H) * p.qsb + (int64_t)(u % p.H) * p.qsh;
-    uint8_t* sq = smem + c.ly.q + pp * Q_BYTES;
-    for (int e = tid; e < NQ * (D / 8); e += NT) {
-      const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
-      const int i = g * 8 + rr;
-      uint4 v = make_uint4(0, 0, 0, 0);
-      if (i < p.q) v = __ldg(reinterpret_cast<const uint4*>(qb + (int64_t)i * p.qss + ch * 8));
-      *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
-    }
-  }
-  fence_proxy_async();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  c.tmem = ms.tmem_base;
-  cluster_sync();  // every CTA's barriers exist before any remote arrival
-
-  if (warp < MMA_WARP) {
-    compute_role<WIDE>(c, p);
-  } else if (warp == MMA_WARP) {
-    if ((tid & 31) == 0) mma_role<S>(c, p);
-    __syncwarp();
-  } else {
+  __syncthreads();  // this CTA's barriers exist
+  if (warp > MMA_WARP) {
+    // The producers touch only this CTA's ring and barriers, so they start at
+    // once: they join the cluster barrier's first phase now (nothing of theirs
+    // needs ordering before other CTAs' remote stores) and wait for it at the
+    // end, while the other warps finish the set-up.
+    cluster_arrive_relaxed();
+    grid_dep_wait();  // the rows come from the grids before a programmatic launch
     producer_role<S>(c, p);
+    cluster_wait();
+  } else {
+    constexpr int NS = NT - NPT;  // the set-up threads: compute warps and the MMA warp
+    if (tid == 0) {
+      // Arm the first phase of every receive barrier (bytes this CTA expects).
+      for (int pp = 0; pp < c.np; ++pp) {
+        mbar_arrive_expect_tx(bar_addr(ms.xbar[pp]), c.cs * NQ * 8u);
+        mbar_arrive_expect_tx(bar_addr(ms.kbar[pp]),
+                              4u * (uint32_t)m_total(p, c.lev_top) + c.cs * unit_warps<WIDE>() * 8u);
+        const uint32_t rows = (uint32_t)(dlo((int)c.rank + 1, c.cs) - dlo((int)c.rank, c.cs));
+        mbar_arrive_expect_tx(bar_addr(ms.cbar[pp]), c.cs * rows * NQ * 4u + c.cs * NQ * 8u);
+      }
+    }
+    if (warp == MMA_WARP) {
+      tmem_alloc(smem_u32(&ms.tmem_base), p.tmem_cols);
+      tmem_relinquish();
+    }
+    // The Top-K scratch starts zeroed (histogram, list counter, masks).
+    for (int pp = 0; pp < c.np; ++pp) {
+      uint8_t* sc = smem + c.ly.p + pp * UNIT_P_BYTES;
+      for (int e = tid; e < (int)((sizeof(SelScratch) + 15) / 16); e += NS)
+        *reinterpret_cast<uint4*>(sc + 16 * e) = make_uint4(0, 0, 0, 0);
+    }
+    // Global memory only after the grids this launch depends on are done (the
+    // set-up above overlaps their tail when the launch is programmatic).
+    grid_dep_wait();
+    grid_dep_launch();
+    // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
+    for (int pp = 0; pp < c.np; ++pp) {
+      const int u = c.u0 + pp;
+      const bf16* qb = p.Q + (int64_t)(u / p.H) * p.qsb + (int64_t)(u % p.H) * p.qsh;
+      uint8_t* sq = smem + c.ly.q + pp * Q_BYTES;
+      for (int e = tid; e < NQ * (D / 8); e += NS) {
+        const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
+        const int i = g * 8 + rr;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (i < p.q) v = __ldg(reinterpret_cast<const uint4*>(qb + (int64_t)i * p.qss + ch * 8));
+        *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
+      }
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    named_sync(kSetupSyncId, NS);
+    tc_fence_after();
+    c.tmem = ms.tmem_base;
+    cluster_sync();  // every CTA's barriers are armed before any remote arrival
+    if (warp < MMA_WARP) {
+      compute_role<WIDE>(c, p);
+    } else {
+      if ((tid & 31) == 0) mma_role<S>(c, p);
+      __syncwarp();
+    }
   }
 
   tc_fence_before();

@@ -54,6 +54,10 @@ __device__ __forceinline__ void st_cluster_v4f32(uint32_t addr, float a, float b
 // Split cluster barrier (every thread of every CTA of the cluster; not
 // warp-aligned, so it may follow divergent code).
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
+// Arrival with no ordering of this thread's earlier memory operations.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
+}
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
 
 // Asynchronous stores into the shared memory of a CTA of this cluster (which
