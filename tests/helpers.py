@@ -14,7 +14,7 @@ def f64(t: torch.Tensor) -> np.ndarray:
     return t.detach().to("cpu", torch.float64).numpy()
 
 
-class GpuRun:
+class LibRun:
     """Buffers and outputs of one libwf pass over a [B, H, ...] layer."""
 
     def __init__(self, Q, K, V, Kg, Vg, L, keep, want_sets=True):

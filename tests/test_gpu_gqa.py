@@ -13,7 +13,7 @@ import pytest
 import torch
 
 import oracle
-from helpers import GpuRun, assert_close_out, f64
+from helpers import LibRun, assert_close_out, f64
 from paper_2606_00724_gb300 import synth, wf
 
 pytestmark = pytest.mark.gpu
@@ -60,11 +60,11 @@ def test_gqa_per_stage(base, kw, dtype):
     cfg = base
     batch = synth.make_batch(w, planted=True, device="cuda", cfg=cfg)
     assert batch.Q.dtype == dtype and batch.Q.shape[1] == w.heads * w.group
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
     torch.cuda.synchronize()
     _check_units(w, batch, run, range(w.units), dtype)
     # wf_step takes the per-stage path for grouped heads: same indices, same output.
-    step = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
+    step = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
     step.step()
     torch.cuda.synchronize()
     assert torch.equal(step.idx, run.idx)
@@ -78,7 +78,7 @@ def test_gqa_dream_shape_sampled_units():
     w = synth.WORKLOADS["g1"]
     units = [0, 13, w.units - 1]
     batch = synth.make_batch(w, planted=True, device="cuda", cfg="g1", units=units)
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().step(refresh=False)
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().step(refresh=False)
     torch.cuda.synchronize()
     _check_units(w, batch, run, units, torch.bfloat16)
 
@@ -90,7 +90,7 @@ def test_gqa_attention_equals_repeated_key_heads():
     w = _workload("g1", batch=2, heads=2, group=3, n=2048, levels=2, k=256)
     batch = synth.make_batch(w, planted=True, device="cuda", cfg="g1")
     G = w.group
-    grouped = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    grouped = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
     rep = lambda t: t.repeat_interleave(G, dim=1).contiguous()
     K1, V1, Kg1, Vg1 = rep(batch.K), rep(batch.V), rep(batch.Kg), rep(batch.Vg)
     idx1 = grouped.idx.repeat_interleave(G, dim=0).contiguous()

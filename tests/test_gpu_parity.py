@@ -11,7 +11,7 @@ import pytest
 import torch
 
 import oracle
-from helpers import GpuRun, assert_close_out, eps_valid, f64, make_layer, oracle_unit
+from helpers import LibRun, assert_close_out, eps_valid, f64, make_layer, oracle_unit
 from paper_2606_00724_gb300 import synth
 
 pytestmark = pytest.mark.gpu
@@ -40,7 +40,7 @@ def _check_units(w, batch, run, units):
 @pytest.mark.parametrize("cfg", ["c1", "c2"])
 def test_small_configs_all_units(cfg):
     w, batch = make_layer(cfg)
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
     torch.cuda.synchronize()
     _check_units(w, batch, run, range(w.units))
 
@@ -54,7 +54,7 @@ def test_full_size_sampled_units(cfg):
     w = synth.WORKLOADS[cfg]
     units = [0, w.units // 2 + 3, w.units - 1]
     w, batch = make_layer(cfg, units=None)
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
     torch.cuda.synchronize()
     _check_units(w, batch, run, units)
     # Every unit's planted answer (no oracle needed).
@@ -86,7 +86,7 @@ def _rand_case(seed, B, H, n, d, q, ng, dtype, bshd=False, device="cuda"):
 def test_random_shapes(dtype, n, d, q, ng, L, keep, bshd):
     B, H = 2, 3
     Q, K, V, Kg, Vg = _rand_case(n + d + q + L, B, H, n, d, q, ng, dtype, bshd)
-    run = GpuRun(Q, K, V, Kg, Vg, L, keep).run()
+    run = LibRun(Q, K, V, Kg, Vg, L, keep).run()
     torch.cuda.synchronize()
     for u in range(B * H):
         b, h = divmod(u, H)
@@ -111,7 +111,7 @@ def test_attention_full_selection_is_dense(dtype):
     # k = n: the sparse attention equals dense cached attention over [K; Kg].
     B, H, n, d, q, ng = 1, 2, 192, 128, 16, 8
     Q, K, V, Kg, Vg = _rand_case(7, B, H, n, d, q, ng, dtype)
-    run = GpuRun(Q, K, V, Kg, Vg, 1, [n, n // 2])
+    run = LibRun(Q, K, V, Kg, Vg, 1, [n, n // 2])
     idx = torch.arange(n, dtype=torch.int32, device="cuda").repeat(B * H, 1)
     run.attn(idx)
     torch.cuda.synchronize()
@@ -124,7 +124,7 @@ def test_attention_full_selection_is_dense(dtype):
 def test_attention_unsorted_indices_and_scale():
     B, H, n, d, q, ng = 1, 1, 300, 64, 4, 0
     Q, K, V, _, _ = _rand_case(8, B, H, n, d, q, ng, torch.float32)
-    run = GpuRun(Q, K, V, None, None, 1, [10, 5])
+    run = LibRun(Q, K, V, None, None, 1, [10, 5])
     sel = torch.tensor([[299, 3, 150, 7, 8, 42, 0]], dtype=torch.int32, device="cuda")
     run.attn(sel, scale=0.3)
     torch.cuda.synchronize()
@@ -136,7 +136,7 @@ def test_attention_unsorted_indices_and_scale():
 def test_step_matches_separate_calls():
     from paper_2606_00724_gb300 import wf
     w, batch = make_layer("c2")
-    a = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    a = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
     idx = torch.empty_like(a.idx)
     O = torch.empty_like(a.O)
     coeffs = torch.empty_like(a.coeffs)

@@ -10,7 +10,7 @@ import pytest
 import torch
 
 import oracle
-from helpers import GpuRun, assert_close_out, eps_valid, f64, make_layer, oracle_unit
+from helpers import LibRun, assert_close_out, eps_valid, f64, make_layer, oracle_unit
 from paper_2606_00724_gb300 import synth, wf
 
 pytestmark = pytest.mark.gpu
@@ -35,7 +35,7 @@ def _check(w, batch, run, units):
 @pytest.mark.parametrize("cfg", ["c2", "c3", "c4", "c5"])
 def test_step_full_size(cfg):
     w, batch = make_layer(cfg)
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).step()
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).step()
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
     units = [0, 1, w.units // 2 + 3, w.units - 1]
@@ -59,7 +59,7 @@ def test_step_unplanted_timing_inputs(cfg):
     # answers) and its output must match the oracle's attention over the
     # kernel's own indices.
     w, batch = make_layer(cfg, planted=False)
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).step()
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).step()
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
     for u in [0, 5, w.units // 2 + 1, w.units - 1]:
@@ -78,8 +78,8 @@ def test_step_matches_per_stage_kernels():
     # Planted 8K layer: the fused kernel and the per-stage kernels select the
     # same indices and agree on the output.
     w, batch = make_layer("c2")
-    a = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
-    b = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
+    a = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
+    b = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
     b.coeffs.copy_(a.coeffs)
     b.step(refresh=False)
     torch.cuda.synchronize()
@@ -109,7 +109,7 @@ def _rand(seed, B, H, n, q, ng, bshd=False):
 ])
 def test_step_random_shapes(B, H, n, q, ng, L, keep, bshd):
     Q, K, V, Kg, Vg = _rand(n + q + L, B, H, n, q, ng, bshd)
-    run = GpuRun(Q, K, V, Kg, Vg, L, keep).step()
+    run = LibRun(Q, K, V, Kg, Vg, L, keep).step()
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
     for u in range(B * H):
@@ -141,7 +141,7 @@ def test_step_level0_schedule(cfg):
     assert keep[0] < 2 * keep[1]
     w = dataclasses.replace(w0, keep=keep, name=w0.name + "_level0")
     batch = synth.make_batch(w, planted=True, device="cuda", cfg=cfg)
-    run = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, list(w.keep)).step()
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, list(w.keep)).step()
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
     _check(w, batch, run, [0, w.units // 2 + 1, w.units - 1])
@@ -168,7 +168,7 @@ def test_step_exact_ties(n, period, L, keep):
         return torch.randn(B, H, rows, d, generator=g).to(torch.bfloat16)
     Q, V, Kg, Vg = r(q).cuda(), r(n).cuda(), r(ng).cuda(), r(ng).cuda()
     K = r(period).repeat(1, 1, n // period, 1).contiguous().cuda()
-    run = GpuRun(Q, K, V, Kg, Vg, L, keep).step()
+    run = LibRun(Q, K, V, Kg, Vg, L, keep).step()
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
     for u in range(B * H):

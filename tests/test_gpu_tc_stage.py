@@ -12,7 +12,7 @@ import pytest
 import torch
 
 import oracle
-from helpers import GpuRun, assert_close_out, f64
+from helpers import LibRun, assert_close_out, f64
 from paper_2606_00724_gb300 import synth, wf
 
 pytestmark = pytest.mark.gpu
@@ -33,7 +33,7 @@ def test_tc_filter_and_attention(q, group, k, ng):
     batch = synth.make_batch(w, planted=True, device="cuda", cfg="g1")
     Kg = batch.Kg if ng else None
     Vg = batch.Vg if ng else None
-    run = GpuRun(batch.Q, batch.K, batch.V, Kg, Vg, w.levels, w.keep).run()
+    run = LibRun(batch.Q, batch.K, batch.V, Kg, Vg, w.levels, w.keep).run()
     wf.wf_workspace_status(run.ws)
     torch.cuda.synchronize()
     G = w.group

@@ -11,7 +11,7 @@ import pytest
 import torch
 
 import oracle
-from helpers import GpuRun, assert_close_out, f64
+from helpers import LibRun, assert_close_out, f64
 from paper_2606_00724_gb300 import synth, wf
 
 pytestmark = pytest.mark.gpu
@@ -109,7 +109,7 @@ def test_filter_wavelet_haar_equals_filter(cfg):
     w = synth.WORKLOADS[cfg]
     batch = synth.make_batch(w, planted=True, device="cuda", cfg=cfg, units=[0, 5, w.units - 1])
     idx, sets = _filter_wavelet(batch, w, wf.WF_WAVELET_HAAR)
-    ref = GpuRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().filter()
+    ref = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().filter()
     torch.cuda.synchronize()
     assert torch.equal(idx, ref.idx)
     assert torch.equal(sets, ref.sets)
