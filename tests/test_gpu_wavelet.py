@@ -6,6 +6,8 @@ the oracle's literal filter on planted inputs (every scale, bit-exact), and
 wf_step_wavelet's indices and output against the oracle.  For bf16 keys with
 head_dim 128 and one query head per key head both calls run the fused
 kernel once per scale."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -168,3 +170,36 @@ def test_step_wavelet_db2_matches_oracle(cfg, units):
         ref = oracle.sparse_attn(f64(Q[b, h]), f64(K[b, h]), f64(V[b, h]), idx_h[u], f64(batch.Kg[b, h]),
                                  f64(batch.Vg[b, h]))
         assert_close_out(f64(O[b, h]), ref, torch.bfloat16)
+
+
+@pytest.mark.parametrize("basis", ["db2", "haar"])
+def test_step_wavelet_odd_units_no_generation_rows(basis):
+    # Three units (a two-unit cluster plan leaves its last cluster one unit)
+    # and no generation rows: every unit against the oracle's literal filter
+    # (indices at every scale) and attention over the selected rows only.
+    wv, ov = BASES[basis]
+    w = dataclasses.replace(synth.WORKLOADS["c3"], name="odd_units", batch=1, heads=3, n=4096, levels=3, ng=0,
+                            keep=tuple(int(x) for x in oracle.default_schedule(4096, 3, 512)))
+    batch = synth.make_batch(w, planted=True, device="cuda", cfg="c3")
+    Q, K, V = batch.Q, batch.K, batch.V
+    B, H = K.shape[:2]
+    top = torch.empty(B, H, w.n >> w.levels, w.head_dim, dtype=K.dtype, device="cuda")
+    wf.wf_wavelet_approx(K, w.levels, wv, top)
+    ws = torch.zeros(wf.wf_step_wavelet_workspace_bytes(Q, K, w.levels, w.keep, wv, 0), dtype=torch.uint8,
+                     device="cuda")
+    idx = torch.empty(B * H, w.k, dtype=torch.int32, device="cuda")
+    sets = torch.empty(B * H, sum(w.keep), dtype=torch.int32, device="cuda")
+    O = torch.empty_like(Q)
+    wf.wf_step_wavelet(Q, top, K, V, None, None, w.levels, w.keep, wv, idx, O, ws, level_sets=sets)
+    wf.wf_workspace_status(ws)
+    torch.cuda.synchronize()
+    for u in range(w.units):
+        b, h = divmod(u, w.heads)
+        Qu, Ku, Vu = f64(Q[b, h]), f64(K[b, h]), f64(V[b, h])
+        mu0, osets = oracle.filter_wavelet(Qu, Ku, w.levels, np.array(w.keep), ov, spec32=True, store_bf16=True,
+                                           want_sets=True)
+        gsets = oracle.split_level_sets(sets[u].cpu().numpy(), w.levels, w.keep)
+        for lev in range(w.levels, -1, -1):
+            assert np.array_equal(gsets[lev], osets[lev]), f"unit {u} scale {lev}"
+        assert np.array_equal(idx[u].cpu().numpy(), mu0), f"unit {u}"
+        assert_close_out(f64(O[b, h]), oracle.sparse_attn(Qu, Ku, Vu, mu0), torch.bfloat16)
