@@ -107,8 +107,9 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* tile = smem;                        // 2 x HALF, 1024-aligned
   uint8_t* sq = smem + 2 * HALF;               // nq / 8 groups of QGRP
-  float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [NWG][4][32]
-  float* col = red + NWG * 4 * 32;             // [256]: per-warpgroup column maxima ([NWG][32]), or the c_i
+  // [NWG][4 lane quarters][4 chunks][32] (max, sum) of each warp's rows per column (MODE 0)
+  float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);
+  float* col = red + NWG * 4 * 4 * 32 * 2;     // [256]: the c_i (MODE 1)
   float2* xch = reinterpret_cast<float2*>(col + 256);  // [128]: the second warpgroup's (max, sum) per row
   unsigned long long* bar = reinterpret_cast<unsigned long long*>(xch + 128);
   uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 1);
@@ -190,53 +191,89 @@ __global__ void __launch_bounds__(NTH) tc_score_kernel(const __grid_constant__ T
   const bool valid = j < a.m;
   const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
   const int nch = a.nq / 32;
-  float* rw = red + wg * 4 * 32;
-  float* cw = col + wg * 32;
   if (ok && MODE == 0) {
+    // Each warp takes its own column maxima (the warp-wide max instruction)
+    // and sums its rows against them, with no barrier per chunk; the four
+    // lane quarters' (max, sum) of a column then merge into the tile's.
     float2* pt = a.part + (int64_t)u * a.part_unit + (int64_t)t * a.q;
+    float2* sl = reinterpret_cast<float2*>(red);
+    int k = 0;
 #pragma unroll 1
-    for (int ch = wg; ch < nch; ch += NWG) {
+    for (int ch = wg; ch < nch; ch += NWG, ++k) {
       float v[32], w[32];
       tmem_ld32(lane_base + 32 * ch, v);
+      float mcol = -INFINITY;  // lane i: this warp's max of column i (x sl2)
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        v[i] = valid ? v[i] * a.sl2 : -INFINITY;
-        w[i] = v[i];
+        const float mi = warp_max_f32(valid ? v[i] : -INFINITY) * a.sl2;
+        mcol = lane == i ? mi : mcol;
+        w[i] = valid ? ex2(fmaf(v[i], a.sl2, -mi)) : 0.f;
       }
-      rw[quarter * 32 + lane] = xpose_reduce32<true>(w, lane);
-      wg_sync(wg);
-      if (wt < 32) cw[wt] = fmaxf(fmaxf(rw[wt], rw[32 + wt]), fmaxf(rw[64 + wt], rw[96 + wt]));
-      wg_sync(wg);
+      const float sum = xpose_reduce32<false>(w, lane);
+      sl[((wg * 4 + quarter) * 4 + k) * 32 + lane] = make_float2(mcol, sum);
+    }
+    wg_sync(wg);
+    k = 0;
+#pragma unroll 1
+    for (int ch = wg; ch < nch; ch += NWG, ++k) {
+      if (wt < 32 && ch * 32 + wt < a.q) {
+        float2 r[4];
 #pragma unroll
-      for (int i = 0; i < 32; ++i) w[i] = valid ? ex2(v[i] - cw[i]) : 0.f;
-      rw[quarter * 32 + lane] = xpose_reduce32<false>(w, lane);
-      wg_sync(wg);
-      if (wt < 32 && ch * 32 + wt < a.q)
-        pt[ch * 32 + wt] = make_float2(cw[wt], (rw[wt] + rw[32 + wt]) + (rw[64 + wt] + rw[96 + wt]));
-      wg_sync(wg);
+        for (int q4 = 0; q4 < 4; ++q4) r[q4] = sl[((wg * 4 + q4) * 4 + k) * 32 + wt];
+        float M = -INFINITY;
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4)
+          if (r[q4].y > 0.f) M = fmaxf(M, r[q4].x);
+        float S = 0.f;
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4)
+          if (r[q4].y > 0.f) S = fmaf(r[q4].y, ex2(r[q4].x - M), S);
+        pt[ch * 32 + wt] = make_float2(M, S);
+      }
     }
   }
   if (ok && MODE == 1) {
     // The normalisers (columns past q never count).
     for (int i = tid; i < a.nq; i += NTH) col[i] = i < a.q ? a.cvec[(int64_t)u * a.q + i] : INFINITY;
     __syncthreads();
-    float mx = -INFINITY;
+    // Every exponent l sl2 - c_i is at most 0 (c_i is the log of a sum that
+    // contains this candidate's own term), so the sum is taken unshifted; the
+    // padded columns have c_i = +inf and add 0.  A warp with a valid row whose
+    // sum is tiny (below 2^-96, where flushed terms could matter) takes that
+    // row again shifted by its largest exponent (TMEM loads are warp-wide, so
+    // the whole warp runs the pass).
+    float mx = 0.f, z = 0.f;
 #pragma unroll 1
     for (int ch = wg; ch < nch; ch += NWG) {
       float v[32];
       tmem_ld32(lane_base + 32 * ch, v);
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (ch * 32 + i < a.q) mx = fmaxf(mx, fmaf(v[i], a.sl2, -col[ch * 32 + i]));
+      for (int i = 0; i < 32; ++i) z += ex2(fmaf(v[i], a.sl2, -col[ch * 32 + i]));
     }
-    float z = 0.f;
+    const bool tiny = valid && z < 0x1p-96f;
+    if (__any_sync(0xffffffffu, tiny)) {
+      float m2 = -INFINITY;
 #pragma unroll 1
-    for (int ch = wg; ch < nch; ch += NWG) {
-      float v[32];
-      tmem_ld32(lane_base + 32 * ch, v);
+      for (int ch = wg; ch < nch; ch += NWG) {
+        float v[32];
+        tmem_ld32(lane_base + 32 * ch, v);
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (ch * 32 + i < a.q) z += ex2(fmaf(v[i], a.sl2, -col[ch * 32 + i]) - mx);
+        for (int i = 0; i < 32; ++i)
+          if (ch * 32 + i < a.q) m2 = fmaxf(m2, fmaf(v[i], a.sl2, -col[ch * 32 + i]));
+      }
+      float z2 = 0.f;
+#pragma unroll 1
+      for (int ch = wg; ch < nch; ch += NWG) {
+        float v[32];
+        tmem_ld32(lane_base + 32 * ch, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (ch * 32 + i < a.q) z2 += ex2(fmaf(v[i], a.sl2, -col[ch * 32 + i]) - m2);
+      }
+      if (tiny) {
+        mx = m2;
+        z = z2;
+      }
     }
     // Fold the second warpgroup's (max, sum) of the row into the first's.
     if (wg == 1) xch[wt] = make_float2(mx, z);
@@ -285,8 +322,8 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
   // Shared memory: the tile, the query block, the reductions, the barrier.
   // At most 512 / cols CTAs may share an SM (TMEM); the request is padded so
   // that shared memory enforces it.
-  size_t smem =
-      2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 256) + sizeof(float2) * 128 + 16;
+  size_t smem = 2 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 4 * 32 * 2 + 256) +
+                sizeof(float2) * 128 + 16;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;  // CTAs per SM the TMEM allows
   const size_t floor_smem = per_sm / (cap + 1) + 1;
