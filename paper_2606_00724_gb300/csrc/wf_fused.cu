@@ -28,6 +28,12 @@
 // (m, l, O^T) is reduce-scattered over head-dimension slices: CTA r combines
 // rows d of O for its slice and writes them.
 //
+// A launch may also run part of the chain (a range of scales, the previous
+// selection handed in, the last one handed out, the attention optional): the
+// literal-basis path runs one launch per scale, each a programmatic dependent
+// of the kernel before it (every thread waits for that grid before its first
+// global access).
+//
 // Every wait is bounded (~1 s): on timeout the CTA records a status word,
 // stops issuing MMAs and skips the remaining waits, so every thread reaches
 // the final cluster barrier.
