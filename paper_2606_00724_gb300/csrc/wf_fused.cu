@@ -94,6 +94,7 @@ struct UnitState {
   float cw[NCW][NQ];        // softmax normaliser c_i, one copy per compute warp
   float fw[NCW][NQ];        // 2^(stabiliser - c_i) of each warp (keys from stored exponentials)
   float mloc[NQ], lacc[NQ];
+  float alpha[NQ];          // attention: factor 2^(m_old - m_new) of a raised stabiliser
   float red[NCW][32];
 };
 
@@ -103,6 +104,7 @@ struct Misc {
   unsigned long long tdone[MAXP][MAXT];  // scale tile t of a unit scored (one phase per scale)
   unsigned long long pfull[MAXP][2], pempty[MAXP][2], cbar[MAXP], cready[MAXP];
   UnitState us[MAXP];
+  unsigned long long qfull;     // the query blocks have landed (the producers' first copies)
   unsigned long long stallbar;  // completed by nothing (the test-only stalled first wait)
   unsigned long long drainbar;  // the MMA thread's final commit
   long long wait_limit;         // bound of the waits that can give up (cycles)
@@ -348,6 +350,34 @@ __device__ __forceinline__ RowSrc attn_src(const Ctx& c, const FusedParams& p, i
   return s;
 }
 
+// Top-K scratch.  It lives in the unit's P buffers, which nothing uses before
+// the attention.  The histogram and the list counter are zero between calls
+// (zeroed at kernel start, cleared again at the end of every call).
+constexpr int NB = 2048;     // histogram buckets
+constexpr int MAXUW = 2 * NCW;  // most compute warps of a unit
+struct SelScratch {
+  uint32_t hist[NB];
+  float2 blist[32 * MAXUW];  // boundary-bucket keys (key, position)
+  float2 sred[2][MAXUW];     // (min, max) per warp, alternating rounds
+  int wsum[4][MAXUW];        // per-warp sums of the scans (slot per scan, 32 bytes)
+  uint32_t taken[2 * 32 * MAXUW];  // boundary keys taken, as each owner's position mask (zero between uses)
+  uint32_t bcnt;
+};
+static_assert((sizeof(SelScratch) + 15) / 16 * 16 <= UNIT_P_BYTES, "Top-K scratch must fit the P buffers");
+static_assert((NB / NCT) % 8 == 0, "buckets are cleared four at a time by up to twice NCT threads");
+static_assert(offsetof(SelScratch, wsum) % 16 == 0, "the scan's warp sums are read 16 bytes at a time");
+
+#define SC_ADDR(sc_a, field) ((sc_a) + (uint32_t)offsetof(SelScratch, field))
+
+// Positions a Top-K thread owns for a list of m: the smallest power of two
+// (at least 4) with R times the unit's compute threads >= m.
+template <bool WIDE>
+__host__ __device__ constexpr int topk_run(int m) {
+  int R = 4;
+  while (R * 32 * unit_warps<WIDE>() < m) R <<= 1;
+  return R;
+}
+
 // ---------------------------------------------------------------------------
 // Producer warps.
 // ---------------------------------------------------------------------------
@@ -395,11 +425,13 @@ __device__ __forceinline__ void load_share(uint32_t st, int t, const RowSrc& src
   }
 }
 
+// Tiles t0 .. t0 + ntl - 1 of the source into ring slots it0, it0 + 1, ...
 template <int S>
-__device__ __noinline__ void produce(Misc& ms, int* status, uint32_t ring, int it0, int ntl, const RowSrc src, int pt) {
+__device__ __noinline__ void produce(Misc& ms, int* status, uint32_t ring, int it0, int t0, int ntl, const RowSrc src,
+                                     int pt) {
 #pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
-    const int it = it0 + t, s = it % S, n = it / S;
+  for (int t = t0; t < t0 + ntl; ++t) {
+    const int it = it0 + t - t0, s = it % S, n = it / S;
     if (n > 0) wait_or_abort(bar_addr(ms.empty[s]), (uint32_t)(n - 1) & 1u, ms, status);
     if (!aborted(ms)) {
       const uint32_t st = ring + s * TILE_BYTES;
@@ -418,6 +450,22 @@ template <int S>
 __device__ void producer_role(const Ctx& c, const FusedParams& p) {
   Misc& ms = *c.ms;
   const int pt = threadIdx.x - P0;
+  // The query blocks go first, ahead of every row copy: they are the MMA
+  // thread's first operands, and requests queued behind the whole grid's
+  // first burst of rows would reach it only after that burst.  K-major core
+  // matrices; rows >= q are zero-filled (no bytes read).
+  for (int pp = 0; pp < c.np; ++pp) {
+    const int u = c.u0 + pp;
+    const bf16* qb = p.Q + (int64_t)(u / p.H) * p.qsb + (int64_t)(u % p.H) * p.qsh;
+    const uint32_t sq = smem_u32(c.smem + c.ly.q + pp * Q_BYTES);
+    for (int e = pt; e < NQ * (D / 8); e += NPT) {
+      const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
+      const int i = g * 8 + rr;
+      cp_async16_zfill(sq + (uint32_t)(g * QGRP + ch * 128 + rr * 16), qb + (int64_t)min(i, p.q - 1) * p.qss + ch * 8,
+                       i < p.q);
+    }
+  }
+  cp_async_arrive_noinc(bar_addr(ms.qfull));
   int it = 0;
   for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
     for (int pp = 0; pp < c.np; ++pp) {
@@ -426,7 +474,7 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
       int g0, mc;
       scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
       const int ntl = tiles_of(mc);
-      produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, scale_src(c, p, pp, lev, g0, mc), pt);
+      produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, scale_src(c, p, pp, lev, g0, mc), pt);
       it += ntl;
     }
   }
@@ -436,9 +484,13 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
     int a0, mc;
     attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
     const int ntl = tiles_of(mc);
-    produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, attn_src(c, p, pp, false, a0, mc), pt);
+    // The key tiles, then the value tiles.  A key tile's slot frees as soon
+    // as its S product is done and a value tile's once its PV product is,
+    // whose P the compute warps form from each S tile as it lands, so the
+    // value stream follows the key stream without waiting for all of S.
+    produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, attn_src(c, p, pp, false, a0, mc), pt);
     it += ntl;
-    produce<S>(ms, p.status, smem_u32(c.smem), it, ntl, attn_src(c, p, pp, true, a0, mc), pt);
+    produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, attn_src(c, p, pp, true, a0, mc), pt);
     it += ntl;
   }
   // Copies still in flight (only after a wait gave up) land before the CTA
@@ -450,69 +502,67 @@ __device__ void producer_role(const Ctx& c, const FusedParams& p) {
 // MMA thread.
 // ---------------------------------------------------------------------------
 
-// S^T tile t = rows . Q^T into TMEM columns tb + 32 t, for ntl landed tiles.
-// With tdone != 0 (a scale), tile t's completion is also signalled on the
-// barrier at tdone + 8 t, so the compute warps start on it at once.
+// S^T = rows . Q^T of the landed tile in ring slot `it` into TMEM columns
+// [dcol, dcol + 32); its completion frees the slot and completes `tbar`, so the
+// compute warps start on the tile at once.
 template <int S>
-__device__ __forceinline__ void mma_scores(const Ctx& c, const FusedParams& p, int it0, int ntl, uint32_t tb,
-                                           uint32_t sq, uint32_t tdone) {
+__device__ __forceinline__ void mma_score_tile(const Ctx& c, const FusedParams& p, int it, uint32_t dcol, uint32_t sq,
+                                               uint32_t tbar) {
   Misc& ms = *c.ms;
-#pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
-    const int it = it0 + t, s = it % S, n = it / S;
-    wait_or_abort(bar_addr(ms.full[s]), (uint32_t)n & 1u, ms, p.status);
-    fence_proxy_async();
-    if (!aborted(ms)) {
-      tc_fence_after();
-      const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
+  const int s = it % S, n = it / S;
+  wait_or_abort(bar_addr(ms.full[s]), (uint32_t)n & 1u, ms, p.status);
+  fence_proxy_async();
+  if (!aborted(ms)) {
+    tc_fence_after();
+    const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
+    for (int h = 0; h < 2; ++h)
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          mma_bf16(tb + 32 * t, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
-                   smem_desc(sq + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
-    }
-    mma_commit(bar_addr(ms.empty[s]));
-    if (tdone) mma_commit(tdone + 8u * (uint32_t)t);
+      for (int kk = 0; kk < 4; ++kk)
+        mma_bf16(dcol, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
+                 smem_desc(sq + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
   }
+  mma_commit(bar_addr(ms.empty[s]));
+  mma_commit(tbar);
 }
 
-// O^T += V_s^T P^T over ntl landed V tiles, P tile t from unit pp's compute warps.
+// O^T += V_t^T P_t^T for the value tile in ring slot `it` and unit pp's P tile
+// t (the P double buffer t % 2, filled by the compute warps).
 template <int S>
-__device__ __forceinline__ void mma_pv(const Ctx& c, const FusedParams& p, int pp, int it0, int ntl, uint32_t ocol) {
+__device__ __forceinline__ void mma_pv_tile(const Ctx& c, const FusedParams& p, int pp, int it, int t, uint32_t ocol) {
   Misc& ms = *c.ms;
   const uint32_t pa = smem_u32(c.smem + c.ly.p + pp * UNIT_P_BYTES);
-#pragma unroll 1
-  for (int t = 0; t < ntl; ++t) {
-    const int it = it0 + t, s = it % S, n = it / S;
-    const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
-    wait_or_abort(bar_addr(ms.full[s]), (uint32_t)n & 1u, ms, p.status);
-    wait_or_abort(bar_addr(ms.pfull[pp][pb]), pn & 1u, ms, p.status);
-    fence_proxy_async();
-    if (!aborted(ms)) {
-      tc_fence_after();
-      const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
+  const int s = it % S, n = it / S;
+  const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
+  wait_or_abort(bar_addr(ms.full[s]), (uint32_t)n & 1u, ms, p.status);
+  wait_or_abort(bar_addr(ms.pfull[pp][pb]), pn & 1u, ms, p.status);
+  fence_proxy_async();
+  if (!aborted(ms)) {
+    tc_fence_after();
+    const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
 #pragma unroll
-      for (int kq = 0; kq < TM / 16; ++kq)
-        mma_bf16(ocol, smem_desc_sw128(st + kq * 2048, HALF_BYTES, 1024),
-                 smem_desc(pa + pb * P_BYTES + kq * 1024, 512, 128), kIdescPV, (t > 0 || kq > 0) ? 1u : 0u);
-    }
-    mma_commit(bar_addr(ms.empty[s]));
-    mma_commit(bar_addr(ms.pempty[pp][pb]));
+    for (int kq = 0; kq < TM / 16; ++kq)
+      mma_bf16(ocol, smem_desc_sw128(st + kq * 2048, HALF_BYTES, 1024),
+               smem_desc(pa + pb * P_BYTES + kq * 1024, 512, 128), kIdescPV, (t > 0 || kq > 0) ? 1u : 0u);
   }
+  mma_commit(bar_addr(ms.empty[s]));
+  mma_commit(bar_addr(ms.pempty[pp][pb]));
 }
 
 template <int S>
 __device__ void mma_role_body(const Ctx& c, const FusedParams& p) {
   Misc& ms = *c.ms;
+  wait_or_abort(bar_addr(ms.qfull), 0u, ms, p.status);
+  fence_proxy_async();
   int it = 0;
   for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
     for (int pp = 0; pp < c.np; ++pp) {
       int g0, mc;
       scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
       const int ntl = tiles_of(mc);
-      mma_scores<S>(c, p, it, ntl, c.tmem + pp * p.ucols, smem_u32(c.smem + c.ly.q + pp * Q_BYTES),
-                    bar_addr(ms.tdone[pp][0]));
+      const uint32_t tb = c.tmem + pp * p.ucols, sq = smem_u32(c.smem + c.ly.q + pp * Q_BYTES);
+#pragma unroll 1
+      for (int t = 0; t < ntl; ++t) mma_score_tile<S>(c, p, it + t, tb + 32 * t, sq, bar_addr(ms.tdone[pp][t]));
       it += ntl;
     }
   }
@@ -520,14 +570,17 @@ __device__ void mma_role_body(const Ctx& c, const FusedParams& p) {
     int a0, mc;
     attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
     const int ntl = tiles_of(mc);
-    const uint32_t tb = c.tmem + pp * p.ucols;
+    const uint32_t tb = c.tmem + pp * p.ucols, sq = smem_u32(c.smem + c.ly.q + pp * Q_BYTES);
     if (ntl == 0) continue;
-    mma_scores<S>(c, p, it, ntl, tb, smem_u32(c.smem + c.ly.q + pp * Q_BYTES), 0u);
+    // S_t as each key tile lands (its completion on the tile's barrier), then
+    // the PV products as the value tiles land and their P tiles are formed.
+#pragma unroll 1
+    for (int t = 0; t < ntl; ++t) mma_score_tile<S>(c, p, it + t, tb + 32 * t, sq, bar_addr(ms.tdone[pp][t]));
     it += ntl;
-    mma_commit(bar_addr(ms.mdone[pp]));
-    mma_pv<S>(c, p, pp, it, ntl, tb + p.ucols - 32);
+#pragma unroll 1
+    for (int t = 0; t < ntl; ++t) mma_pv_tile<S>(c, p, pp, it + t, t, tb + p.ucols - 32);
     it += ntl;
-    mma_commit(bar_addr(ms.mdone[pp]));
+    mma_commit(bar_addr(ms.mdone[pp]));  // every PV product of the unit is done
   }
 }
 
@@ -565,24 +618,6 @@ __device__ __forceinline__ float transpose_reduce32(float (&v)[32], int lane) {
   return v[0];
 }
 
-// Top-K scratch.  It lives in the unit's P buffers, which nothing uses before
-// the attention.  The histogram and the list counter are zero between calls
-// (zeroed at kernel start, cleared again at the end of every call).
-constexpr int NB = 2048;     // histogram buckets
-constexpr int MAXUW = 2 * NCW;  // most compute warps of a unit
-struct SelScratch {
-  uint32_t hist[NB];
-  float2 blist[32 * MAXUW];  // boundary-bucket keys (key, position)
-  float2 sred[2][MAXUW];     // (min, max) per warp, alternating rounds
-  int wsum[4][MAXUW];        // per-warp sums of the scans (slot per scan, 32 bytes)
-  uint32_t taken[2 * 32 * MAXUW];  // boundary keys taken, as each owner's position mask (zero between uses)
-  uint32_t bcnt;
-};
-static_assert((sizeof(SelScratch) + 15) / 16 * 16 <= UNIT_P_BYTES, "Top-K scratch must fit the P buffers");
-static_assert((NB / NCT) % 8 == 0, "buckets are cleared four at a time by up to twice NCT threads");
-static_assert(offsetof(SelScratch, wsum) % 16 == 0, "the scan's warp sums are read 16 bytes at a time");
-
-#define SC_ADDR(sc_a, field) ((sc_a) + (uint32_t)offsetof(SelScratch, field))
 
 // Exclusive prefix sum over the unit's compute threads (thread order), with
 // its per-warp sums in the words at wsum_a.  One barrier: the caller does not
@@ -924,50 +959,9 @@ __device__ __noinline__ void select_keys(uint32_t keys_a, int m, int kk, uint32_
 template <bool WIDE>
 __device__ __forceinline__ void select_topk(uint32_t keys_a, int m, int kk, uint32_t jprev_a, int top, uint32_t sc_a,
                                             float lo, float hi) {
-  int R = 4;
-  while (R * 32 * unit_warps<WIDE>() < m) R <<= 1;
+  const int R = topk_run<WIDE>(m);
   if (WIDE || R <= 32) select_keys<uint32_t, WIDE>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
   else select_keys<unsigned long long, WIDE>(keys_a, m, kk, jprev_a, top, sc_a, lo, hi, R);
-}
-
-// Per-query max (x sl2, log2 units) of the valid rows of TMEM tiles
-// 0..ntl-1 of region tb (this warpgroup's share of them) -> mloc of unit pp.
-// The column maxima across a warp come from the warp-wide max instruction.
-template <bool WIDE>
-__device__ __noinline__ void pass_max(Misc& ms, int pp, uint32_t tb, int ntl, int mc, float sl2) {
-  const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
-  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-  UnitState& us = ms.us[pp];
-  float mx[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) mx[i] = -INFINITY;
-#pragma unroll 1
-  for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
-    uint32_t ra[32];
-    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
-    tmem_wait_ld();
-    if (t * TM + row < mc) {
-#pragma unroll
-      for (int i = 0; i < 32; ++i) mx[i] = fmaxf(mx[i], __uint_as_float(ra[i]));
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < 32; ++i) mx[i] = warp_max_f32(mx[i]);
-  if (lane == 0) {
-#pragma unroll
-    for (int i = 0; i < 32; i += 4)
-      sts_v4(smem_u32(&wslots<WIDE>(ms, pp, warp).red[warp & 3][i]),
-             make_uint4(__float_as_uint(mx[i]), __float_as_uint(mx[i + 1]), __float_as_uint(mx[i + 2]),
-                        __float_as_uint(mx[i + 3])));
-  }
-  csync<WIDE>();
-  if (tid < 32) {
-    float m = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < unit_warps<WIDE>(); ++w) m = fmaxf(m, wslots<WIDE>(ms, pp, w).red[w & 3][tid]);
-    us.mloc[tid] = m * sl2;
-  }
-  csync<WIDE>();
 }
 
 // The warp's (stabiliser, sum of 2^(l sl2 - stabiliser)) per query over its
@@ -1252,57 +1246,149 @@ __device__ __noinline__ void pass_keys(uint32_t rank, uint32_t cs, Misc& ms, int
   tc_fence_before();
 }
 
-// Attention: P = 2^(s - m) (bf16, P^T MN-major core matrices) of every S tile
-// into the unit's P double buffer for the MMA thread, and the row sums of P
-// -> us.lacc.
-// WIDE: each warpgroup forms the P tiles of its tiles (t = wg, wg + 2, ...),
-// so each always fills the same one of the two buffers.
+// OR of a predicate over the unit's compute threads (a barrier of theirs).
 template <bool WIDE>
-__device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* pbase, int pp, uint32_t tb, int ntl,
-                                    int mc) {
+__device__ __forceinline__ bool csync_or(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\tsetp.ne.u32 pi, %1, 0;\n\tbar.red.or.pred po, %2, %3, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v), "r"(kCsyncId + (WIDE ? 0u : (threadIdx.x >> 7))), "r"(32u * unit_warps<WIDE>())
+      : "memory");
+  return r != 0;
+}
+
+// Attention of unit pp over its key slice, tile by tile as the MMA thread
+// completes each S tile: P = 2^(s sl2 - m) (bf16, P^T MN-major core matrices)
+// into the unit's P double buffer for the MMA thread, so the value tiles are
+// consumed while later key tiles still stream.  The stabiliser m_i (x sl2,
+// log2 units) is the largest logit of query i in the first step's tiles (one
+// tile, or one per warpgroup in the WIDE mode).  A later step whose logits
+// exceed m_i by more than kRaise raises m_i to that step's maximum first (a
+// decision taken jointly by the unit's threads; real inputs do not take it):
+// every PV product issued so far completes, column i of the O^T accumulator
+// and the running sums are scaled by 2^(m_old - m_new), and the step's P uses
+// the new m.  Otherwise P <= 2^kRaise, which bf16 holds and fp32 sums over
+// any key list accumulate without overflow; terms more than 2^126 below the
+// stabiliser flush to zero, as they do below the largest term.  Rows past the
+// slice get P = 0.  The final m -> us.mloc, the row sums of P -> us.lacc.
+// WIDE: warpgroup w forms the P tiles t = w, w + 2, ... (always P buffer w).
+constexpr float kRaise = 64.f;
+template <bool WIDE>
+__device__ __noinline__ void attn_online(Misc& ms, int* status, float sl2, uint8_t* pbase, int pp, uint32_t tb,
+                                         int ntl, int mc, uint32_t& tpar, uint32_t ocol) {
   const int tid = ctid<WIDE>(), lane = tid & 31, warp = tid >> 5, row = tid & (TM - 1);
+  const int wg = unit_wg<WIDE>();
+  constexpr int NW = unit_warps<WIDE>();
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
   UnitState& us = ms.us[pp];
+  UnitState& ws = wslots<WIDE>(ms, pp, warp);
   const f32x2 s2 = pk2(sl2, sl2);
   f32x2 nml[16], lsum2[16];
 #pragma unroll
   for (int k = 0; k < 16; ++k) {
-    nml[k] = pk2(-us.mloc[2 * k], -us.mloc[2 * k + 1]);
+    nml[k] = pk2(0.f, 0.f);
     lsum2[k] = pk2(0.f, 0.f);
   }
+  const int nsteps = (ntl + tile_step<WIDE>() - 1) / tile_step<WIDE>();
 #pragma unroll 1
-  for (int t = unit_wg<WIDE>(); t < ntl; t += tile_step<WIDE>()) {
-    const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
-    if (t >= 2) {
-      if (lane == 0) wait_or_abort(bar_addr(ms.pempty[pp][pb]), (pn - 1) & 1u, ms, status);
-      __syncwarp();
-    }
+  for (int j = 0; j < nsteps; ++j) {
+    const int t = j * tile_step<WIDE>() + wg;
+    const bool has = t < ntl;  // warp-uniform
     uint32_t ra[32];
-    tmem_ld32_issue(tb + lane_base + 32 * t, ra);
-    tmem_wait_ld();
-    uint32_t w[16];
-    if (t * TM + row < mc) {
+    if (has) {
+      wait_or_abort(bar_addr(ms.tdone[pp][t]), (tpar >> t) & 1u, ms, status);
+      tpar ^= 1u << t;
+      tc_fence_after();
+      tmem_ld32_issue(tb + lane_base + 32 * t, ra);
+      tmem_wait_ld();
+    }
+    const bool valid = has && t * TM + row < mc;
+    bool raise = j == 0;
+    if (j > 0) {
+      bool over = false;
+      if (valid) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
+          over |= fmaxf(x.x, x.y) > kRaise;
+        }
+      }
+      raise = csync_or<WIDE>(over);
+    }
+    if (raise) {
+      // The step's column maxima: lane i of each warp keeps column i's.
+      float mcol = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float m = warp_max_f32(valid ? __uint_as_float(ra[i]) : -INFINITY);
+        mcol = lane == i ? m : mcol;
+      }
+      ws.red[warp & 3][lane] = mcol;
+      csync<WIDE>();
+      if (tid < 32) {
+        float m = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) m = fmaxf(m, wslots<WIDE>(ms, pp, w).red[w & 3][tid]);
+        m *= sl2;
+        const float mn = j == 0 ? m : fmaxf(us.mloc[tid], m);
+        us.alpha[tid] = j == 0 ? 1.f : ex2(us.mloc[tid] - mn);
+        us.mloc[tid] = mn;
+      }
+      csync<WIDE>();
 #pragma unroll
       for (int k = 0; k < 16; ++k) {
-        const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
-        const __nv_bfloat162 h2 = __floats2bfloat162_rn(ex2(x.x), ex2(x.y));
-        lsum2[k] = add2(lsum2[k], pk2(__low2float(h2), __high2float(h2)));
-        w[k] = *reinterpret_cast<const uint32_t*>(&h2);
+        nml[k] = pk2(-us.mloc[2 * k], -us.mloc[2 * k + 1]);
+        lsum2[k] = mul2(lsum2[k], pk2(us.alpha[2 * k], us.alpha[2 * k + 1]));
       }
-    } else {
+      if (j > 0 && wg == 0) {
+        // Every PV product issued so far (through tile tl) completes; then the
+        // accumulator's columns take the factor.  The tile's P is not
+        // announced before, so the next product sees the scaled O^T.
+        const int tl = j * tile_step<WIDE>() - 1;
+        if (lane == 0) wait_or_abort(bar_addr(ms.pempty[pp][tl & 1]), (uint32_t)(tl >> 1) & 1u, ms, status);
+        __syncwarp();
+        tc_fence_after();
+        uint32_t o[32];
+        tmem_ld32_issue(ocol + lane_base, o);
+        tmem_wait_ld();
 #pragma unroll
-      for (int k = 0; k < 16; ++k) w[k] = 0u;  // rows past the slice: P = 0
+        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * us.alpha[i]);
+        tmem_st32(ocol + lane_base, o);
+        tmem_wait_st();
+        tc_fence_before();
+      }
     }
-    // P^T, MN-major core matrices: key group r / 8, query chunk ch.
-    const int r = row;
-    uint8_t* dst = pbase + pb * P_BYTES + (r >> 3) * 512 + (r & 7) * 16;
+    if (has) {
+      const uint32_t pb = (uint32_t)t & 1u, pn = (uint32_t)t >> 1;
+      if (t >= 2) {
+        if (lane == 0) wait_or_abort(bar_addr(ms.pempty[pp][pb]), (pn - 1) & 1u, ms, status);
+        __syncwarp();
+      }
+      uint32_t w[16];
+      if (valid) {
 #pragma unroll
-    for (int ch = 0; ch < 4; ++ch)
-      *reinterpret_cast<uint4*>(dst + ch * 128) = make_uint4(w[4 * ch], w[4 * ch + 1], w[4 * ch + 2], w[4 * ch + 3]);
-    fence_proxy_async();
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive(bar_addr(ms.pfull[pp][pb]));
+        for (int k = 0; k < 16; ++k) {
+          const float2 x = up2(fma2(pk2(__uint_as_float(ra[2 * k]), __uint_as_float(ra[2 * k + 1])), s2, nml[k]));
+          const __nv_bfloat162 h2 = __floats2bfloat162_rn(ex2(x.x), ex2(x.y));
+          lsum2[k] = add2(lsum2[k], pk2(__low2float(h2), __high2float(h2)));
+          w[k] = *reinterpret_cast<const uint32_t*>(&h2);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) w[k] = 0u;  // rows past the slice: P = 0
+      }
+      // P^T, MN-major core matrices: key group r / 8, query chunk ch.
+      uint8_t* dst = pbase + pb * P_BYTES + (row >> 3) * 512 + (row & 7) * 16;
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch)
+        *reinterpret_cast<uint4*>(dst + ch * 128) = make_uint4(w[4 * ch], w[4 * ch + 1], w[4 * ch + 2], w[4 * ch + 3]);
+      fence_proxy_async();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_addr(ms.pfull[pp][pb]));
+    }
   }
   float lsum[32];
 #pragma unroll
@@ -1311,13 +1397,14 @@ __device__ __noinline__ void attn_p(Misc& ms, int* status, float sl2, uint8_t* p
     lsum[2 * k] = v.x;
     lsum[2 * k + 1] = v.y;
   }
-  wslots<WIDE>(ms, pp, warp).red[warp & 3][lane] = transpose_reduce32<false>(lsum, lane);
+  ws.red[warp & 3][lane] = transpose_reduce32<false>(lsum, lane);
   csync<WIDE>();
   if (tid < 32) {
     float sum = 0.f;
 #pragma unroll
-    for (int w = 0; w < unit_warps<WIDE>(); ++w) sum += wslots<WIDE>(ms, pp, w).red[w & 3][tid];
+    for (int w = 0; w < NW; ++w) sum += wslots<WIDE>(ms, pp, w).red[w & 3][tid];
     us.lacc[tid] = sum;
+    if (nsteps == 0) us.mloc[tid] = -INFINITY;  // no keys in this CTA's slice
   }
   csync<WIDE>();
 }
@@ -1435,13 +1522,10 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   const float sl2 = p.scale_log2;
   int64_t sets_off = 0;  // the level sets of the scales above this launch's first
   for (int l = p.L; l > c.lev_top; --l) sets_off += p.keep[l];
-  // Parity of the unit's next mdone phase (the attention's two: S tiles
-  // scored, then PV products done).  The MMA thread commits a phase only for
-  // a non-empty stream.
-  uint32_t mdp = 0;
+  // The unit's mdone barrier completes one phase, when the attention's PV
+  // products are done (the MMA thread commits it only for a non-empty slice).
   auto wait_mdone = [&]() {
-    wait_or_abort(bar_addr(ms.mdone[pp]), mdp, ms, p.status);
-    mdp ^= 1u;
+    wait_or_abort(bar_addr(ms.mdone[pp]), 0u, ms, p.status);
     tc_fence_after();
   };
   // A launch that starts below the top scale (its rows dense, so the
@@ -1453,6 +1537,26 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
     int32_t* Jp = unit_J(c, p, pp, c.lev_top + 1);
 #pragma unroll 1
     for (int i = tid; i < p.keep[c.lev_top + 1]; i += TN) Jp[i] = src[2 * i] >> 1;
+  }
+  // The first pass through the Top-K's code fetches its instructions from
+  // memory, where they queue behind the first scale's row streams (several us
+  // at 32K).  In a two-unit cluster unit 1's warpgroup, which waits for its
+  // first rows until unit 0's have streamed, runs the Top-K once on synthetic
+  // keys with the first scale's list length, so unit 0's first selection
+  // finds the code cached (measured: 32K step 82.6 -> 80.5 us; in one-unit
+  // clusters the warm-up delays the unit's own first scale and the 128K step
+  // was 2 us slower).  Its key buffer is the one the scale below receives,
+  // which no CTA fills before this one has finished its first selection; the
+  // Top-K leaves its scratch cleared.
+  if (!WIDE && pp == 1 && c.lev_top == p.L && c.lev_top > c.lev_end) {
+    const int m0 = m_total(p, c.lev_top);
+    int32_t* wk = unit_J(c, p, pp, c.lev_top - 1);
+    // 512 distinct values, each several times: one bucket round whose
+    // boundary bucket holds more keys than it needs, like real keys.
+#pragma unroll 1
+    for (int i = tid; i < m0; i += TN) wk[i] = __float_as_int((float)((((uint32_t)i * 2654435761u) >> 8) & 511u));
+    csync<WIDE>();
+    select_topk<WIDE>(smem_u32(wk), m0, p.keep[c.lev_top], 0u, 1, sc_a, 0.f, 511.f);
   }
   uint32_t tpar = 0;  // parity of each scale-tile barrier's next phase
 #pragma unroll 1
@@ -1531,10 +1635,8 @@ __device__ void compute_role(const Ctx& c, const FusedParams& p) {
   int a0, mc;
   attn_slice(p.keep[0] + p.ng, c.rank, c.cs, a0, mc);
   const int ntl = tiles_of(mc);
-  if (ntl > 0) wait_mdone();
-  pass_max<WIDE>(ms, pp, tb, ntl, mc, sl2);
-  attn_p<WIDE>(ms, p.status, sl2, ubuf, pp, tb, ntl, mc);
-  if (ntl > 0) wait_mdone();
+  attn_online<WIDE>(ms, p.status, sl2, ubuf, pp, tb, ntl, mc, tpar, tb + p.ucols - 32);
+  if (ntl > 0) wait_mdone();  // every PV product of the unit is done
   if (unit_wg<WIDE>() != 0) return;  // one warpgroup combines
   attn_combine(ms, p, c.rank, c.cs, u, ubuf, us, pp, tb + p.ucols - 32);
 }
@@ -1576,6 +1678,7 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
       mbar_init(bar_addr(ms.cbar[pp]), 1);
       mbar_init(bar_addr(ms.cready[pp]), c.cs);
     }
+    mbar_init(bar_addr(ms.qfull), NPT);
     mbar_init(bar_addr(ms.stallbar), 1);
     mbar_init(bar_addr(ms.drainbar), 1);
     ms.wait_limit = p.wait_limit;
@@ -1618,20 +1721,6 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
     // set-up above overlaps their tail when the launch is programmatic).
     grid_dep_wait();
     grid_dep_launch();
-    // Query blocks -> shared memory, K-major core matrices, rows >= q zero.
-    for (int pp = 0; pp < c.np; ++pp) {
-      const int u = c.u0 + pp;
-      const bf16* qb = p.Q + (int64_t)(u / p.H) * p.qsb + (int64_t)(u % p.H) * p.qsh;
-      uint8_t* sq = smem + c.ly.q + pp * Q_BYTES;
-      for (int e = tid; e < NQ * (D / 8); e += NS) {
-        const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
-        const int i = g * 8 + rr;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (i < p.q) v = __ldg(reinterpret_cast<const uint4*>(qb + (int64_t)i * p.qss + ch * 8));
-        *reinterpret_cast<uint4*>(sq + g * QGRP + ch * 128 + rr * 16) = v;
-      }
-    }
-    fence_proxy_async();
     tc_fence_before();
     named_sync(kSetupSyncId, NS);
     tc_fence_after();

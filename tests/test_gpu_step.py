@@ -179,3 +179,42 @@ def test_step_exact_ties(n, period, L, keep):
             assert np.array_equal(gsets[lev], sets[lev]), f"unit {u} scale {lev}"
         assert np.array_equal(run.idx[u].cpu().numpy(), mu0), f"unit {u} mu0"
         assert_close_out(f64(run.O[0, u]), O, torch.bfloat16)
+
+
+@pytest.mark.parametrize("B,H,n,L,keep", [
+    (1, 32, 8192, 3, [476, 442, 410, 819]),                # one unit a cluster: raised at the last key tile
+    (2, 32, 32768, 4, [1024, 1024, 1024, 1024, 2048]),     # two units a cluster: raised mid-stream
+    (1, 32, 32768, 4, [1024, 1024, 1024, 1024, 2048]),     # one unit on both warpgroups: raised at step 1
+])
+def test_step_raised_stabiliser(B, H, n, L, keep):
+    # Generation row 0 of every unit gets logits of 55 to several hundred
+    # (natural units) against every query row, far above the sparse keys'.
+    # It sits in a later key tile of the last CTA of each cluster, so that
+    # CTA's attention raises its stabiliser mid-stream (the accumulator and
+    # the running sums are rescaled); the output must match the oracle's
+    # attention over the kernel's own indices.
+    Q, K, V, Kg, Vg = _rand(n + L + 77, B, H, n, 32, 32)
+    # Every query row gets a component of 6 along one random direction per
+    # unit, and generation row 0 points along it.
+    g = torch.Generator(device="cpu").manual_seed(n + B)
+    uvec = torch.randn(B, H, 128, generator=g, dtype=torch.float64)
+    uvec = (uvec / uvec.norm(dim=-1, keepdim=True)).cuda()
+    Q = (Q.double() + 6.0 * uvec[:, :, None, :]).to(torch.bfloat16)
+    proj = torch.einsum("bhqd,bhd->bhq", Q.double(), uvec)
+    lo = proj.min(dim=2).values
+    assert torch.all(lo > 0.5)
+    c = 55.0 * 128 ** 0.5 / lo
+    Kg = Kg.clone()
+    Kg[:, :, 0, :] = (c[..., None] * uvec).to(torch.bfloat16)
+    run = LibRun(Q, K, V, Kg, Vg, L, keep).step()
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    for u in [0, 1, H - 1, B * H - 1]:
+        b, h = divmod(u, H)
+        Qn, Kn, Vn, Kgn, Vgn = (f64(t[b, h]) for t in (Q, K, V, Kg, Vg))
+        s = Qn @ Kgn[0] / np.sqrt(128)
+        assert s.min() >= 54.0
+        idx = run.idx[u].cpu().numpy()
+        pyr = oracle.haar_pyramid_spec32(Kn.astype(np.float32), L, True).astype(np.float64)
+        eps_valid(Qn, pyr, Kn, n, L, keep, run.level_sets(u))
+        assert_close_out(f64(run.O[b, h]), oracle.sparse_attn(Qn, Kn, Vn, idx, Kgn, Vgn), torch.bfloat16)
