@@ -106,6 +106,14 @@ def fused_shape(w: synth.Workload) -> bool:
     return w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group == 1
 
 
+def grouped_fused(w: synth.Workload) -> bool:
+    """Grouped query heads that wf_step filters with the grouped filter kernel
+    (bf16, head_dim 128, <= 32 rows a query head, <= 256 stacked rows), then
+    attends with the per-stage tensor-core attention (split + combine)."""
+    return (WAVELET is None and w.dtype == "bf16" and w.head_dim == 128 and w.q <= 32 and w.group > 1
+            and w.group * w.q <= 256)
+
+
 def recorded_traffic(w: synth.Workload):
     """DRAM bytes per launch of the fused kernel from the committed ncu record,
     if it was taken on this workload with the current kernel source."""
@@ -128,6 +136,8 @@ def recorded_traffic(w: synth.Workload):
 def launches_per_step(w: synth.Workload) -> int:
     if fused_eligible(w):
         return 1
+    if grouped_fused(w):  # the grouped filter kernel, the attention split and its combine
+        return 3
     trim = int(w.keep[0]) < 2 * int(w.keep[1])
     if WAVELET and fused_shape(w):  # one fused launch per scale, a transform before each below the top
         return w.levels + (w.levels - 1)
@@ -522,7 +532,9 @@ def main():
                        f"wf_step_wavelet ({WAVELET}, periodized; the gathered candidate blocks transformed at every "
                        "scale" + ("; one fused filter launch per scale, the last with the sparse attention)"
                                   if fused_shape(w) else "; per-stage kernels)") + " per layer" if WAVELET else
-                       "wf_step (per-stage filter and sparse-attention kernels) per layer") + (
+                       ("wf_step (grouped filter kernel, then the per-stage sparse-attention kernels) per layer"
+                        if grouped_fused(w) else
+                        "wf_step (per-stage filter and sparse-attention kernels) per layer")) + (
                   f"; wf_dwt_build refresh every {w.refresh_every} steps" if w.refresh_every else
                   ("; scale-L rows built once before timing" if WAVELET else "; pyramid built once before timing")),
               "l2": "flushed before every timed step (256 MiB write)", "parallelism": f"replicas{args.gpus}",
@@ -586,6 +598,7 @@ def main():
     kname = "wf_fused_kernel" if fused_eligible(w) else (
         ("approx_kernel + wf_fused_kernel (one launch per scale)" if fused_shape(w) else
          "per-stage kernels (approx/score/weights/select/attn)") if WAVELET else
+        "wf_gqa_filter_kernel + tc_attn_kernel + attn_combine_kernel" if grouped_fused(w) else
         "per-stage kernels (score/weights/select/attn)")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                 "frac_of_nominal_7900": achieved / 7900.0,

@@ -339,9 +339,18 @@ WF_API wf_status wf_step(const void* Q, const wf_tensor* q, const void* K, const
                          level_sets, O, *o, status, s);
     return cuda_status(e);
   }
-  const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
-  if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, status, s)) != cudaSuccess)
-    return WF_ERR_CUDA;
+  // Grouped query heads: the grouped filter kernel where it applies, else the
+  // per-stage filter; then the per-stage attention.
+  const wf::GqaPlan gp = wf::plan_gqa(*q, *kv, levels, keep, sms);
+  if (gp.ok) {
+    if ((e = wf::launch_gqa_filter(gp, Q, *q, K, *kv, coeffs, levels, keep, idx, level_sets, status, s)) !=
+        cudaSuccess)
+      return WF_ERR_CUDA;
+  } else {
+    const wf::FilterPlan fl = wf::plan_filter(*q, *kv, levels, keep);
+    if ((e = wf::launch_filter(fl, Q, *q, coeffs, K, *kv, idx, level_sets, scratch, status, s)) != cudaSuccess)
+      return WF_ERR_CUDA;
+  }
   const wf::AttnPlan ap = wf::plan_attn(*q, keep[0], n_g, group_of(q, kv));
   const float sc = 1.0f / sqrtf((float)q->head_dim);
   e = wf::launch_attn(ap, Q, *q, K, V, *kv, idx, Kg, Vg, n_g > 0 ? g : nullptr, O, *o, sc, scratch, status, s);

@@ -105,6 +105,7 @@ struct Misc {
   unsigned long long pfull[MAXP][2], pempty[MAXP][2], cbar[MAXP], cready[MAXP];
   UnitState us[MAXP];
   unsigned long long qfull;     // the query blocks have landed (the producers' first copies)
+  unsigned long long rdone[2], rfree[2];  // grouped filter: a TMEM region's logits are ready / read
   unsigned long long stallbar;  // completed by nothing (the test-only stalled first wait)
   unsigned long long drainbar;  // the MMA thread's final commit
   long long wait_limit;         // bound of the waits that can give up (cycles)
@@ -158,6 +159,7 @@ struct FusedParams {
   uint32_t ecol;              // column of the stored exponentials in a unit region (0: none)
   long long wait_limit;       // bound of the waits that can give up (cycles)
   int stall;                  // test-only: the MMA thread's first wait never completes
+  int G, nch;                 // grouped filter: query heads per key head, 32-row chunks of the stacked block
   int32_t keep[12];
   float scale_log2;           // log2(e) / sqrt(d)
   // The scales this launch runs, lev_top down to lev_bot (the whole chain, L
@@ -1754,6 +1756,423 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Grouped query heads (reading 21): the filter of one key head for the
+// stacked query rows of its G query heads, W_j summed over every row of the
+// group (Eq. 7-11; Dream-7B's 7 query heads per key head give 224 rows).
+// ---------------------------------------------------------------------------
+//
+// One cluster of CS CTAs per (batch, key head) unit, both compute warpgroups
+// on the unit, the same producers and Top-K as the one-head kernel.  The
+// stacked query block (G q rows in chunks of 32) is the N side of the MMAs: a
+// tile's logits take 32 nch TMEM columns, so the CTA holds two tiles at a
+// time (warpgroup w reads region w, the tiles t = w, w + 2, ...), and every
+// scale runs two passes over its rows, the second re-streamed (from L2):
+//   1. per query column, the largest logit (x sl2) and the sum of
+//      exponentials over the CTA's rows: each tile's exponentials are taken
+//      relative to that tile's column maxima and merged as they come, so
+//      nothing overflows; the warps' statistics merge into the CTA's (M, S),
+//      which the cluster exchanges into the normalisers c_i = M + log2 S;
+//   2. each row's ranking key log2 W_j = log2 sum_i 2^(l_ij sl2 - c_i) over
+//      all stacked rows (a running maximum over the chunks keeps tiny sums
+//      exact), all-gathered, then the Top-K (Eq. 9).
+// The selection is written as mu^0 (and the level sets); the attention runs
+// afterwards on the per-stage tensor-core kernels.
+constexpr int GQ_MAXCH = 8;  // chunks of 32 stacked query rows (G q <= 256)
+
+struct GqaLayout {
+  uint32_t q, sc, misc, wst, xst, cvec, buf, bufw, total;
+};
+__host__ __device__ inline GqaLayout gqa_layout(int stages, int nch, int cs, int cmax, int kmax) {
+  GqaLayout l;
+  const uint32_t nq = 32u * (uint32_t)nch;
+  l.q = (uint32_t)stages * TILE_BYTES;
+  l.sc = l.q + (uint32_t)nch * Q_BYTES;                            // Top-K scratch
+  l.misc = (l.sc + (uint32_t)sizeof(SelScratch) + 127u) / 128u * 128u;
+  l.wst = (l.misc + (uint32_t)sizeof(Misc) + 15u) / 16u * 16u;     // [4][nq] float2: one warpgroup's column statistics
+  l.xst = l.wst + 4u * nq * 8u;                                    // [cs][nq] float2: every CTA's (M, S) per column
+  l.cvec = l.xst + (uint32_t)cs * nq * 8u;                         // [nq] float: the normalisers c_i
+  l.buf = (l.cvec + nq * 4u + 127u) / 128u * 128u;                 // two key / selection buffers
+  l.bufw = (uint32_t)((max(cmax, kmax) + 3) / 4 * 4);
+  l.total = l.buf + 2u * 4u * l.bufw;
+  return l;
+}
+
+// (m, s) pairs of sums of 2^(x - m): the pair of their union.
+__device__ __forceinline__ float2 merge_ms(float2 a, float2 b) {
+  if (!(b.y > 0.f)) return a;
+  if (!(a.y > 0.f)) return b;
+  const float M = fmaxf(a.x, b.x);
+  return make_float2(M, a.y * ex2(a.x - M) + b.y * ex2(b.x - M));
+}
+
+template <int S>
+__device__ void gqa_producer_role(const Ctx& c, const FusedParams& p) {
+  Misc& ms = *c.ms;
+  const int pt = threadIdx.x - P0;
+  // The stacked query block first: row i = g q + r is row r of query head
+  // h G + g; chunk ch holds rows 32 ch .. 32 ch + 31 (K-major core matrices),
+  // rows >= G q zero-filled.
+  const int64_t b = c.u0 / p.H, h = c.u0 % p.H;
+  const int nq = p.G * p.q;
+  for (int ch = 0; ch < p.nch; ++ch) {
+    const uint32_t sq = smem_u32(c.smem + c.ly.q + ch * Q_BYTES);
+    for (int e = pt; e < NQ * (D / 8); e += NPT) {
+      const int rr = e & 7, c16 = (e >> 3) & (D / 8 - 1), g8 = e >> 7;
+      const int i = ch * NQ + g8 * 8 + rr;
+      const int ic = min(i, nq - 1), hd = ic / p.q, r = ic - hd * p.q;
+      const bf16* src = p.Q + b * p.qsb + (h * p.G + hd) * p.qsh + (int64_t)r * p.qss + c16 * 8;
+      cp_async16_zfill(sq + (uint32_t)(g8 * QGRP + c16 * 128 + rr * 16), src, i < nq);
+    }
+  }
+  cp_async_arrive_noinc(bar_addr(ms.qfull));
+  int it = 0;
+  for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
+    if (lev != c.lev_top) wait_or_abort(bar_addr(ms.jready[0]), (uint32_t)(c.lev_top - lev - 1) & 1u, ms, p.status);
+    int g0, mc;
+    scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
+    const int ntl = tiles_of(mc);
+    const RowSrc src = scale_src(c, p, 0, lev, g0, mc);
+    produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, src, pt);  // pass 1
+    it += ntl;
+    produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, src, pt);  // pass 2: the same rows again
+    it += ntl;
+  }
+  cp_async_wait_all();
+}
+
+// Both passes of every scale: tile t's logits for every query chunk into
+// TMEM region t % 2 once the warpgroup reading that region has released it.
+template <int S>
+__device__ void gqa_mma_role(const Ctx& c, const FusedParams& p) {
+  Misc& ms = *c.ms;
+  if (p.stall) wait_or_abort(bar_addr(ms.stallbar), 0u, ms, p.status);
+  wait_or_abort(bar_addr(ms.qfull), 0u, ms, p.status);
+  fence_proxy_async();
+  const uint32_t sq = smem_u32(c.smem + c.ly.q);
+  const uint32_t rcols = 32u * (uint32_t)p.nch;
+  uint32_t used[2] = {0u, 0u};
+  int it = 0;
+  for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
+    int g0, mc;
+    scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
+    const int ntl = tiles_of(mc);
+#pragma unroll 1
+    for (int k = 0; k < 2 * ntl; ++k) {
+      const int t = k < ntl ? k : k - ntl, r = t & 1, slot = it + k, s = slot % S;
+      if (used[r] > 0) wait_or_abort(bar_addr(ms.rfree[r]), (used[r] - 1u) & 1u, ms, p.status);
+      ++used[r];
+      wait_or_abort(bar_addr(ms.full[s]), (uint32_t)(slot / S) & 1u, ms, p.status);
+      fence_proxy_async();
+      if (!aborted(ms)) {
+        tc_fence_after();
+        const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
+#pragma unroll 1
+        for (int ch = 0; ch < p.nch; ++ch)
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16(c.tmem + (uint32_t)r * rcols + 32u * ch, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
+                       smem_desc(sq + ch * Q_BYTES + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
+      }
+      mma_commit(bar_addr(ms.empty[s]));
+      mma_commit(bar_addr(ms.rdone[r]));
+    }
+    it += 2 * ntl;
+  }
+  mma_commit(bar_addr(ms.drainbar));
+  (void)mbar_wait_bounded(bar_addr(ms.drainbar), 0u, kDefaultWaitLimit);
+}
+
+__device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLayout gl) {
+  Misc& ms = *c.ms;
+  constexpr int TN = 32 * unit_warps<true>();
+  const int tid = ctid<true>(), lane = tid & 31, warp = tid >> 5, wg = tid >> 7, qd = warp & 3, row = tid & (TM - 1);
+  const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+  const int nch = p.nch, nqp = 32 * nch, nq = p.G * p.q;
+  const uint32_t treg = c.tmem + (uint32_t)wg * 32u * (uint32_t)nch;  // this warpgroup's TMEM region
+  const uint32_t sc_a = smem_u32(c.smem + gl.sc);
+  float2* wst = reinterpret_cast<float2*>(c.smem + gl.wst);
+  float2* xst = reinterpret_cast<float2*>(c.smem + gl.xst);
+  float* cvec = reinterpret_cast<float*>(c.smem + gl.cvec);
+  const uint32_t cvec_a = smem_u32(cvec);
+  const float sl2 = p.scale_log2;
+  const int u = c.u0;
+  int64_t sets_off = 0;
+  uint32_t dpar = 0;  // parity of the next phase of this warpgroup's rdone barrier
+#pragma unroll 1
+  for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
+    const uint32_t ph = (uint32_t)(c.lev_top - lev) & 1u;
+    const int m = m_total(p, lev);
+    int g0, mc;
+    scale_slice(m, c.rank, c.cs, g0, mc);
+    const int ntl = tiles_of(mc);
+    const int kb = p.keep[lev];
+    int32_t* J = unit_J(c, p, 0, lev);
+    const uint32_t keys_a = smem_u32(J);
+
+    // Pass 1: this warp's (max, sum) of each query column over its rows;
+    // lane l keeps column 32 ch + l of every chunk (a dynamically indexed,
+    // so thread-local, array).
+    float2 st[GQ_MAXCH];
+#pragma unroll
+    for (int ch = 0; ch < GQ_MAXCH; ++ch) st[ch] = make_float2(-INFINITY, 0.f);
+#pragma unroll 1
+    for (int t = wg; t < ntl; t += 2) {
+      wait_or_abort(bar_addr(ms.rdone[wg]), dpar, ms, p.status);
+      dpar ^= 1u;
+      tc_fence_after();
+      const bool valid = t * TM + row < mc;
+#pragma unroll 1
+      for (int ch = 0; ch < nch; ++ch) {
+        uint32_t ra[32];
+        tmem_ld32_issue(treg + 32u * ch + lane_base, ra);
+        tmem_wait_ld();
+        float e[32];
+        float tm = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float v = valid ? __uint_as_float(ra[i]) : -INFINITY;
+          const float mi = warp_max_f32(v);  // column i's largest logit among the warp's rows
+          tm = lane == i ? mi : tm;
+          e[i] = valid ? ex2((v - mi) * sl2) : 0.f;
+        }
+        const float ts = transpose_reduce32<false>(e, lane);  // lane l: column l's sum
+        st[ch] = merge_ms(st[ch], make_float2(tm * sl2, ts));
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_addr(ms.rfree[wg]));
+    }
+    // The eight warps' statistics -> the CTA's (M, S) per column, sent to
+    // every cluster CTA.
+    if (wg == 1)
+#pragma unroll 1
+      for (int ch = 0; ch < nch; ++ch) wst[qd * nqp + 32 * ch + lane] = st[ch];
+    csync<true>();
+    if (wg == 0)
+#pragma unroll 1
+      for (int ch = 0; ch < nch; ++ch) {
+        float2& w = wst[qd * nqp + 32 * ch + lane];
+        w = merge_ms(st[ch], w);
+      }
+    csync<true>();
+    {
+      const uint32_t xbar = bar_addr(ms.xbar[0]);
+      const uint32_t nr = aborted(ms) ? 0u : c.cs;  // after a wait gave up, nothing goes to the cluster
+#pragma unroll 1
+      for (int col = tid; col < nqp; col += TN) {
+        float2 a = wst[col];
+#pragma unroll
+        for (int q4 = 1; q4 < 4; ++q4) a = merge_ms(a, wst[q4 * nqp + col]);
+        const uint32_t dst = smem_u32(&xst[c.rank * nqp + col]);
+#pragma unroll 1
+        for (uint32_t r = 0; r < nr; ++r)
+          st_async_v2(map_rank(dst, r), __float_as_uint(a.x), __float_as_uint(a.y), map_rank(xbar, r));
+      }
+    }
+    wait_cluster_or_abort(bar_addr(ms.xbar[0]), ph, ms, p.status);
+    if (tid == 0 && lev > c.lev_end && !aborted(ms))
+      mbar_arrive_expect_tx(bar_addr(ms.xbar[0]), c.cs * (uint32_t)nqp * 8u);
+#pragma unroll 1
+    for (int col = tid; col < nqp; col += TN) {
+      float2 a = make_float2(-INFINITY, 0.f);
+#pragma unroll 1
+      for (uint32_t r = 0; r < c.cs; ++r) a = merge_ms(a, xst[r * nqp + col]);
+      cvec[col] = col < nq ? a.x + lg2(a.y) : INFINITY;  // padded rows weigh 0
+    }
+    csync<true>();
+
+    // Pass 2: each row's ranking key over every stacked query row.
+    float kmin = INFINITY, kmax = -INFINITY;
+    const uint32_t kbar = bar_addr(ms.kbar[0]);
+    const uint32_t nr = aborted(ms) ? 0u : c.cs;
+#pragma unroll 1
+    for (int t = wg; t < ntl; t += 2) {
+      wait_or_abort(bar_addr(ms.rdone[wg]), dpar, ms, p.status);
+      dpar ^= 1u;
+      tc_fence_after();
+      float rm = -INFINITY, rs = 0.f;
+#pragma unroll 1
+      for (int ch = 0; ch < nch; ++ch) {
+        uint32_t ra[32];
+        tmem_ld32_issue(treg + 32u * ch + lane_base, ra);
+        tmem_wait_ld();
+        float x[32];
+        float mx = -INFINITY;
+#pragma unroll
+        for (int k4 = 0; k4 < 8; ++k4) {
+          const uint4 cv = lds_v4(cvec_a + 16u * (uint32_t)(8 * ch + k4));
+          x[4 * k4] = __uint_as_float(ra[4 * k4]) * sl2 - __uint_as_float(cv.x);
+          x[4 * k4 + 1] = __uint_as_float(ra[4 * k4 + 1]) * sl2 - __uint_as_float(cv.y);
+          x[4 * k4 + 2] = __uint_as_float(ra[4 * k4 + 2]) * sl2 - __uint_as_float(cv.z);
+          x[4 * k4 + 3] = __uint_as_float(ra[4 * k4 + 3]) * sl2 - __uint_as_float(cv.w);
+          mx = fmaxf(mx, fmax3(x[4 * k4], x[4 * k4 + 1], fmaxf(x[4 * k4 + 2], x[4 * k4 + 3])));
+        }
+        if (mx > rm) {
+          rs = rm == -INFINITY ? 0.f : rs * ex2(rm - mx);
+          rm = mx;
+        }
+        float z = 0.f;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) z += ex2(x[i] - rm);
+        rs += z;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_addr(ms.rfree[wg]));
+      const int j = t * TM + row;
+      if (j < mc) {
+        const float key = rm + lg2(rs);
+        kmin = fminf(kmin, key);
+        kmax = fmaxf(kmax, key);
+        const uint32_t dst = keys_a + 4u * (uint32_t)(g0 + j);
+#pragma unroll 1
+        for (uint32_t r = 0; r < nr; ++r) st_async_b32(map_rank(dst, r), __float_as_uint(key), map_rank(kbar, r));
+      }
+    }
+    kmin = warp_min_f32(kmin);
+    kmax = warp_max_f32(kmax);
+    if (lane == 0) {
+      const uint32_t dst = smem_u32(&wslots<true>(ms, 0, warp).kmm[c.rank][warp & 3]);
+#pragma unroll 1
+      for (uint32_t r = 0; r < nr; ++r)
+        st_async_v2(map_rank(dst, r), __float_as_uint(kmin), __float_as_uint(kmax), map_rank(kbar, r));
+    }
+    wait_cluster_or_abort(kbar, ph, ms, p.status);
+    float lo, hi;
+    {
+      constexpr int NW = unit_warps<true>();
+      float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll 1
+      for (int e = lane; e < (int)c.cs * NW; e += 32) {  // entry (CTA e / NW, warp e % NW)
+        const int w = e % NW;
+        const uint2 v = lds_v2(smem_u32(&wslots<true>(ms, 0, w).kmm[e / NW][w & 3]));
+        mm = make_float2(fminf(mm.x, __uint_as_float(v.x)), fmaxf(mm.y, __uint_as_float(v.y)));
+      }
+      lo = warp_min_f32(mm.x);
+      hi = warp_max_f32(mm.y);
+    }
+    // Eq. 9: Top-K (the same result in every CTA of the cluster).
+    select_topk<true>(keys_a, m, kb, smem_u32(unit_J(c, p, 0, lev + 1)), lev == p.L, sc_a, lo, hi);
+    if (tid == 0) {
+      if (lev > c.lev_end && !aborted(ms))
+        mbar_arrive_expect_tx(kbar, 4u * (uint32_t)m_total(p, lev - 1) + c.cs * unit_warps<true>() * 8u);
+      mbar_arrive(bar_addr(ms.jready[0]));
+    }
+    if (c.rank == 0) {
+      int32_t* ls = p.level_sets ? p.level_sets + (int64_t)u * p.sets_stride + sets_off : nullptr;
+      if (lev >= 1 && ls) {
+#pragma unroll 1
+        for (int i = tid; i < kb; i += TN) ls[i] = J[i];
+      }
+      if (lev == c.lev_end) {
+        // mu^0: the children of J^1, or the trimmed level-0 selection.
+        const int kk = p.keep[0];
+        int32_t* out = p.idx + (int64_t)u * kk;
+        int32_t* ls0 = ls ? ls + (lev >= 1 ? kb : 0) : nullptr;
+#pragma unroll 1
+        for (int t = tid; t < kk; t += TN) {
+          const int tok = p.trim ? J[t] : 2 * J[t >> 1] + (t & 1);
+          out[t] = tok;
+          if (ls0) ls0[t] = tok;
+        }
+      }
+    }
+    if (lev >= 1) sets_off += kb;
+  }
+}
+
+template <int S>
+__global__ void __launch_bounds__(NT, 1) wf_gqa_filter_kernel(const __grid_constant__ FusedParams p) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const GqaLayout gl = gqa_layout(S, p.nch, (int)cluster_size(), p.cmax, p.kmax);
+  Ctx c;
+  c.smem = smem;
+  c.ly.q = gl.q;
+  c.ly.p = gl.sc;
+  c.ly.misc = gl.misc;
+  c.ly.buf = gl.buf;
+  c.ly.bufw = gl.bufw;
+  c.ly.total = gl.total;
+  c.ms = reinterpret_cast<Misc*>(smem + gl.misc);
+  Misc& ms = *c.ms;
+  c.rank = cluster_rank();
+  c.cs = cluster_size();
+  c.u0 = (int)cluster_id_x();
+  c.np = 1;
+  c.lev_top = p.L;
+  c.lev_end = p.trim ? 0 : 1;
+  c.stages = S;
+  const int tid = threadIdx.x, warp = tid >> 5;
+
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(bar_addr(ms.full[s]), NPT);
+      mbar_init(bar_addr(ms.empty[s]), 1);
+    }
+    mbar_init(bar_addr(ms.jready[0]), 1);
+    mbar_init(bar_addr(ms.xbar[0]), 1);
+    mbar_init(bar_addr(ms.kbar[0]), 1);
+    for (int r = 0; r < 2; ++r) {
+      mbar_init(bar_addr(ms.rdone[r]), 1);
+      mbar_init(bar_addr(ms.rfree[r]), NCW);
+    }
+    mbar_init(bar_addr(ms.qfull), NPT);
+    mbar_init(bar_addr(ms.stallbar), 1);
+    mbar_init(bar_addr(ms.drainbar), 1);
+    ms.wait_limit = p.wait_limit;
+    ms.abort = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (warp > MMA_WARP) {
+    cluster_arrive_relaxed();
+    gqa_producer_role<S>(c, p);
+    cluster_wait();
+  } else {
+    constexpr int NS = NT - NPT;
+    if (tid == 0) {
+      mbar_arrive_expect_tx(bar_addr(ms.xbar[0]), c.cs * 32u * (uint32_t)p.nch * 8u);
+      mbar_arrive_expect_tx(bar_addr(ms.kbar[0]),
+                            4u * (uint32_t)m_total(p, c.lev_top) + c.cs * unit_warps<true>() * 8u);
+    }
+    if (warp == MMA_WARP) {
+      tmem_alloc(smem_u32(&ms.tmem_base), p.tmem_cols);
+      tmem_relinquish();
+    }
+    // The Top-K scratch starts zeroed (histogram, list counter, masks).
+    for (int e = tid; e < (int)((sizeof(SelScratch) + 15) / 16); e += NS)
+      *reinterpret_cast<uint4*>(smem + gl.sc + 16 * e) = make_uint4(0, 0, 0, 0);
+    tc_fence_before();
+    named_sync(kSetupSyncId, NS);
+    tc_fence_after();
+    c.tmem = ms.tmem_base;
+    cluster_sync();  // every CTA's barriers are armed before any remote arrival
+    if (warp < MMA_WARP) {
+      gqa_compute_role(c, p, gl);
+    } else {
+      if ((tid & 31) == 0) gqa_mma_role<S>(c, p);
+      __syncwarp();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_arrive();
+  cluster_wait();
+  if (warp == MMA_WARP) {
+    if (aborted(ms)) {
+      const unsigned long long t0 = globaltimer_ns();
+      while (globaltimer_ns() - t0 < 20000ull) {
+      }
+    }
+    tc_fence_after();
+    tmem_dealloc(c.tmem, p.tmem_cols);
+  }
+}
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -1994,6 +2413,138 @@ cudaError_t launch_fused(const FusedPlan& fp, const void* Q, const wf_tensor& qd
   cudaError_t e = ensure_smem_limit(fp.stages, fp.wide, cfg.dynamicSmemBytes);
   if (e != cudaSuccess) return e;
   e = cudaLaunchKernelEx(&cfg, fused_kernel(fp.stages, fp.wide), p);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+// The grouped filter (wf_gqa_filter_kernel): bf16, d = 128, G >= 2 query
+// heads per key head with q <= 32 rows each and G q <= 256, candidate lists
+// within the Top-K's 8192.  One unit per cluster; the largest cluster of up
+// to 8 CTAs whose grid fits the SMs in one wave with every cluster resident.
+GqaPlan plan_gqa(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int num_sms) {
+  GqaPlan gp{};
+  gp.ok = false;
+  if (kv.dtype != WF_BF16 || kv.head_dim != D || q.dtype != WF_BF16 || kv.heads <= 0 || levels > 10) return gp;
+  if (q.heads % kv.heads != 0 || q.batch != kv.batch) return gp;
+  const int G = q.heads / kv.heads;
+  if (G < 2 || q.seq > NQ || G * q.seq > GQ_MAXCH * NQ) return gp;
+  const int U = kv.batch * kv.heads;
+  int cmax = kv.seq >> levels, kmax = 0;
+  for (int l = 0; l <= levels; ++l) kmax = kmax > keep[l] ? kmax : keep[l];
+  for (int l = 1; l <= levels; ++l) cmax = cmax > 2 * keep[l] ? cmax : 2 * keep[l];
+  if (cmax > kMaxCand || kmax > kMaxCand) return gp;
+  const int nch = (G * q.seq + NQ - 1) / NQ;
+  constexpr int kStages = 3;
+  const size_t kMaxSmem = 227 * 1024;
+  int cs = 0;
+  size_t smem = 0;
+  for (int c = MAXCS; c >= 1 && cs == 0; --c) {
+    smem = gqa_layout(kStages, nch, c, cmax, kmax).total;
+    if (smem > kMaxSmem || U * c > num_sms) continue;
+    static std::mutex mu;
+    static std::map<std::tuple<int, int, size_t>, int> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return gp;
+    int n = 0;
+    {
+      std::lock_guard<std::mutex> lock(mu);
+      const auto key = std::make_tuple(dev, c, smem);
+      auto it = cache.find(key);
+      if (it != cache.end()) {
+        n = it->second;
+      } else {
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)c, 1, 1);
+        cfg.blockDim = dim3(NT, 1, 1);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = c;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        cudaError_t e = cudaFuncSetAttribute(wf_gqa_filter_kernel<kStages>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kMaxSmem);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, wf_gqa_filter_kernel<kStages>, &cfg);
+        if (e != cudaSuccess) {
+          (void)cudaGetLastError();
+          n = 0;
+        }
+        cache.emplace(key, n);
+      }
+    }
+    if (U <= n) cs = c;
+  }
+  if (cs == 0) {  // more units than one wave holds: single-CTA clusters in several waves
+    cs = 1;
+    smem = gqa_layout(kStages, nch, 1, cmax, kmax).total;
+    if (smem > kMaxSmem) return gp;
+  }
+  int cols = 32;
+  while (cols < 2 * NQ * nch) cols *= 2;
+  gp.ok = true;
+  gp.cs = cs;
+  gp.stages = kStages;
+  gp.smem = smem;
+  gp.tmem_cols = cols;
+  gp.nch = nch;
+  gp.G = G;
+  gp.cmax = cmax;
+  gp.kmax = kmax;
+  gp.trim = keep[0] < 2 * keep[1];
+  gp.U = U;
+  return gp;
+}
+
+cudaError_t launch_gqa_filter(const GqaPlan& gp, const void* Q, const wf_tensor& qd, const void* K,
+                              const wf_tensor& kv, const void* coeffs, int levels, const int32_t* keep, int32_t* idx,
+                              int32_t* level_sets, int* status, cudaStream_t s) {
+  FusedParams p;
+  memset(&p, 0, sizeof(p));
+  p.Q = static_cast<const bf16*>(Q);
+  p.qsb = qd.stride_b; p.qsh = qd.stride_h; p.qss = qd.stride_s;
+  p.K = static_cast<const bf16*>(K);
+  p.ksb = kv.stride_b; p.ksh = kv.stride_h; p.kss = kv.stride_s;
+  p.coeffs = static_cast<const bf16*>(coeffs);
+  p.rows_total = (int64_t)kv.seq - ((int64_t)kv.seq >> levels);
+  p.idx = idx;
+  p.level_sets = level_sets;
+  int64_t stride = 0;
+  for (int l = 0; l <= levels; ++l) stride += keep[l];
+  p.sets_stride = stride;
+  p.status = status;
+  p.q = qd.seq; p.n = kv.seq; p.U = gp.U; p.H = kv.heads; p.L = levels;
+  p.trim = gp.trim ? 1 : 0;
+  p.P = 1;
+  p.cmax = gp.cmax; p.kmax = gp.kmax;
+  p.tmem_cols = (uint32_t)gp.tmem_cols;
+  const WaitControls wc = wait_controls();
+  p.wait_limit = wc.limit;
+  p.stall = wc.stall;
+  for (int l = 0; l <= levels; ++l) p.keep[l] = keep[l];
+  p.scale_log2 = kLog2e / sqrtf((float)D);
+  p.lev_top = levels;
+  p.lev_bot = gp.trim ? 0 : 1;
+  p.final_sel = 1;
+  p.G = gp.G;
+  p.nch = gp.nch;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)(gp.U * gp.cs), 1, 1);
+  cfg.blockDim = dim3(NT, 1, 1);
+  cfg.dynamicSmemBytes = gp.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = gp.cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaFuncSetAttribute(wf_gqa_filter_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)gp.smem);
+  if (e != cudaSuccess) return e;
+  e = cudaLaunchKernelEx(&cfg, wf_gqa_filter_kernel<3>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -181,6 +181,20 @@ cudaError_t launch_literal_fused(const FusedPlan& fp, const FilterPlan& fl, cons
                                  const void* Vg, const wf_tensor* g, int wavelet, int32_t* idx, int32_t* level_sets,
                                  void* O, const wf_tensor* od, void* ws, int* status, cudaStream_t s);
 
+// The grouped-query filter on the fused kernel design (one cluster per
+// (batch, key head); the stacked query rows of the G query heads as MMA
+// columns): mu^0 and the level sets, for the per-stage attention after it.
+struct GqaPlan {
+  bool ok;
+  int cs, stages, tmem_cols, nch, G, cmax, kmax, U;
+  size_t smem;
+  bool trim;
+};
+GqaPlan plan_gqa(const wf_tensor& q, const wf_tensor& kv, int levels, const int32_t* keep, int num_sms);
+cudaError_t launch_gqa_filter(const GqaPlan& gp, const void* Q, const wf_tensor& qd, const void* K,
+                              const wf_tensor& kv, const void* coeffs, int levels, const int32_t* keep, int32_t* idx,
+                              int32_t* level_sets, int* status, cudaStream_t s);
+
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Bounds of the tensor-core kernels' waits.  The default, about one second of

@@ -63,7 +63,8 @@ def test_gqa_per_stage(base, kw, dtype):
     run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).run()
     torch.cuda.synchronize()
     _check_units(w, batch, run, range(w.units), dtype)
-    # wf_step takes the per-stage path for grouped heads: same indices, same output.
+    # wf_step (the grouped filter kernel for bf16, else the per-stage path):
+    # same indices, same output.
     step = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep)
     step.step()
     torch.cuda.synchronize()
@@ -100,3 +101,32 @@ def test_gqa_attention_equals_repeated_key_heads():
     wf.wf_workspace_status(ws)
     torch.cuda.synchronize()
     assert torch.equal(O1, grouped.O)
+
+
+@pytest.mark.parametrize("kw,units", [
+    (dict(), [0, 17, 31]),                                    # the Dream-shaped layer: clusters of 4, 4 tiles a scale
+    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3]),  # clusters of 8, one tile a scale, level-0 trim
+])
+def test_gqa_step_unplanted_valid_topk(kw, units):
+    # wf_step's grouped filter kernel on unplanted inputs: at every scale the
+    # selection must be a valid Top-K of W summed over the key head's stacked
+    # query rows (near-ties allow several answers), and the output must match
+    # the oracle's grouped attention over the kernel's own indices.
+    from helpers import eps_valid
+    w = _workload("g1", **kw) if kw else synth.WORKLOADS["g1"]
+    batch = synth.make_batch(w, planted=False, device="cuda", cfg="g1", units=units)
+    run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().step(refresh=False)
+    wf.wf_workspace_status(run.ws_step)
+    torch.cuda.synchronize()
+    G = w.group
+    for u in units:
+        b, h = divmod(u, w.heads)
+        Qh = f64(batch.Q[b, h * G:(h + 1) * G])
+        K, V, Kg, Vg = (f64(t[b, h]) for t in (batch.K, batch.V, batch.Kg, batch.Vg))
+        pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, True).astype(np.float64)
+        gsets = run.level_sets(u)
+        eps_valid(Qh.reshape(-1, Qh.shape[-1]), pyr, K, w.n, w.levels, list(w.keep), gsets)
+        idx = run.idx[u].cpu().numpy()
+        assert np.array_equal(idx, gsets[0])
+        O = oracle.sparse_attn_gqa(Qh, K, V, idx, Kg, Vg)
+        assert_close_out(f64(run.O[b, h * G:(h + 1) * G]), O, torch.bfloat16)
