@@ -1769,10 +1769,12 @@ __global__ void __launch_bounds__(NT, 1) wf_fused_kernel(const __grid_constant__
 // tile's logits take 32 nch TMEM columns, so the CTA holds two tiles at a
 // time (warpgroup w reads region w, the tiles t = w, w + 2, ...), and every
 // scale runs two passes over its rows, the second re-streamed (from L2):
-//   1. per query column, the largest logit (x sl2) and the sum of
-//      exponentials over the CTA's rows: each tile's exponentials are taken
-//      relative to that tile's column maxima and merged as they come, so
-//      nothing overflows; the warps' statistics merge into the CTA's (M, S),
+//   1. per query column, a stabiliser (x sl2) and the sum of exponentials
+//      over the CTA's rows: each tile's exponentials are taken relative to the
+//      largest logit of the query chunk among the warp's rows of that tile
+//      (a column whose terms would all flush to zero takes its own maximum),
+//      and merged as they come, so nothing overflows; the warps' statistics
+//      merge into the CTA's (M, S),
 //      which the cluster exchanges into the normalisers c_i = M + log2 S;
 //   2. each row's ranking key log2 W_j = log2 sum_i 2^(l_ij sl2 - c_i) over
 //      all stacked rows (a running maximum over the chunks keeps tiny sums
@@ -1852,6 +1854,7 @@ __device__ void gqa_mma_role(const Ctx& c, const FusedParams& p) {
   fence_proxy_async();
   const uint32_t sq = smem_u32(c.smem + c.ly.q);
   const uint32_t rcols = 32u * (uint32_t)p.nch;
+  const uint32_t idesc = idesc_bf16(TM, 32 * p.nch, 0, 0);  // A = rows (K-major), B = the stacked queries (K-major)
   uint32_t used[2] = {0u, 0u};
   int it = 0;
   for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
@@ -1868,14 +1871,14 @@ __device__ void gqa_mma_role(const Ctx& c, const FusedParams& p) {
       if (!aborted(ms)) {
         tc_fence_after();
         const uint32_t st = smem_u32(c.smem) + s * TILE_BYTES;
-#pragma unroll 1
-        for (int ch = 0; ch < p.nch; ++ch)
+        // One MMA per K step over every query chunk at once (N = 32 nch: the
+        // chunks' 8-row groups follow each other at the same stride).
 #pragma unroll
-          for (int h = 0; h < 2; ++h)
+        for (int h = 0; h < 2; ++h)
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-              mma_bf16(c.tmem + (uint32_t)r * rcols + 32u * ch, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
-                       smem_desc(sq + ch * Q_BYTES + (4 * h + kk) * 256, 128, QGRP), kIdescScore, (h | kk) != 0);
+          for (int kk = 0; kk < 4; ++kk)
+            mma_bf16(c.tmem + (uint32_t)r * rcols, smem_desc_sw128(st + h * HALF_BYTES + kk * 32, 16, 1024),
+                     smem_desc(sq + (4 * h + kk) * 256, 128, QGRP), idesc, (h | kk) != 0);
       }
       mma_commit(bar_addr(ms.empty[s]));
       mma_commit(bar_addr(ms.rdone[r]));
@@ -1930,16 +1933,29 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
         uint32_t ra[32];
         tmem_ld32_issue(treg + 32u * ch + lane_base, ra);
         tmem_wait_ld();
+        // Exponentials relative to the chunk's largest logit among the warp's
+        // rows (one warp-wide max), summed per column across the rows.
         float e[32];
-        float tm = -INFINITY;
+        float vm = -INFINITY;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float v = valid ? __uint_as_float(ra[i]) : -INFINITY;
-          const float mi = warp_max_f32(v);  // column i's largest logit among the warp's rows
-          tm = lane == i ? mi : tm;
-          e[i] = valid ? ex2((v - mi) * sl2) : 0.f;
+        for (int i = 0; i < 32; i += 2) vm = fmax3(vm, __uint_as_float(ra[i]), __uint_as_float(ra[i + 1]));
+        float tm = warp_max_f32(valid ? vm : -INFINITY);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) e[i] = valid ? ex2((__uint_as_float(ra[i]) - tm) * sl2) : 0.f;
+        float ts = transpose_reduce32<false>(e, lane);  // lane l: column l's sum
+        // A column whose every term flushed to zero (logits more than ~126
+        // below the chunk's largest, in log2 units) is summed again against
+        // each column's own maximum (the warp decides together).
+        if (__any_sync(0xffffffffu, !(ts > 0.f) && tm > -INFINITY)) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float v = valid ? __uint_as_float(ra[i]) : -INFINITY;
+            const float mi = warp_max_f32(v);  // column i's largest logit among the warp's rows
+            tm = lane == i ? mi : tm;
+            e[i] = valid ? ex2((v - mi) * sl2) : 0.f;
+          }
+          ts = transpose_reduce32<false>(e, lane);
         }
-        const float ts = transpose_reduce32<false>(e, lane);  // lane l: column l's sum
         st[ch] = merge_ms(st[ch], make_float2(tm * sl2, ts));
       }
       tc_fence_before();

@@ -103,18 +103,27 @@ def test_gqa_attention_equals_repeated_key_heads():
     assert torch.equal(O1, grouped.O)
 
 
-@pytest.mark.parametrize("kw,units", [
-    (dict(), [0, 17, 31]),                                    # the Dream-shaped layer: clusters of 4, 4 tiles a scale
-    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3]),  # clusters of 8, one tile a scale, level-0 trim
+@pytest.mark.parametrize("kw,units,hot", [
+    (dict(), [0, 17, 31], 0.0),                                    # the Dream-shaped layer: clusters of 4, 4 tiles a scale
+    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 0.0),  # clusters of 8, one tile a scale, level-0 trim
+    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 80.0),  # one query row 80x: other rows' terms flush
 ])
-def test_gqa_step_unplanted_valid_topk(kw, units):
+def test_gqa_step_unplanted_valid_topk(kw, units, hot):
     # wf_step's grouped filter kernel on unplanted inputs: at every scale the
     # selection must be a valid Top-K of W summed over the key head's stacked
     # query rows (near-ties allow several answers), and the output must match
-    # the oracle's grouped attention over the kernel's own indices.
+    # the oracle's grouped attention over the kernel's own indices.  With
+    # `hot`, row 0 of every unit's first query head is scaled so that its
+    # logits lie hundreds of units above the chunk's other rows: their
+    # exponentials against the chunk's largest logit flush to zero, and the
+    # filter must sum those columns against their own maxima.
     from helpers import eps_valid
     w = _workload("g1", **kw) if kw else synth.WORKLOADS["g1"]
     batch = synth.make_batch(w, planted=False, device="cuda", cfg="g1", units=units)
+    if hot:
+        Q = batch.Q.clone()
+        Q[:, ::w.group, 0, :] = (Q[:, ::w.group, 0, :].float() * hot).to(Q.dtype)
+        batch = dataclasses.replace(batch, Q=Q)
     run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().step(refresh=False)
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
