@@ -1792,8 +1792,8 @@ __host__ __device__ inline GqaLayout gqa_layout(int stages, int nch, int cs, int
   l.q = (uint32_t)stages * TILE_BYTES;
   l.sc = l.q + (uint32_t)nch * Q_BYTES;                            // Top-K scratch
   l.misc = (l.sc + (uint32_t)sizeof(SelScratch) + 127u) / 128u * 128u;
-  l.wst = (l.misc + (uint32_t)sizeof(Misc) + 15u) / 16u * 16u;     // [4][nq] float2: one warpgroup's column statistics
-  l.xst = l.wst + 4u * nq * 8u;                                    // [cs][nq] float2: every CTA's (M, S) per column
+  l.wst = (l.misc + (uint32_t)sizeof(Misc) + 15u) / 16u * 16u;     // [8][nq] float2: each warp's column statistics
+  l.xst = l.wst + 8u * nq * 8u;                                    // [cs][nq] float2: every CTA's (M, S) per column
   l.cvec = l.xst + (uint32_t)cs * nq * 8u;                         // [nq] float: the normalisers c_i
   l.buf = (l.cvec + nq * 4u + 127u) / 128u * 128u;                 // two key / selection buffers
   l.bufw = (uint32_t)((max(cmax, kmax) + 3) / 4 * 4);
@@ -1916,12 +1916,11 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
     int32_t* J = unit_J(c, p, 0, lev);
     const uint32_t keys_a = smem_u32(J);
 
-    // Pass 1: this warp's (max, sum) of each query column over its rows;
-    // lane l keeps column 32 ch + l of every chunk (a dynamically indexed,
-    // so thread-local, array).
-    float2 st[GQ_MAXCH];
-#pragma unroll
-    for (int ch = 0; ch < GQ_MAXCH; ++ch) st[ch] = make_float2(-INFINITY, 0.f);
+    // Pass 1: this warp's (stabiliser, sum) of each query column over its
+    // rows, in its own slots (lane l: column 32 ch + l of every chunk).
+    float2* wsw = wst + warp * nqp;
+#pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) wsw[32 * ch + lane] = make_float2(-INFINITY, 0.f);
 #pragma unroll 1
     for (int t = wg; t < ntl; t += 2) {
       wait_or_abort(bar_addr(ms.rdone[wg]), dpar, ms, p.status);
@@ -1956,7 +1955,7 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
           }
           ts = transpose_reduce32<false>(e, lane);
         }
-        st[ch] = merge_ms(st[ch], make_float2(tm * sl2, ts));
+        wsw[32 * ch + lane] = merge_ms(wsw[32 * ch + lane], make_float2(tm * sl2, ts));
       }
       tc_fence_before();
       __syncwarp();
@@ -1964,16 +1963,6 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
     }
     // The eight warps' statistics -> the CTA's (M, S) per column, sent to
     // every cluster CTA.
-    if (wg == 1)
-#pragma unroll 1
-      for (int ch = 0; ch < nch; ++ch) wst[qd * nqp + 32 * ch + lane] = st[ch];
-    csync<true>();
-    if (wg == 0)
-#pragma unroll 1
-      for (int ch = 0; ch < nch; ++ch) {
-        float2& w = wst[qd * nqp + 32 * ch + lane];
-        w = merge_ms(st[ch], w);
-      }
     csync<true>();
     {
       const uint32_t xbar = bar_addr(ms.xbar[0]);
@@ -1982,7 +1971,7 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
       for (int col = tid; col < nqp; col += TN) {
         float2 a = wst[col];
 #pragma unroll
-        for (int q4 = 1; q4 < 4; ++q4) a = merge_ms(a, wst[q4 * nqp + col]);
+        for (int w8 = 1; w8 < 8; ++w8) a = merge_ms(a, wst[w8 * nqp + col]);
         const uint32_t dst = smem_u32(&xst[c.rank * nqp + col]);
 #pragma unroll 1
         for (uint32_t r = 0; r < nr; ++r)

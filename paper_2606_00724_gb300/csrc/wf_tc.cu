@@ -379,6 +379,7 @@ struct TcAttnArgs {
   int nq;                     // MMA columns of a block (its query rows rounded up to 32)
   uint32_t tcols;
   int nsplit;
+  int tps;                    // key tiles of 128 a split (a CTA), taken one after the other
   float* Opart;               // [query unit][nsplit][qstride][D]
   float2* ML;                 // [query unit][nsplit][qstride]
   int qstride;
@@ -397,15 +398,16 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
   // the K rows are dead once the S^T products have completed.
   uint8_t* pb = kt;
   float* red = reinterpret_cast<float*>(sq + (a.nq / 8) * QGRP);  // [NWG][4][32]
-  float* cm = red + NWG * 4 * 32;              // [256] split max per query (log2 units)
-  float* cl = cm + 256;                        // [256] split row sums of P
-  unsigned long long* bar = reinterpret_cast<unsigned long long*>(cl + 256);  // [3]: S done, PV done, stall
+  float* cm = red + NWG * 4 * 32;              // [256] running max per query (log2 units)
+  float* cl = cm + 256;                        // [256] running row sums of P
+  float* ca = cl + 256;                        // [256] this tile's factor 2^(m_old - m_new)
+  unsigned long long* bar = reinterpret_cast<unsigned long long*>(ca + 256);  // [3]: S done, PV done, stall
   uint32_t* tbase = reinterpret_cast<uint32_t*>(bar + 3);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int wg = tid >> 7, wt = tid & 127, quarter = warp & 3;
   const int sp = blockIdx.x, u = blockIdx.y;
   const int64_t bb = u / a.H, hh = u % a.H;
-  const int total = a.k + a.ng, t0 = sp * TM;
+  const int total = a.k + a.ng;
   const int c0 = blockIdx.z * a.cb;           // first query row of this column block
   const int qb = min(a.cb, a.q - c0);         // its query rows
 
@@ -419,38 +421,9 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
     mbar_init(smem_u32(&bar[2]), 1);
     fence_mbar_init();
   }
-  // K and V rows of the split: chunk c = tid % 16 of rows r0 + 16 i
-  // (r0 = tid / 16).  Lane c resolves the K and V rows of row r0 + 16 (c % 8)
-  // (a sparse key or a generation row) and the half-warp shares the two row
-  // addresses by shuffles; the swizzle term of a thread's rows is constant.
-  {
-    constexpr int RPT = TM / (NTH / 16);
-    static_assert(RPT == 8 && (NTH / 16) % 8 == 0, "rows of a thread share r % 8");
-    const int c = tid & 15, r0 = tid >> 4, half = tid & 16;
-    const int32_t* ui = a.idx + (int64_t)u * a.k;
-    const uint32_t xs = (uint32_t)r0 * 128u + (uint32_t)(((c ^ r0) & 7) << 4);
-    const uint32_t koff = smem_u32(kt) + ((c >> 3) * HALF) + xs, voff = smem_u32(vt) + ((c >> 3) * HALF) + xs;
-    const int tl = min(t0 + r0 + (NTH / 16) * (c & (RPT - 1)), total - 1);  // keys past the list repeat its last key (P = 0 there)
-    const bf16 *kl, *vl;
-    if (tl < a.k) {
-      int row = ui[tl];
-      row = row < 0 ? 0 : (row >= a.n ? a.n - 1 : row);
-      const int64_t o = bb * a.ksb + hh * a.ksh + (int64_t)row * a.kss;
-      kl = a.K + o;
-      vl = a.V + o;
-    } else {
-      const int64_t o = bb * a.gsb + hh * a.gsh + (int64_t)(tl - a.k) * a.gss;
-      kl = a.Kg + o;
-      vl = a.Vg + o;
-    }
-    const unsigned long long ka = reinterpret_cast<unsigned long long>(kl), va = reinterpret_cast<unsigned long long>(vl);
-#pragma unroll
-    for (int i = 0; i < RPT; ++i) {
-      const unsigned long long kp = __shfl_sync(0xffffffffu, ka, half | i), vp = __shfl_sync(0xffffffffu, va, half | i);
-      const uint32_t so = (uint32_t)(NTH / 16) * 128u * i;
-      cp_async16(koff + so, reinterpret_cast<const bf16*>(kp) + c * 8);
-      cp_async16(voff + so, reinterpret_cast<const bf16*>(vp) + c * 8);
-    }
+  for (int e = tid; e < 256; e += NTH) {
+    cm[e] = -INFINITY;
+    cl[e] = 0.f;
   }
   for (int e = tid; e < a.nq * (D / 8); e += NTH) {
     const int rr = e & 7, ch = (e >> 3) & (D / 8 - 1), g = e >> 7;
@@ -465,41 +438,86 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
       sts_v4(dst, make_uint4(0, 0, 0, 0));
     }
   }
-  cp_async_wait_all();
-  fence_proxy_async();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tbase;
-  const uint32_t ocol = tmem + (uint32_t)a.nq;  // O^T columns after S^T
-  if (tid == 0) {
-    const uint32_t idesc = idesc_bf16(TM, a.nq, 0, 0);
-#pragma unroll
-    for (int h = 0; h < 2; ++h)
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk)
-        mma_bf16(tmem, smem_desc_sw128(smem_u32(kt) + h * HALF + kk * 32, 16, 1024),
-                 smem_desc(smem_u32(sq) + (4 * h + kk) * 256, 128, QGRP), idesc, (h | kk) != 0);
-    mma_commit(smem_u32(&bar[0]));
-  }
-  __syncwarp();
-  bool ok = mbar_wait_bounded(smem_u32(&bar[a.stall ? 2 : 0]), 0u, a.wait_limit);
-  if (!ok) {
-    // Drain the score MMAs (default bound) before the TMEM is freed.
-    atomicExch(a.status, 1);
-    (void)mbar_wait_bounded(smem_u32(&bar[0]), 0u, kWait);
-  }
-  ok = __syncthreads_and(ok);
-  tc_fence_after();
-
-  // Thread wt of either warpgroup owns key t0 + wt (TMEM lane wt); the two
-  // warpgroups take alternate 32-column chunks.
-  const bool valid = t0 + wt < total;
   const uint32_t qoff = (uint32_t)(quarter * 32) << 16;
   const int nch = a.nq / 32;
   float* rw = red + wg * 4 * 32;
-  if (ok) {
+  uint32_t tmem = 0, ocol = 0;
+  bool ok = true;
+  // The split's tiles of 128 sparse keys, one after the other: S^T, P with a
+  // running per-query max (a raised max rescales the partial O^T and the row
+  // sums by 2^(m_old - m_new)), O^T += V^T P^T.
+#pragma unroll 1
+  for (int j = 0; j < a.tps && ok; ++j) {
+    const int t0 = (sp * a.tps + j) * TM;
+    if (t0 >= total) break;  // the last split may hold fewer tiles
+    // K and V rows of the tile: chunk c = tid % 16 of rows r0 + 16 i
+    // (r0 = tid / 16).  Lane c resolves the K and V rows of row r0 + 16 (c % 8)
+    // (a sparse key or a generation row) and the half-warp shares the two row
+    // addresses by shuffles; the swizzle term of a thread's rows is constant.
+    {
+      constexpr int RPT = TM / (NTH / 16);
+      static_assert(RPT == 8 && (NTH / 16) % 8 == 0, "rows of a thread share r % 8");
+      const int c = tid & 15, r0 = tid >> 4, half = tid & 16;
+      const int32_t* ui = a.idx + (int64_t)u * a.k;
+      const uint32_t xs = (uint32_t)r0 * 128u + (uint32_t)(((c ^ r0) & 7) << 4);
+      const uint32_t koff = smem_u32(kt) + ((c >> 3) * HALF) + xs, voff = smem_u32(vt) + ((c >> 3) * HALF) + xs;
+      const int tl = min(t0 + r0 + (NTH / 16) * (c & (RPT - 1)), total - 1);  // keys past the list repeat its last key (P = 0 there)
+      const bf16 *kl, *vl;
+      if (tl < a.k) {
+        int row = ui[tl];
+        row = row < 0 ? 0 : (row >= a.n ? a.n - 1 : row);
+        const int64_t o = bb * a.ksb + hh * a.ksh + (int64_t)row * a.kss;
+        kl = a.K + o;
+        vl = a.V + o;
+      } else {
+        const int64_t o = bb * a.gsb + hh * a.gsh + (int64_t)(tl - a.k) * a.gss;
+        kl = a.Kg + o;
+        vl = a.Vg + o;
+      }
+      const unsigned long long ka = reinterpret_cast<unsigned long long>(kl),
+                               va = reinterpret_cast<unsigned long long>(vl);
+#pragma unroll
+      for (int i = 0; i < RPT; ++i) {
+        const unsigned long long kp = __shfl_sync(0xffffffffu, ka, half | i), vp = __shfl_sync(0xffffffffu, va, half | i);
+        const uint32_t so = (uint32_t)(NTH / 16) * 128u * i;
+        cp_async16(koff + so, reinterpret_cast<const bf16*>(kp) + c * 8);
+        cp_async16(voff + so, reinterpret_cast<const bf16*>(vp) + c * 8);
+      }
+    }
+    cp_async_wait_all();
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    tmem = *tbase;
+    ocol = tmem + (uint32_t)a.nq;  // O^T columns after S^T
+    const uint32_t ph = (uint32_t)j & 1u;
+    if (tid == 0) {
+      const uint32_t idesc = idesc_bf16(TM, a.nq, 0, 0);
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_bf16(tmem, smem_desc_sw128(smem_u32(kt) + h * HALF + kk * 32, 16, 1024),
+                   smem_desc(smem_u32(sq) + (4 * h + kk) * 256, 128, QGRP), idesc, (h | kk) != 0);
+      mma_commit(smem_u32(&bar[0]));
+    }
+    __syncwarp();
+    bool sok = mbar_wait_bounded(smem_u32(&bar[(a.stall && j == 0) ? 2 : 0]), ph, a.wait_limit);
+    if (!sok) {
+      // Drain the score MMAs (default bound) before the TMEM is freed.
+      atomicExch(a.status, 1);
+      (void)mbar_wait_bounded(smem_u32(&bar[0]), ph, kWait);
+    }
+    ok = __syncthreads_and(sok);
+    tc_fence_after();
+    if (!ok) break;
+
+    // Thread wt of either warpgroup owns key t0 + wt (TMEM lane wt); the two
+    // warpgroups take alternate 32-column chunks.
+    const bool valid = t0 + wt < total;
     uint8_t* prow = pb + (wt >> 3) * (a.nq * 16) + (wt & 7) * 16;
+    bool raised = false;
 #pragma unroll 1
     for (int ch = wg; ch < nch; ch += NWG) {
       float v[32], w[32];
@@ -511,8 +529,14 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
       }
       rw[quarter * 32 + lane] = xpose_reduce32<true>(w, lane);
       wg_sync(wg);
-      if (wt < 32) cm[ch * 32 + wt] = fmaxf(fmaxf(rw[wt], rw[32 + wt]), fmaxf(rw[64 + wt], rw[96 + wt]));
+      if (wt < 32) {
+        const float mo = cm[ch * 32 + wt];
+        const float mn = fmaxf(mo, fmaxf(fmaxf(rw[wt], rw[32 + wt]), fmaxf(rw[64 + wt], rw[96 + wt])));
+        ca[ch * 32 + wt] = mo == mn ? 1.f : ex2(mo - mn);  // mo = -inf: nothing accumulated yet
+        cm[ch * 32 + wt] = mn;
+      }
       wg_sync(wg);
+      raised |= j > 0;
       uint32_t pk[16];
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
@@ -529,8 +553,18 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
             make_uint4(pk[4 * c4], pk[4 * c4 + 1], pk[4 * c4 + 2], pk[4 * c4 + 3]);
       rw[quarter * 32 + lane] = xpose_reduce32<false>(w, lane);
       wg_sync(wg);
-      if (wt < 32) cl[ch * 32 + wt] = (rw[wt] + rw[32 + wt]) + (rw[64 + wt] + rw[96 + wt]);
+      if (wt < 32) cl[ch * 32 + wt] = cl[ch * 32 + wt] * ca[ch * 32 + wt] + ((rw[wt] + rw[32 + wt]) + (rw[64 + wt] + rw[96 + wt]));
       wg_sync(wg);
+      if (raised) {
+        // The partial O^T of the tiles before (every PV product of them is
+        // done) takes the columns' factors.
+        float o[32];
+        tmem_ld32(ocol + qoff + 32 * ch, o);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[i] *= ca[ch * 32 + i];
+        tmem_st32(ocol + qoff + 32 * ch, reinterpret_cast<const uint32_t*>(o));
+        tmem_wait_st();
+      }
     }
     fence_proxy_async();
     tc_fence_before();
@@ -541,49 +575,49 @@ __global__ void __launch_bounds__(NTH) tc_attn_kernel(const __grid_constant__ Tc
 #pragma unroll
       for (int kq = 0; kq < TM / 16; ++kq)
         mma_bf16(ocol, smem_desc_sw128(smem_u32(vt) + kq * 2048, HALF, 1024),
-                 smem_desc(smem_u32(pb) + kq * 2 * (a.nq * 16), a.nq * 16, 128), idesc, kq > 0 ? 1u : 0u);
+                 smem_desc(smem_u32(pb) + kq * 2 * (a.nq * 16), a.nq * 16, 128), idesc, (j > 0 || kq > 0) ? 1u : 0u);
       mma_commit(smem_u32(&bar[1]));
     }
     __syncwarp();
-    bool ok2 = mbar_wait_bounded(smem_u32(&bar[1]), 0u, a.wait_limit);
-    if (!ok2) {
+    bool pok = mbar_wait_bounded(smem_u32(&bar[1]), ph, a.wait_limit);
+    if (!pok) {
       atomicExch(a.status, 1);
-      (void)mbar_wait_bounded(smem_u32(&bar[1]), 0u, kWait);
+      (void)mbar_wait_bounded(smem_u32(&bar[1]), ph, kWait);
     }
-    ok2 = __syncthreads_and(ok2);
+    ok = __syncthreads_and(pok);
     tc_fence_after();
-    if (ok2) {
-      // Thread wt holds head-dim row wt of O^T: its warpgroup's query chunks.
-      const float ln2 = 0.69314718055994531f;
+  }
+  if (ok) {  // every split holds at least one tile, so the loop ran
+    // Thread wt holds head-dim row wt of O^T: its warpgroup's query chunks.
+    const float ln2 = 0.69314718055994531f;
 #pragma unroll 1
-      for (int ch = wg; ch < nch; ch += NWG) {
-        float o[32];
-        tmem_ld32(ocol + qoff + 32 * ch, o);
+    for (int ch = wg; ch < nch; ch += NWG) {
+      float o[32];
+      tmem_ld32(ocol + qoff + 32 * ch, o);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int cl_ = ch * 32 + i;  // column within the block
-          if (cl_ < qb) {
-            const int colq = c0 + cl_;
-            const int hq = head_of(colq, a.rqs);
-            const int64_t uq = bb * (a.H * a.G) + hh * a.G + hq;
-            const int iq = colq - hq * a.qs;
-            a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + wt] = o[i];
-          }
+      for (int i = 0; i < 32; ++i) {
+        const int cl_ = ch * 32 + i;  // column within the block
+        if (cl_ < qb) {
+          const int colq = c0 + cl_;
+          const int hq = head_of(colq, a.rqs);
+          const int64_t uq = bb * (a.H * a.G) + hh * a.G + hq;
+          const int iq = colq - hq * a.qs;
+          a.Opart[(((int64_t)uq * a.nsplit + sp) * a.qstride + iq) * D + wt] = o[i];
         }
       }
-      for (int cl_ = tid; cl_ < qb; cl_ += NTH) {
-        const int colq = c0 + cl_;
-        const int hq = head_of(colq, a.rqs);
-        const int64_t uq = bb * (a.H * a.G) + hh * a.G + hq;
-        a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq - hq * a.qs] = make_float2(cm[cl_] * ln2, cl[cl_]);
-      }
+    }
+    for (int cl_ = tid; cl_ < qb; cl_ += NTH) {
+      const int colq = c0 + cl_;
+      const int hq = head_of(colq, a.rqs);
+      const int64_t uq = bb * (a.H * a.G) + hh * a.G + hq;
+      a.ML[((int64_t)uq * a.nsplit + sp) * a.qstride + colq - hq * a.qs] = make_float2(cm[cl_] * ln2, cl[cl_]);
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, a.tcols);
+    tmem_dealloc(*tbase, a.tcols);
   }
 }
 
@@ -618,7 +652,16 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   uint32_t cols = 32;
   while ((int)cols < 2 * a.nq) cols *= 2;
   a.tcols = cols;
-  a.nsplit = (p.k + p.ng + TM - 1) / TM;
+  // Splits of several key tiles when the grid would otherwise exceed about
+  // two CTAs an SM (a CTA keeps a running max across its tiles): fewer
+  // partials to write and fold.
+  const int tiles = (p.k + p.ng + TM - 1) / TM;
+  int sms = 148, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) (void)cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t ctas_per_split = (int64_t)kv.batch * kv.heads * nblk;
+  a.tps = 1;
+  while (a.tps < tiles && ctas_per_split * ((tiles + a.tps - 1) / a.tps) > 2 * sms) ++a.tps;
+  a.nsplit = (tiles + a.tps - 1) / a.tps;
   a.Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
   a.ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
   a.qstride = p.qstride;
@@ -627,7 +670,7 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   const WaitControls wc = wait_controls();
   a.wait_limit = wc.limit;
   a.stall = wc.stall;
-  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 512) + 32;
+  size_t smem = 4 * HALF + (size_t)(a.nq / 8) * QGRP + sizeof(float) * (NWG * 4 * 32 + 768) + 32;
   const size_t per_sm = 228 * 1024;
   const size_t cap = 512 / cols;
   const size_t floor_smem = per_sm / (cap + 1) + 1;
