@@ -1838,8 +1838,11 @@ __device__ void gqa_producer_role(const Ctx& c, const FusedParams& p) {
     const RowSrc src = scale_src(c, p, 0, lev, g0, mc);
     produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, src, pt);  // pass 1
     it += ntl;
-    produce<S>(ms, p.status, smem_u32(c.smem), it, 0, ntl, src, pt);  // pass 2: the same rows again
-    it += ntl;
+    // Pass 2: the same rows again, but for the last two tiles, which stay in
+    // TMEM from pass 1.
+    const int nre = max(ntl - 2, 0);
+    produce<S>(ms, p.status, smem_u32(c.smem), it, 0, nre, src, pt);
+    it += nre;
   }
   cp_async_wait_all();
 }
@@ -1861,8 +1864,12 @@ __device__ void gqa_mma_role(const Ctx& c, const FusedParams& p) {
     int g0, mc;
     scale_slice(m_total(p, lev), c.rank, c.cs, g0, mc);
     const int ntl = tiles_of(mc);
+    // Pass 1: every tile; pass 2: all but the last two, whose logits are
+    // still in their regions (each issue into a region is released once by
+    // the warpgroup reading it, the kept tiles after their second reading).
+    const int nre = max(ntl - 2, 0);
 #pragma unroll 1
-    for (int k = 0; k < 2 * ntl; ++k) {
+    for (int k = 0; k < ntl + nre; ++k) {
       const int t = k < ntl ? k : k - ntl, r = t & 1, slot = it + k, s = slot % S;
       if (used[r] > 0) wait_or_abort(bar_addr(ms.rfree[r]), (used[r] - 1u) & 1u, ms, p.status);
       ++used[r];
@@ -1883,7 +1890,7 @@ __device__ void gqa_mma_role(const Ctx& c, const FusedParams& p) {
       mma_commit(bar_addr(ms.empty[s]));
       mma_commit(bar_addr(ms.rdone[r]));
     }
-    it += 2 * ntl;
+    it += ntl + nre;
   }
   mma_commit(bar_addr(ms.drainbar));
   (void)mbar_wait_bounded(bar_addr(ms.drainbar), 0u, kDefaultWaitLimit);
@@ -1899,12 +1906,22 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
   const uint32_t sc_a = smem_u32(c.smem + gl.sc);
   float2* wst = reinterpret_cast<float2*>(c.smem + gl.wst);
   float2* xst = reinterpret_cast<float2*>(c.smem + gl.xst);
-  float* cvec = reinterpret_cast<float*>(c.smem + gl.cvec);
-  const uint32_t cvec_a = smem_u32(cvec);
+  float* cvec = reinterpret_cast<float*>(c.smem + gl.cvec);  // -c_i
+  const uint32_t ncvec_a = smem_u32(cvec);
   const float sl2 = p.scale_log2;
   const int u = c.u0;
   int64_t sets_off = 0;
   uint32_t dpar = 0;  // parity of the next phase of this warpgroup's rdone barrier
+  // body(ra, ch) for every query chunk of the tile in the region.
+  auto for_chunks = [&](auto&& body) {
+#pragma unroll 1
+    for (int ch = 0; ch < nch; ++ch) {
+      uint32_t ra[32];
+      tmem_ld32_issue(treg + 32u * ch + lane_base, ra);
+      tmem_wait_ld();
+      body(ra, ch);
+    }
+  };
 #pragma unroll 1
   for (int lev = c.lev_top; lev >= c.lev_end; --lev) {
     const uint32_t ph = (uint32_t)(c.lev_top - lev) & 1u;
@@ -1921,17 +1938,15 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
     float2* wsw = wst + warp * nqp;
 #pragma unroll 1
     for (int ch = 0; ch < nch; ++ch) wsw[32 * ch + lane] = make_float2(-INFINITY, 0.f);
+    // This warpgroup's last tile stays in its region for pass 2.
+    const int tkeep = ntl - 1 - wg >= 0 ? wg + (ntl - 1 - wg) / 2 * 2 : -1;
 #pragma unroll 1
     for (int t = wg; t < ntl; t += 2) {
       wait_or_abort(bar_addr(ms.rdone[wg]), dpar, ms, p.status);
       dpar ^= 1u;
       tc_fence_after();
       const bool valid = t * TM + row < mc;
-#pragma unroll 1
-      for (int ch = 0; ch < nch; ++ch) {
-        uint32_t ra[32];
-        tmem_ld32_issue(treg + 32u * ch + lane_base, ra);
-        tmem_wait_ld();
+      for_chunks([&](const uint32_t (&ra)[32], int ch) {
         // Exponentials relative to the chunk's largest logit among the warp's
         // rows (one warp-wide max), summed per column across the rows.
         float e[32];
@@ -1939,8 +1954,9 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
 #pragma unroll
         for (int i = 0; i < 32; i += 2) vm = fmax3(vm, __uint_as_float(ra[i]), __uint_as_float(ra[i + 1]));
         float tm = warp_max_f32(valid ? vm : -INFINITY);
+        const float ntm = -tm * sl2;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) e[i] = valid ? ex2((__uint_as_float(ra[i]) - tm) * sl2) : 0.f;
+        for (int i = 0; i < 32; ++i) e[i] = valid ? ex2(fmaf(__uint_as_float(ra[i]), sl2, ntm)) : 0.f;
         float ts = transpose_reduce32<false>(e, lane);  // lane l: column l's sum
         // A column whose every term flushed to zero (logits more than ~126
         // below the chunk's largest, in log2 units) is summed again against
@@ -1956,10 +1972,10 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
           ts = transpose_reduce32<false>(e, lane);
         }
         wsw[32 * ch + lane] = merge_ms(wsw[32 * ch + lane], make_float2(tm * sl2, ts));
-      }
+      });
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar_addr(ms.rfree[wg]));
+      if (lane == 0 && t != tkeep) mbar_arrive(bar_addr(ms.rfree[wg]));
     }
     // The eight warps' statistics -> the CTA's (M, S) per column, sent to
     // every cluster CTA.
@@ -1986,7 +2002,7 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
       float2 a = make_float2(-INFINITY, 0.f);
 #pragma unroll 1
       for (uint32_t r = 0; r < c.cs; ++r) a = merge_ms(a, xst[r * nqp + col]);
-      cvec[col] = col < nq ? a.x + lg2(a.y) : INFINITY;  // padded rows weigh 0
+      cvec[col] = col < nq ? -(a.x + lg2(a.y)) : -INFINITY;  // -c_i; padded rows weigh 0
     }
     csync<true>();
 
@@ -1994,36 +2010,60 @@ __device__ void gqa_compute_role(const Ctx& c, const FusedParams& p, const GqaLa
     float kmin = INFINITY, kmax = -INFINITY;
     const uint32_t kbar = bar_addr(ms.kbar[0]);
     const uint32_t nr = aborted(ms) ? 0u : c.cs;
+    // The kept tile first (its logits are in the region), then the earlier
+    // tiles as the MMA thread re-issues them.
 #pragma unroll 1
-    for (int t = wg; t < ntl; t += 2) {
-      wait_or_abort(bar_addr(ms.rdone[wg]), dpar, ms, p.status);
-      dpar ^= 1u;
-      tc_fence_after();
-      float rm = -INFINITY, rs = 0.f;
-#pragma unroll 1
-      for (int ch = 0; ch < nch; ++ch) {
-        uint32_t ra[32];
-        tmem_ld32_issue(treg + 32u * ch + lane_base, ra);
-        tmem_wait_ld();
-        float x[32];
-        float mx = -INFINITY;
-#pragma unroll
-        for (int k4 = 0; k4 < 8; ++k4) {
-          const uint4 cv = lds_v4(cvec_a + 16u * (uint32_t)(8 * ch + k4));
-          x[4 * k4] = __uint_as_float(ra[4 * k4]) * sl2 - __uint_as_float(cv.x);
-          x[4 * k4 + 1] = __uint_as_float(ra[4 * k4 + 1]) * sl2 - __uint_as_float(cv.y);
-          x[4 * k4 + 2] = __uint_as_float(ra[4 * k4 + 2]) * sl2 - __uint_as_float(cv.z);
-          x[4 * k4 + 3] = __uint_as_float(ra[4 * k4 + 3]) * sl2 - __uint_as_float(cv.w);
-          mx = fmaxf(mx, fmax3(x[4 * k4], x[4 * k4 + 1], fmaxf(x[4 * k4 + 2], x[4 * k4 + 3])));
-        }
-        if (mx > rm) {
-          rs = rm == -INFINITY ? 0.f : rs * ex2(rm - mx);
-          rm = mx;
-        }
+    for (int k = 0; tkeep >= 0 && k <= tkeep / 2; ++k) {
+      const int t = k == 0 ? tkeep : wg + 2 * (k - 1);
+      if (k > 0) {
+        wait_or_abort(bar_addr(ms.rdone[wg]), dpar, ms, p.status);
+        dpar ^= 1u;
+        tc_fence_after();
+      }
+      // Every exponent l sl2 - c_i is at most 0 (c_i is the log of a sum that
+      // holds the row's own term), so the sum is taken unshifted; a row whose
+      // sum is tiny (below 2^-96, where flushed terms could matter) is taken
+      // again shifted by its largest exponent (the warp together).
+      float rm = 0.f, rs = 0.f;
+      for_chunks([&](const uint32_t (&ra)[32], int ch) {
         float z = 0.f;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) z += ex2(x[i] - rm);
+        for (int k4 = 0; k4 < 8; ++k4) {
+          const uint4 cv = lds_v4(ncvec_a + 16u * (uint32_t)(8 * ch + k4));
+          z += ex2(fmaf(__uint_as_float(ra[4 * k4]), sl2, __uint_as_float(cv.x)));
+          z += ex2(fmaf(__uint_as_float(ra[4 * k4 + 1]), sl2, __uint_as_float(cv.y)));
+          z += ex2(fmaf(__uint_as_float(ra[4 * k4 + 2]), sl2, __uint_as_float(cv.z)));
+          z += ex2(fmaf(__uint_as_float(ra[4 * k4 + 3]), sl2, __uint_as_float(cv.w)));
+        }
         rs += z;
+      });
+      if (__any_sync(0xffffffffu, rs < 0x1p-96f && t * TM + row < mc)) {
+        float mxr = -INFINITY;
+        for_chunks([&](const uint32_t (&ra)[32], int ch) {
+#pragma unroll
+          for (int k4 = 0; k4 < 8; ++k4) {
+            const uint4 cv = lds_v4(ncvec_a + 16u * (uint32_t)(8 * ch + k4));
+            mxr = fmaxf(mxr, fmax3(fmaf(__uint_as_float(ra[4 * k4]), sl2, __uint_as_float(cv.x)),
+                                   fmaf(__uint_as_float(ra[4 * k4 + 1]), sl2, __uint_as_float(cv.y)),
+                                   fmaxf(fmaf(__uint_as_float(ra[4 * k4 + 2]), sl2, __uint_as_float(cv.z)),
+                                         fmaf(__uint_as_float(ra[4 * k4 + 3]), sl2, __uint_as_float(cv.w)))));
+          }
+        });
+        float z2 = 0.f;
+        for_chunks([&](const uint32_t (&ra)[32], int ch) {
+#pragma unroll
+          for (int k4 = 0; k4 < 8; ++k4) {
+            const uint4 cv = lds_v4(ncvec_a + 16u * (uint32_t)(8 * ch + k4));
+            z2 += ex2(fmaf(__uint_as_float(ra[4 * k4]), sl2, __uint_as_float(cv.x)) - mxr);
+            z2 += ex2(fmaf(__uint_as_float(ra[4 * k4 + 1]), sl2, __uint_as_float(cv.y)) - mxr);
+            z2 += ex2(fmaf(__uint_as_float(ra[4 * k4 + 2]), sl2, __uint_as_float(cv.z)) - mxr);
+            z2 += ex2(fmaf(__uint_as_float(ra[4 * k4 + 3]), sl2, __uint_as_float(cv.w)) - mxr);
+          }
+        });
+        if (rs < 0x1p-96f) {
+          rm = mxr;
+          rs = z2;
+        }
       }
       tc_fence_before();
       __syncwarp();

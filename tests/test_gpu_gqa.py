@@ -103,12 +103,13 @@ def test_gqa_attention_equals_repeated_key_heads():
     assert torch.equal(O1, grouped.O)
 
 
-@pytest.mark.parametrize("kw,units,hot", [
-    (dict(), [0, 17, 31], 0.0),                                    # the Dream-shaped layer: clusters of 4, 4 tiles a scale
-    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 0.0),  # clusters of 8, one tile a scale, level-0 trim
-    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 80.0),  # one query row 80x: other rows' terms flush
+@pytest.mark.parametrize("kw,units,hot,cold", [
+    (dict(), [0, 17, 31], 0.0, False),                                    # the Dream-shaped layer: clusters of 4, 4 tiles a scale
+    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 0.0, False),  # clusters of 8, one tile a scale, level-0 trim
+    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 80.0, False),  # one query row 80x: other rows' terms flush
+    (dict(batch=1, heads=4, n=8192, levels=3, k=819), [0, 3], 0.0, True),   # key rows far below every query: tiny W
 ])
-def test_gqa_step_unplanted_valid_topk(kw, units, hot):
+def test_gqa_step_unplanted_valid_topk(kw, units, hot, cold):
     # wf_step's grouped filter kernel on unplanted inputs: at every scale the
     # selection must be a valid Top-K of W summed over the key head's stacked
     # query rows (near-ties allow several answers), and the output must match
@@ -116,7 +117,8 @@ def test_gqa_step_unplanted_valid_topk(kw, units, hot):
     # `hot`, row 0 of every unit's first query head is scaled so that its
     # logits lie hundreds of units above the chunk's other rows: their
     # exponentials against the chunk's largest logit flush to zero, and the
-    # filter must sum those columns against their own maxima.
+    # filter must sum those columns against their own maxima.  With `cold`,
+    # some candidates' W are tiny and their keys are taken shifted.
     from helpers import eps_valid
     w = _workload("g1", **kw) if kw else synth.WORKLOADS["g1"]
     batch = synth.make_batch(w, planted=False, device="cuda", cfg="g1", units=units)
@@ -124,6 +126,18 @@ def test_gqa_step_unplanted_valid_topk(kw, units, hot):
         Q = batch.Q.clone()
         Q[:, ::w.group, 0, :] = (Q[:, ::w.group, 0, :].float() * hot).to(Q.dtype)
         batch = dataclasses.replace(batch, Q=Q)
+    if cold:
+        # Every query row of a unit gets a component of 6 along one direction
+        # u; 256 key tokens point along -u with logits near -80 for every
+        # query row, so their candidates' W lie far below 2^-96.
+        g = torch.Generator(device="cpu").manual_seed(5)
+        u = torch.randn(w.batch, w.heads, w.head_dim, generator=g, dtype=torch.float64)
+        u = (u / u.norm(dim=-1, keepdim=True)).cuda()
+        ug = u.repeat_interleave(w.group, dim=1)
+        Q = (batch.Q.double() + 6.0 * ug[:, :, None, :]).to(batch.Q.dtype)
+        K = batch.K.clone()
+        K[:, :, 2048:2304, :] = (-(80.0 / 6.0) * 128 ** 0.5 * u[:, :, None, :]).to(K.dtype)
+        batch = dataclasses.replace(batch, Q=Q, K=K)
     run = LibRun(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, w.levels, w.keep).dwt().step(refresh=False)
     wf.wf_workspace_status(run.ws_step)
     torch.cuda.synchronize()
