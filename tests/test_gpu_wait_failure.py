@@ -118,3 +118,45 @@ def test_tensor_core_attention_wait_gives_up_then_recovers():
         ref = oracle.sparse_attn(Q, K, V, idx_list[u].cpu().numpy(), Kg, Vg)
         assert_close_out(f64(O[b, h]), ref, torch.bfloat16)
 
+
+
+def test_grouped_filter_wait_gives_up_then_recovers():
+    # wf_step on grouped query heads (the grouped filter kernel, then the
+    # tensor-core attention) under the same stalled first wait: the status
+    # word reports WF_ERR_TIMEOUT, nothing is written outside idx and O, and
+    # the next normal call matches the oracle.
+    n, levels, k = 4096, 3, 512
+    w = dataclasses.replace(synth.WORKLOADS["g1"], name="wait_failure_gqa", batch=1, heads=2, n=n, levels=levels,
+                            keep=tuple(int(x) for x in oracle.default_schedule(n, levels, k)))
+    b = synth.make_batch(w, planted=True, device="cpu", cfg="g1")
+    batch = dataclasses.replace(b, Q=b.Q.cuda(), K=b.K.cuda(), V=b.V.cuda(), Kg=b.Kg.cuda(), Vg=b.Vg.cuda())
+    keep = list(w.keep)
+    G = w.group
+    coeffs = torch.empty(wf.wf_coeffs_bytes(batch.K, w.levels), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(wf.wf_step_workspace_bytes(batch.Q, batch.K, w.levels, keep, w.ng), dtype=torch.uint8,
+                     device="cuda")
+    O_full, O = _guarded_out(batch.Q)
+    idx_full, idx = _guarded_idx(w.units, w.k, "cuda")
+    wf.wf_dwt_build(batch.K, w.levels, coeffs)
+    try:
+        wf.wf_testing_set_wait_failure(True, 100_000)
+        wf.wf_step(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, coeffs, False, w.levels, keep, idx, O, ws)
+        with pytest.raises(wf.WfError) as ei:
+            wf.wf_workspace_status(ws)
+        assert ei.value.status == WF_ERR_TIMEOUT
+    finally:
+        wf.wf_testing_set_wait_failure(False, 0)
+    torch.cuda.synchronize()
+    _guards_intact(O_full, idx_full)
+    wf.wf_step(batch.Q, batch.K, batch.V, batch.Kg, batch.Vg, coeffs, False, w.levels, keep, idx, O, ws)
+    wf.wf_workspace_status(ws)
+    torch.cuda.synchronize()
+    _guards_intact(O_full, idx_full)
+    for u in range(w.units):
+        bb, h = divmod(u, w.heads)
+        Qh = f64(batch.Q[bb, h * G:(h + 1) * G])
+        K, V, Kg, Vg = (f64(t[bb, h]) for t in (batch.K, batch.V, batch.Kg, batch.Vg))
+        pyr = oracle.haar_pyramid_spec32(K.astype(np.float32), w.levels, True)
+        mu0 = oracle.filter_gqa(Qh, pyr, K, w.n, w.levels, np.array(w.keep))
+        assert np.array_equal(idx[u].cpu().numpy(), mu0), f"unit {u}"
+        assert_close_out(f64(O[bb, h * G:(h + 1) * G]), oracle.sparse_attn_gqa(Qh, K, V, mu0, Kg, Vg), torch.bfloat16)
