@@ -242,15 +242,17 @@ __device__ __forceinline__ int m_total(const FusedParams& p, int lev) {
 // together).
 __device__ __forceinline__ void scale_slice(int m, uint32_t rank, uint32_t cs, int& g0, int& mc) {
   const int pairs = (m + 1) >> 1;
-  g0 = min(m, 2 * (int)((int64_t)rank * pairs / cs));
-  const int g1 = min(m, 2 * (int)((int64_t)(rank + 1) * pairs / cs));
+  // 32-bit arithmetic: rank <= 8 and pairs <= 2^16 (a 64-bit division is a
+  // called routine on the path between two scales).
+  g0 = min(m, 2 * (int)(rank * (uint32_t)pairs / cs));
+  const int g1 = min(m, 2 * (int)((rank + 1u) * (uint32_t)pairs / cs));
   mc = g1 - g0;
 }
 
 // This CTA's slice of the sparse key list of `total` rows.
 __device__ __forceinline__ void attn_slice(int total, uint32_t rank, uint32_t cs, int& a0, int& mc) {
-  a0 = (int)((int64_t)rank * total / cs);
-  mc = (int)((int64_t)(rank + 1) * total / cs) - a0;
+  a0 = (int)(rank * (uint32_t)total / cs);
+  mc = (int)((rank + 1u) * (uint32_t)total / cs) - a0;
 }
 
 __device__ __forceinline__ int tiles_of(int mc) { return (mc + TM - 1) / TM; }
