@@ -305,8 +305,11 @@ wf_status wf_noalloc_status(void* stream);
  *
  * For bf16 with head_dim 128, at most 32 query rows and one query head per
  * key head, the filter and the attention run as one fused kernel (one
- * thread-block cluster per (batch, head)); other shapes, grouped query
- * heads included, run the per-stage kernels.  The fused kernel's waits
+ * thread-block cluster per (batch, head)).  Grouped query heads with bf16,
+ * head_dim 128, at most 32 rows a query head and at most 256 stacked rows a
+ * key head run the grouped filter kernel (one cluster per (batch, key head),
+ * the stacked rows as the MMA columns), then the tensor-core attention.
+ * Other shapes run the per-stage kernels.  The fused kernels' waits
  * (on copies, tensor-core completion and the cluster's exchanges) are
  * bounded: if one gives up (it never should), the kernel returns early,
  * outputs are undefined, and a status word in the first 4 bytes of ws is set;
