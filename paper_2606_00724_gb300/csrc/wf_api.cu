@@ -4,6 +4,9 @@
 #include <string.h>
 
 #include <atomic>
+#include <map>
+#include <mutex>
+#include <utility>
 
 #include "wf_internal.cuh"
 #include "wf_testing.h"
@@ -64,12 +67,47 @@ wf_status cuda_status(cudaError_t e) { return e == cudaSuccess ? WF_OK : WF_ERR_
 
 // Number of SMs of the current device.
 bool device_sms(int* sms) {
-  int dev = 0;
-  return cudaGetDevice(&dev) == cudaSuccess &&
-         cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
+  *sms = wf::sm_count();
+  return *sms > 0;
 }
 
 int64_t ceil_guarded(double v) { return (int64_t)ceil(v - 1e-9); }
+
+}  // namespace
+
+namespace wf {
+
+cudaError_t raise_smem_limit(const void* kernel, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::pair<int, const void*>, size_t> raised;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  size_t& cur = raised[std::make_pair(dev, kernel)];
+  if (cur >= smem) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) cur = smem;
+  return e;
+}
+
+int sm_count() {
+  static std::mutex mu;
+  static std::map<int, int> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(dev);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) n = 0;
+  cache.emplace(dev, n);
+  return n;
+}
+
+}  // namespace wf
+
+namespace {
 
 wf_status check_filter_args(const wf_tensor* q, const wf_tensor* kv, int levels, const int32_t* keep) {
   wf_status st;

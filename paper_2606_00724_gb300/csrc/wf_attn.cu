@@ -204,8 +204,7 @@ cudaError_t run(const AttnPlan& p, const void* Q, const wf_tensor& qd, const voi
   float* Opart = reinterpret_cast<float*>(static_cast<char*>(ws) + p.off_o);
   float2* ML = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.off_ml);
   const size_t smem = sizeof(float) * (size_t)(QM * D + CH * (D + 4) + CH * D + QM * (CH + 1));
-  cudaError_t e = cudaFuncSetAttribute(attn_split_kernel<T, D, QM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(attn_split_kernel<T, D, QM>), smem);
   if (e != cudaSuccess) return e;
   const int64_t gsb = g ? g->stride_b : 0, gsh = g ? g->stride_h : 0, gss = g ? g->stride_s : 0;
   attn_split_kernel<T, D, QM><<<dim3(p.nsplit, p.U), 256, smem, s>>>(

@@ -310,7 +310,7 @@ template <typename T, int D, int QM>
 cudaError_t run_score_q(const FilterPlan& p, const void* Q, const wf_tensor& qd, RowSrc src, const int32_t* cand,
                         int m, float* logits, float2* part, cudaStream_t s) {
   const size_t smem = sizeof(float) * (size_t)(QM * D + TILE * (D + 4));
-  cudaError_t e = cudaFuncSetAttribute(score_kernel<T, D, QM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(score_kernel<T, D, QM>), smem);
   if (e != cudaSuccess) return e;
   dim3 grid((m + TILE - 1) / TILE, p.U, (p.q + QM - 1) / QM);
   score_kernel<T, D, QM><<<grid, 256, smem, s>>>(static_cast<const T*>(Q), qd.stride_b, qd.stride_h, qd.stride_s, p.q,

@@ -197,6 +197,13 @@ cudaError_t launch_gqa_filter(const GqaPlan& gp, const void* Q, const wf_tensor&
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// A kernel's dynamic shared-memory limit, raised once per device and kernel
+// to the largest size requested so far (otherwise a host call on every
+// launch).
+cudaError_t raise_smem_limit(const void* kernel, size_t smem);
+// The current device's SM count, looked up once per device (0 on an error).
+int sm_count();
+
 // Bounds of the tensor-core kernels' waits.  The default, about one second of
 // SM clock cycles, can be lowered (and a stalled first wait requested) only
 // through the test-only wf_testing_set_wait_failure.

@@ -329,9 +329,9 @@ cudaError_t launch_tc_skim(const FilterPlan& p, const void* Q, const wf_tensor& 
   const size_t floor_smem = per_sm / (cap + 1) + 1;
   if (cap < (size_t)(2048 / NTH) && smem < floor_smem) smem = floor_smem;
   const dim3 grid((unsigned)((m + TM - 1) / TM), (unsigned)p.U);
-  cudaError_t e = cudaFuncSetAttribute(tc_score_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(tc_score_kernel<0>), smem);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_score_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    e = raise_smem_limit(reinterpret_cast<const void*>(tc_score_kernel<1>), smem);
   if (e != cudaSuccess) return e;
   tc_score_kernel<0><<<grid, NTH, smem, s>>>(a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -656,8 +656,8 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   // two CTAs an SM (a CTA keeps a running max across its tiles): fewer
   // partials to write and fold.
   const int tiles = (p.k + p.ng + TM - 1) / TM;
-  int sms = 148, dev = 0;
-  if (cudaGetDevice(&dev) == cudaSuccess) (void)cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int sms = sm_count();
+  if (sms <= 0) sms = 148;
   const int64_t ctas_per_split = (int64_t)kv.batch * kv.heads * nblk;
   a.tps = 1;
   while (a.tps < tiles && ctas_per_split * ((tiles + a.tps - 1) / a.tps) > 2 * sms) ++a.tps;
@@ -675,7 +675,7 @@ cudaError_t launch_tc_attn(const AttnPlan& p, const void* Q, const wf_tensor& qd
   const size_t cap = 512 / cols;
   const size_t floor_smem = per_sm / (cap + 1) + 1;
   if (cap < (size_t)(2048 / NTH) && smem < floor_smem) smem = floor_smem;
-  cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(tc_attn_kernel), smem);
   if (e != cudaSuccess) return e;
   tc_attn_kernel<<<dim3((unsigned)a.nsplit, (unsigned)(kv.batch * kv.heads), (unsigned)nblk), NTH, smem, s>>>(a);
   *nsplit_out = a.nsplit;
