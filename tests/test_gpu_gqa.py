@@ -158,3 +158,46 @@ def test_gqa_step_unplanted_valid_topk(kw, units, hot, cold):
         assert np.array_equal(idx, gsets[0])
         O = oracle.sparse_attn_gqa(Qh, K, V, idx, Kg, Vg)
         assert_close_out(f64(run.O[b, h * G:(h + 1) * G]), O, torch.bfloat16)
+
+
+def test_gqa_attention_raised_stabiliser():
+    # The attention with the query rows on the TMEM lanes raises a row's
+    # stabiliser only when a tile's max exceeds it by more than 8 (log2
+    # units), and then rescales the partial O and row sum.  16 key units of
+    # 17 key tiles give CTAs of two consecutive tiles; every query row has a
+    # component of 4 along one direction u, and the keys of the odd tiles
+    # get one along u too, so that an odd tile's max lies about 5 (tiles
+    # 1, 5, 9, 13: the stabiliser is kept, P up to 2^5) or about 20 (tiles
+    # 3, 7, 11, 15: raised, O rescaled) above the even tile's before it.
+    B, H, G, qs, n, d, k, ng = 2, 8, 7, 32, 8192, 128, 2048, 32
+    gen = torch.Generator(device="cpu").manual_seed(11)
+    u = torch.randn(B, H, d, generator=gen, dtype=torch.float64)
+    u = u / u.norm(dim=-1, keepdim=True)
+    Q = torch.randn(B, H * G, qs, d, generator=gen, dtype=torch.float64)
+    Q = Q + 4.0 * u.repeat_interleave(G, dim=1)[:, :, None, :]
+    K = torch.randn(B, H, n, d, generator=gen, dtype=torch.float64)
+    V = torch.randn(B, H, n, d, generator=gen, dtype=torch.float64)
+    Kg = torch.randn(B, H, ng, d, generator=gen, dtype=torch.float64)
+    Vg = torch.randn(B, H, ng, d, generator=gen, dtype=torch.float64)
+    idx = torch.stack([torch.randperm(n, generator=gen)[:k].sort().values for _ in range(B * H)])
+    amp = torch.zeros(k, dtype=torch.float64)
+    tile = torch.arange(k) // 128
+    amp[tile % 4 == 1] = 10.0
+    amp[tile % 4 == 3] = 40.0
+    for un in range(B * H):
+        b, h = divmod(un, H)
+        K[b, h, idx[un]] += amp[:, None] * u[b, h][None, :]
+    bf = lambda t: t.to(torch.bfloat16).cuda().contiguous()
+    Qd, Kd, Vd, Kgd, Vgd = bf(Q), bf(K), bf(V), bf(Kg), bf(Vg)
+    idx_d = idx.to(torch.int32).cuda()
+    O = torch.empty_like(Qd)
+    ws = torch.zeros(wf.wf_attn_workspace_bytes(Qd, k, ng), dtype=torch.uint8, device="cuda")
+    wf.wf_sparse_attn(Qd, Kd, Vd, idx_d, k, Kgd, Vgd, O, ws)
+    wf.wf_workspace_status(ws)
+    torch.cuda.synchronize()
+    for un in range(B * H):
+        b, h = divmod(un, H)
+        Qh = f64(Qd[b, h * G:(h + 1) * G])
+        want = oracle.sparse_attn_gqa(Qh, f64(Kd[b, h]), f64(Vd[b, h]), idx[un].numpy(), f64(Kgd[b, h]),
+                                      f64(Vgd[b, h]))
+        assert_close_out(f64(O[b, h * G:(h + 1) * G]), want, torch.bfloat16)
