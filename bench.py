@@ -598,7 +598,7 @@ def main():
     kname = "wf_fused_kernel" if fused_eligible(w) else (
         ("approx_kernel + wf_fused_kernel (one launch per scale)" if fused_shape(w) else
          "per-stage kernels (approx/score/weights/select/attn)") if WAVELET else
-        "wf_gqa_filter_kernel + tc_attn_kernel + attn_combine_kernel" if grouped_fused(w) else
+        "wf_gqa_filter_kernel + tc_attn_rows_kernel + attn_combine_kernel" if grouped_fused(w) else
         "per-stage kernels (score/weights/select/attn)")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                 "frac_of_nominal_7900": achieved / 7900.0,
