@@ -369,7 +369,6 @@ namespace {
 
 using namespace sm100;
 
-
 struct TcAttnArgs {
   const bf16* Q;
   int64_t qsb, qsh, qss;
@@ -382,8 +381,8 @@ struct TcAttnArgs {
   const int32_t* idx;
   int n, k, ng, q, G, qs, H;  // q = G qs query rows per key unit; H key heads
   float rqs;                  // 1 / qs
-  int cb;                     // query columns per CTA block (blockIdx.z = block)
-  int nq;                     // MMA columns of a block (its query rows rounded up to 32)
+  int cb;                     // query rows of a CTA's column block (all of the unit's: the grid has one block)
+  int nq;                     // query rows padded: to 32 (keys-on-lanes kernel) or to M tiles of 128 (rows kernel)
   uint32_t tcols;
   int nsplit;
   int tps;                    // key tiles of 128 a split (a CTA), taken one after the other
@@ -684,7 +683,6 @@ __global__ void __launch_bounds__(NTH, 2) tc_attn_kernel(const __grid_constant__
     tmem_dealloc(*tbase, a.tcols);
   }
 }
-
 
 // The same attention with the query rows on the TMEM lanes, for key units of
 // more than 32 query rows (grouped heads): S = Q K^T per M tile of 128 query
