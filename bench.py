@@ -445,6 +445,18 @@ def run_gpu(args, cfg, rank, world, device):
                 layers=len(layers))
 
 
+def kernel_name(w):
+    """The kernels a step of workload w runs (the roofline's "kernel")."""
+    if fused_eligible(w):
+        return "wf_fused_kernel"
+    if WAVELET:
+        return ("approx_kernel + wf_fused_kernel (one launch per scale)" if fused_shape(w) else
+                "per-stage kernels (approx/score/weights/select/attn)")
+    if grouped_fused(w):
+        return "wf_gqa_filter_kernel + tc_attn_rows_kernel + attn_combine_kernel"
+    return "per-stage kernels (score/weights/select/attn)"
+
+
 def measure_extra(args, cfg, device, hbm_peak, peak_kind):
     """A second workload measured in the same process: 10 warm-up steps, 50
     timed steps (L2 flushed before each), median and mean step time, the
@@ -464,7 +476,7 @@ def measure_extra(args, cfg, device, hbm_peak, peak_kind):
                          "unit": "GB/s", "frac": bytes_launch / (med_us * 1e-6) / 1e9 / hbm_peak,
                          "frac_of_mean": bytes_launch / (mean_us * 1e-6) / 1e9 / hbm_peak,
                          "traffic": recorded_traffic(w) if fused_eligible(w) else None,
-                         "kernel": "wf_fused_kernel" if fused_eligible(w) else "per-stage kernels",
+                         "kernel": kernel_name(w),
                          "peak_kind": peak_kind, "bytes_per_launch": bytes_launch},
             "clocks": r["clocks"]}
 
@@ -494,7 +506,7 @@ def main():
                          "--update-rows rows per unit against a full pyramid rebuild")
     ap.add_argument("--update-rows", type=int, default=32)
     ap.add_argument("--no-extra", action="store_true",
-                    help="skip the second workload (c4) that the default single-GPU run also measures")
+                    help="skip the other workloads (c4, g1) that the default single-GPU run also measures")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -595,11 +607,7 @@ def main():
     achieved = ub["step"] * w.units / (per_layer_ms * 1e-3) / 1e9
     if w.refresh_every:
         achieved = step_bytes / w.layers / (per_layer_ms * 1e-3) / 1e9
-    kname = "wf_fused_kernel" if fused_eligible(w) else (
-        ("approx_kernel + wf_fused_kernel (one launch per scale)" if fused_shape(w) else
-         "per-stage kernels (approx/score/weights/select/attn)") if WAVELET else
-        "wf_gqa_filter_kernel + tc_attn_rows_kernel + attn_combine_kernel" if grouped_fused(w) else
-        "per-stage kernels (score/weights/select/attn)")
+    kname = kernel_name(w)
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                 "frac_of_nominal_7900": achieved / 7900.0,
                 "traffic": recorded_traffic(w) if fused_eligible(w) else None, "kernel": kname,
@@ -622,6 +630,7 @@ def main():
     if world == 1 and cfg == DEFAULT_WORKLOAD and not args.no_extra and not (args.batch or args.heads) and \
             not args.wavelet and args.schedule == "default" and not args.graph:
         line["c4"] = measure_extra(args, "c4", device, hbm_peak, peak_kind)
+        line["g1"] = measure_extra(args, "g1", device, hbm_peak, peak_kind)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         units, secs = oracle_units_seconds(w, cfg, args.cpu_seconds)
         line["cpu_baseline"] = {"value": units * ub["step"] / secs / 1e9, "unit": "GB/s", "cores": 1,
